@@ -1,0 +1,283 @@
+"""SAKI oracle: a plain, slow, fp64 CPU restatement of the paper's definitions.
+
+TEST INFRASTRUCTURE.  Only the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline / reference legs of ``bench.py`` may import this module.  It shares
+no code with the CUDA library and imports nothing from it; its inputs are the
+seeded arrays of the synthetic generator (or values the paper prints).
+
+What it follows (sections and equations of arXiv 2608.03228, "SAKI"):
+
+* Sec. 3 (Setup): scores ``s_ij = q_i^T A_h k_j``; GQA query head ``h`` reads
+  KV group ``g(h) = floor(h / (Hq/Hk))`` (the paper names GQA without a
+  mapping; this is the usual repeat-kv convention).
+* Eq. (1): score distortion ``L(P) = tr[A(I-P) Sk (I-P)^T A^T Sq]``; with the
+  rank-r score map ``M = A P`` this is ``|| Sq^{1/2} (A - M) Sk^{1/2} ||_F^2``.
+* Prop. 1, Eq. (3) and App. A: ``C = Sq^{1/2} A Sk^{1/2}``, truncated SVD
+  ``C_r = U_r Lambda_r V_r^T``, optimum ``M_r = Sq^{-1/2} C_r Sk^{-1/2}`` with
+  ``L(M_r) = sum_{i>r} lambda_i(C)^2``; singular covariances use pseudoinverse
+  roots, eigenvalues below ``1e-6 * lambda_max`` are treated as zero.
+* Sec. 5 (SAKI): ``Sq`` uncentered second moment of queries, ``Sk`` and ``mu``
+  from centered keys (uncentered keys are the ``mu = 0`` case, App. A
+  "Centering"); factors ``B_q = Sq^{-1/2} U_r Lambda_r^{1/2}`` (called ``L``
+  here) and ``B_k = Sk^{-1/2} V_r Lambda_r^{1/2}`` (called ``R``); key code
+  ``c_j = R^T (k_j - mu)``; score ``s_hat = (L^T q)^T c_j + q^T A mu``.
+* Sec. 3 protocol: recall of the true top-k attended positions, i.e. the
+  fraction of the exact top-k set (by ``q^T A k``) found by the index.
+
+Readings where the paper is silent (each also listed in the design doc):
+
+* lambda_i(C) in Eq. (3) are the singular values of the (non-symmetric) C.
+* Moments are normalised by 1/n.
+* The eigenvalue floor is a pseudo-inverse: floored eigenvalues are zero in
+  both the root and the inverse root.
+* Signs of singular vectors are arbitrary; ``canonical_signs`` flips each
+  column pair (L[:, c], R[:, c]) so that the largest-magnitude entry of
+  R[:, c] is positive.
+* Ranking: descending score, equal scores broken by the lower key index.
+* Sketch storage: codes are rounded to the sketch dtype (round-to-nearest-even)
+  because that is what an index stores; query projections ``u = L^T q`` are
+  kept exact.
+* The mean term ``q^T A mu`` is a per-query constant: it is added to reported
+  scores but cannot change a ranking, so ranking uses ``u . c`` alone.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+F64 = np.float64
+
+
+# --------------------------------------------------------------------------
+# Sec. 5: calibration moments
+# --------------------------------------------------------------------------
+def moments(X, center: bool):
+    """Second moment of the rows of X [n][d]: ``(1/n) sum_t x_t x_t^T``.
+
+    ``center=True`` returns the covariance of the centered rows and their mean
+    (keys, Sec. 5 / App. A "Centering"); ``center=False`` the uncentered second
+    moment and a zero mean (queries, and the ``mu = 0`` special case)."""
+    X = np.asarray(X, F64)
+    n = X.shape[0]
+    mu = X.mean(axis=0) if center else np.zeros(X.shape[1])
+    Xc = X - mu
+    return (Xc.T @ Xc) / n, mu
+
+
+# --------------------------------------------------------------------------
+# Prop. 1 / App. A: roots of the covariances with the eigenvalue floor
+# --------------------------------------------------------------------------
+def psd_roots(S, floor_rel: float = 1e-6):
+    """Symmetric root ``S^{1/2}`` and pseudo-inverse root ``S^{+1/2}``.
+
+    Eigenvalues below ``floor_rel * lambda_max`` count as zero in both (App. A,
+    "Singular covariances")."""
+    S = np.asarray(S, F64)
+    lam, U = np.linalg.eigh(0.5 * (S + S.T))
+    lmax = lam.max() if lam.size else 0.0
+    keep = (lam > 0) & (lam >= floor_rel * lmax)
+    Uk, lk = U[:, keep], lam[keep]
+    root = (Uk * np.sqrt(lk)) @ Uk.T
+    iroot = (Uk / np.sqrt(lk)) @ Uk.T
+    return root, iroot
+
+
+def canonical_signs(L, R):
+    """Flip column pairs so that each R column's largest-|.| entry is positive."""
+    L = L.copy()
+    R = R.copy()
+    for c in range(R.shape[1]):
+        i = int(np.argmax(np.abs(R[:, c])))
+        if R[i, c] < 0:
+            R[:, c] = -R[:, c]
+            L[:, c] = -L[:, c]
+    return L, R
+
+
+def fit_head(Sq, Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
+    """Prop. 1 (Eq. 3) and the Sec. 5 factors for one head.
+
+    Returns L = B_q [d][r], R = B_k [d][r], the score map M_r = L R^T, the
+    singular values of C (all d, descending) and the optimum
+    ``loss = sum_{i>r} sigma_i^2``."""
+    A = np.asarray(A, F64)
+    rq, iq = psd_roots(Sq, floor_rel)
+    rk, ik = psd_roots(Sk, floor_rel)
+    C = rq @ A @ rk
+    U, sig, Vt = np.linalg.svd(C)
+    V = Vt.T
+    sh = np.sqrt(sig[:r])
+    L = iq @ (U[:, :r] * sh)
+    R = ik @ (V[:, :r] * sh)
+    L, R = canonical_signs(L, R)
+    M = iq @ (U[:, :r] * sig[:r]) @ V[:, :r].T @ ik
+    return dict(L=L, R=R, M=M, sigma=sig, loss=float(np.sum(sig[r:] ** 2)), C=C)
+
+
+def score_loss(M, A, Sq, Sk) -> float:
+    """Eq. (1) written directly: ``tr[(A - M) Sk (A - M)^T Sq]``."""
+    E = np.asarray(A, F64) - np.asarray(M, F64)
+    return float(np.trace(E @ np.asarray(Sk, F64) @ E.T @ np.asarray(Sq, F64)))
+
+
+def fit(q_calib, k_calib, A, rank: int, center: bool, floor_rel: float = 1e-6) -> dict:
+    """All heads: q_calib [Hq][n][d], k_calib [Hk][n][d], A [Hq][d][d].
+
+    Returns L, R [Hq][d][r]; M [Hq][d][d]; mu [Hk][d]; nu = A_h mu_g [Hq][d];
+    sigma [Hq][d]; loss [Hq]; Sq [Hq][d][d]; Sk [Hk][d][d]."""
+    Hq, Hk = len(q_calib), len(k_calib)
+    G = Hq // Hk
+    Sk, mu = zip(*[moments(k_calib[g], center) for g in range(Hk)])
+    Sq = [moments(q_calib[h], False)[0] for h in range(Hq)]
+    out = {k: [] for k in ("L", "R", "M", "sigma", "loss", "nu")}
+    for h in range(Hq):
+        g = h // G
+        res = fit_head(Sq[h], Sk[g], A[h], rank, floor_rel)
+        for k in ("L", "R", "M", "sigma", "loss"):
+            out[k].append(res[k])
+        out["nu"].append(np.asarray(A[h], F64) @ mu[g])
+    res = {k: np.array(v) for k, v in out.items()}
+    res.update(mu=np.array(mu), Sq=np.array(Sq), Sk=np.array(Sk))
+    return res
+
+
+# --------------------------------------------------------------------------
+# Sec. 5: key codes (the index)
+# --------------------------------------------------------------------------
+def round_bf16(x):
+    """Round fp64 values to the bf16 grid, nearest with ties to even.
+
+    bf16 keeps 8 significant bits and the fp32 exponent range; below 2^-126
+    its spacing is the fixed subnormal step 2^-133.  Magnitudes beyond the
+    largest finite bf16 are not produced by this workload and raise."""
+    x = np.asarray(x, F64)
+    m, e = np.frexp(x)                         # x = m 2^e, 0.5 <= |m| < 1
+    out = np.ldexp(np.rint(m * 256.0), e - 8)
+    small = np.abs(x) < 2.0 ** -126
+    out[small] = np.rint(x[small] * 2.0 ** 133) * 2.0 ** -133
+    if np.any(np.abs(out) > 3.3895313892515355e38):
+        raise OverflowError("value outside the bf16 range")
+    return out
+
+
+def round_to(dtype: str, x):
+    """Storage rounding of an index entry: 'f32' (IEEE round-to-nearest-even)
+    or 'bf16' (:func:`round_bf16`)."""
+    if dtype == "f32":
+        return np.asarray(x, F64).astype(np.float32).astype(F64)
+    if dtype == "bf16":
+        return round_bf16(x)
+    raise ValueError(dtype)
+
+
+def build_index(K, R, mu, dtype: str, group: int):
+    """Key codes ``c_j = R_h^T (k_j - mu_g)`` for every query head h (Sec. 5).
+
+    K [Hk][N][d]; R [Hq][d][r]; mu [Hk][d] or None.  Returns [Hq][N][r] rounded
+    to the index dtype."""
+    K = np.asarray(K, F64)
+    Hq = R.shape[0]
+    out = []
+    for h in range(Hq):
+        g = h // group
+        kc = K[g] - (0.0 if mu is None else np.asarray(mu[g], F64))
+        out.append(round_to(dtype, kc @ np.asarray(R[h], F64)))
+    return np.array(out)
+
+
+# --------------------------------------------------------------------------
+# Selection: approximate and exact scores, top-k, recall
+# --------------------------------------------------------------------------
+def approx_scores(q, L, sketch):
+    """``s_hat_j = (L^T q)^T c_j`` for every code row of ``sketch`` (Sec. 5)."""
+    u = np.asarray(L, F64).T @ np.asarray(q, F64)
+    return np.asarray(sketch, F64) @ u
+
+
+def exact_scores(q, A, K):
+    """``s_j = q^T A k_j`` for every key row of ``K`` (Sec. 3)."""
+    return np.asarray(K, F64) @ (np.asarray(A, F64).T @ np.asarray(q, F64))
+
+
+def topk(scores, k: int):
+    """Indices of the k largest scores, descending, equal scores by lower index.
+
+    Returns (idx [k] int64 padded with -1, values [k] padded with -inf)."""
+    s = np.asarray(scores, F64)
+    n = s.shape[0]
+    order = np.lexsort((np.arange(n), -s))[:k]
+    idx = np.full(k, -1, np.int64)
+    val = np.full(k, -np.inf)
+    idx[:len(order)] = order
+    val[:len(order)] = s[order]
+    return idx, val
+
+
+def score_topk(Q, L, sketch, seq_offsets, q_seq, q_visible, k: int, nu=None,
+               heads=None, rows=None):
+    """Per (head, query): top-k of ``u . c_j`` over the query's visible prefix of
+    its own sequence.  Q [Hq][T][d]; L [Hq][d][r]; sketch [Hq][Ntot][r].
+
+    ``heads``/``rows`` restrict the work to a sample.  Returns (idx, scores)
+    with idx seq-local int64 [len(heads)][len(rows)][k] (-1 pad) and scores
+    including the ``q^T nu`` term when ``nu`` is given."""
+    Hq, T = Q.shape[0], Q.shape[1]
+    heads = range(Hq) if heads is None else heads
+    rows = range(T) if rows is None else rows
+    I = np.full((len(heads), len(rows), k), -1, np.int64)
+    S = np.full((len(heads), len(rows), k), -np.inf)
+    for a, h in enumerate(heads):
+        for b, t in enumerate(rows):
+            base = int(seq_offsets[q_seq[t]])
+            vis = int(q_visible[t])
+            s = approx_scores(Q[h, t], L[h], sketch[h, base:base + vis])
+            idx, val = topk(s, k)
+            I[a, b] = idx
+            if nu is not None:
+                val = val + float(np.asarray(Q[h, t], F64) @ np.asarray(nu[h], F64))
+            S[a, b] = val
+    return I, S
+
+
+def exact_topk(Q, A, K, seq_offsets, q_seq, q_visible, k: int, group: int,
+               heads=None, rows=None):
+    """Exact top-k by ``q^T A k`` (the recall reference of Sec. 3)."""
+    Hq, T = Q.shape[0], Q.shape[1]
+    heads = range(Hq) if heads is None else heads
+    rows = range(T) if rows is None else rows
+    I = np.full((len(heads), len(rows), k), -1, np.int64)
+    S = np.full((len(heads), len(rows), k), -np.inf)
+    for a, h in enumerate(heads):
+        g = h // group
+        for b, t in enumerate(rows):
+            base = int(seq_offsets[q_seq[t]])
+            vis = int(q_visible[t])
+            s = exact_scores(Q[h, t], A[h], K[g, base:base + vis])
+            I[a, b], S[a, b] = topk(s, k)
+    return I, S
+
+
+def recall_rows(idx_approx, idx_exact, q_visible, min_visible: int, k: int):
+    """Per-row recall ``|S_hat & S| / k`` (Sec. 3 protocol); NaN for rows with
+    fewer than ``min_visible`` visible keys.  Inputs [rows][k]."""
+    out = np.full(len(idx_approx), np.nan)
+    for t in range(len(idx_approx)):
+        if q_visible[t] < min_visible:
+            continue
+        a = set(int(i) for i in idx_approx[t] if i >= 0)
+        e = set(int(i) for i in idx_exact[t] if i >= 0)
+        out[t] = len(a & e) / k
+    return out
+
+
+def head_recall(idx_approx, idx_exact, q_visible, min_visible: int, k: int):
+    """Mean recall per head over qualifying rows; inputs [H][rows][k]."""
+    res = []
+    for h in range(len(idx_approx)):
+        r = recall_rows(idx_approx[h], idx_exact[h], q_visible, min_visible, k)
+        res.append(np.nanmean(r) if np.any(~np.isnan(r)) else np.nan)
+    return np.array(res)
+
+
+def median_over_heads(recall):
+    """Median across heads (Tab. 1 reports medians over all heads)."""
+    return float(np.median(np.asarray(recall, F64)))

@@ -1,0 +1,313 @@
+"""Pins for the CPU oracle: each test checks it against something other than
+itself -- a hand-derived closed form, a textbook special case, an inequality
+the paper proves, an independent construction, or brute force."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import saki_oracle as O
+from paper_2608_03228_gb300 import synth
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _gold(name):
+    with open(os.path.join(GOLD, name)) as f:
+        return json.load(f)
+
+
+def _case(d=16, s=3, seed=0, n=None):
+    """Small seeded (Sq, Sk, A) from the generator recipe (population moments
+    when n is None, sample moments of n draws otherwise)."""
+    w = synth.Workload("pin", 1, 1, head_dim=d, spikes=(s, s), seed=seed)
+    f = synth.head_factors(w)
+    if n is None:
+        Sq = f.Fq[0] @ f.Fq[0].T
+        Sk = f.Fk[0] @ f.Fk[0].T
+    else:
+        rng = np.random.default_rng(seed + 100)
+        Xq = rng.standard_normal((n, d)) @ f.Fq[0].T
+        Xk = rng.standard_normal((n, d)) @ f.Fk[0].T
+        Sq, Sk = Xq.T @ Xq / n, Xk.T @ Xk / n
+    return Sq, Sk, f.A[0].astype(np.float64)
+
+
+# ---------------------------------------------------------------- closed forms
+@pytest.mark.parametrize("name", ["eckart_young_golden_ratio", "query_weighting_beats_key_pca",
+                                  "weight_svd_is_blind_to_data"])
+def test_hand_examples(name):
+    g = _gold("hand_examples.json")[name]
+    res = O.fit_head(np.array(g["Sq"]), np.array(g["Sk"]), np.array(g["A"]), g["r"])
+    np.testing.assert_allclose(res["sigma"], g["sigma"], rtol=1e-12, atol=1e-12)
+    assert abs(res["loss"] - g["loss"]) < 1e-12
+    np.testing.assert_allclose(res["M"], g["M"], rtol=1e-12, atol=1e-12)
+    if "L" in g:
+        np.testing.assert_allclose(res["L"], g["L"], atol=1e-12)
+        np.testing.assert_allclose(res["R"], g["R"], atol=1e-12)
+    if "M_squared_over_M" in g:
+        M = res["M"]
+        np.testing.assert_allclose(M @ M, g["M_squared_over_M"] * M, atol=1e-12)
+    if "pca_loss" in g:
+        lam, V = np.linalg.eigh(np.array(g["Sk"]))
+        P = np.outer(V[:, -1], V[:, -1])
+        assert abs(O.score_loss(np.array(g["A"]) @ P, g["A"], g["Sq"], g["Sk"]) - g["pca_loss"]) < 1e-12
+    if "weight_svd_loss" in g:
+        U, s, Vt = np.linalg.svd(np.array(g["A"]))
+        W = s[0] * np.outer(U[:, 0], Vt[0])
+        assert abs(O.score_loss(W, g["A"], g["Sq"], g["Sk"]) - g["weight_svd_loss"]) < 1e-12
+
+
+# ------------------------------------------------------- Prop. 1 identities
+@pytest.mark.parametrize("r", [1, 4, 8, 15])
+@pytest.mark.parametrize("seed", [0, 1])
+def test_optimum_equals_discarded_singular_energy(r, seed):
+    """Prop. 1: L(M_r) computed from Eq. (1) directly = sum_{i>r} sigma_i^2."""
+    Sq, Sk, A = _case(seed=seed)
+    res = O.fit_head(Sq, Sk, A, r)
+    direct = O.score_loss(res["M"], A, Sq, Sk)
+    assert abs(direct - res["loss"]) <= 1e-10 * max(1.0, res["loss"])
+    # the total energy is ||C||_F^2 = L(0)
+    assert abs(O.score_loss(0 * A, A, Sq, Sk) - np.sum(res["sigma"] ** 2)) <= 1e-9 * np.sum(res["sigma"] ** 2)
+
+
+def test_full_rank_reproduces_A():
+    Sq, Sk, A = _case(d=24, seed=3)
+    res = O.fit_head(Sq, Sk, A, 24)
+    np.testing.assert_allclose(res["M"], A, atol=1e-10 * np.abs(A).max())
+    assert res["loss"] < 1e-20
+
+
+@pytest.mark.parametrize("r", [1, 5, 11])
+def test_map_has_rank_r(r):
+    Sq, Sk, A = _case(seed=4)
+    s = np.linalg.svd(O.fit_head(Sq, Sk, A, r)["M"], compute_uv=False)
+    assert s[r - 1] / s[0] > 1e-8
+    assert s[r] / s[0] < 1e-12
+
+
+@pytest.mark.parametrize("r", [1, 2, 4, 8, 12])
+def test_saki_never_loses_to_key_pca_or_weight_svd(r):
+    """Remark 1: projector-based maps (key PCA) and operator-only truncation
+    are rank-r maps too, so the exact optimum can only be better."""
+    for seed in range(3):
+        Sq, Sk, A = _case(seed=seed)
+        res = O.fit_head(Sq, Sk, A, r)
+        lam, V = np.linalg.eigh(Sk)
+        Vr = V[:, ::-1][:, :r]
+        pca = O.score_loss(A @ Vr @ Vr.T, A, Sq, Sk)
+        U, s, Vt = np.linalg.svd(A)
+        wsvd = O.score_loss((U[:, :r] * s[:r]) @ Vt[:r], A, Sq, Sk)
+        assert res["loss"] <= pca * (1 + 1e-12)
+        assert res["loss"] <= wsvd * (1 + 1e-12)
+
+
+def test_identity_covariances_reduce_to_eckart_young():
+    _, _, A = _case(seed=5)
+    I = np.eye(A.shape[0])
+    res = O.fit_head(I, I, A, 6)
+    U, s, Vt = np.linalg.svd(A)
+    np.testing.assert_allclose(res["M"], (U[:, :6] * s[:6]) @ Vt[:6], atol=1e-12)
+
+
+def test_identity_operator_with_equal_moments_is_pca_projector():
+    Sq, _, _ = _case(seed=6)
+    d = Sq.shape[0]
+    res = O.fit_head(Sq, Sq, np.eye(d), 5)
+    lam, V = np.linalg.eigh(Sq)
+    Vr = V[:, ::-1][:, :5]
+    np.testing.assert_allclose(res["M"], Vr @ Vr.T, atol=1e-10)
+
+
+def test_cholesky_roots_give_the_same_map():
+    """Any F with F F^T = S gives ||F_q^T X F_k||_F^2 = tr(X^T Sq X Sk), so the
+    optimum built from Cholesky factors must equal the symmetric-root one."""
+    Sq, Sk, A = _case(seed=7, n=400)
+    r = 6
+    Lq, Lk = np.linalg.cholesky(Sq), np.linalg.cholesky(Sk)
+    U, s, Vt = np.linalg.svd(Lq.T @ A @ Lk)
+    Mc = np.linalg.solve(Lq.T, (U[:, :r] * s[:r]) @ Vt[:r]) @ np.linalg.inv(Lk)
+    res = O.fit_head(Sq, Sk, A, r)
+    np.testing.assert_allclose(res["M"], Mc, atol=1e-9 * np.abs(Mc).max())
+    np.testing.assert_allclose(res["sigma"], s, rtol=1e-10)
+
+
+def test_scaling_moments_leaves_the_map_unchanged():
+    Sq, Sk, A = _case(seed=8)
+    a = O.fit_head(Sq, Sk, A, 4)["M"]
+    b = O.fit_head(3.7 * Sq, 0.21 * Sk, A, 4)["M"]
+    np.testing.assert_allclose(a, b, atol=1e-10 * np.abs(a).max())
+
+
+def test_local_optimality_under_rank_r_perturbations():
+    Sq, Sk, A = _case(seed=9)
+    r = 5
+    res = O.fit_head(Sq, Sk, A, r)
+    rng = np.random.default_rng(0)
+    for _ in range(40):
+        X = rng.standard_normal(res["L"].shape)
+        Y = rng.standard_normal(res["R"].shape)
+        for eps in (1e-3, 1e-1):
+            M = (res["L"] + eps * X) @ (res["R"] + eps * Y).T
+            assert O.score_loss(M, A, Sq, Sk) >= res["loss"] * (1 - 1e-12)
+    # random rank-r maps are much worse
+    for _ in range(10):
+        M = rng.standard_normal((16, r)) @ rng.standard_normal((r, 16))
+        assert O.score_loss(M, A, Sq, Sk) > res["loss"]
+
+
+def test_factorisation_identity_and_non_idempotence():
+    """App. A: (L^T q).(R^T k) = q^T M_r k with M_r = Sq^-1/2 C_r Sk^-1/2; Remark 1."""
+    Sq, Sk, A = _case(seed=10)
+    r = 4
+    res = O.fit_head(Sq, Sk, A, r)
+    rng = np.random.default_rng(1)
+    for _ in range(5):
+        q, k = rng.standard_normal(16), rng.standard_normal(16)
+        assert abs((res["L"].T @ q) @ (res["R"].T @ k) - q @ res["M"] @ k) < 1e-10
+    M = res["M"]
+    assert np.linalg.norm(M @ M - M) > 0.1 * np.linalg.norm(M)
+
+
+def test_singular_covariances_match_the_restricted_problem():
+    """App. A 'Singular covariances': with n < d the covariances are rank n; the
+    optimum is the full-rank solution on range(Sq) x range(Sk), zero outside."""
+    d, n, r = 16, 9, 4
+    rng = np.random.default_rng(2)
+    Xq = rng.standard_normal((n, d))
+    Xk = rng.standard_normal((n, d)) * np.linspace(3, 0.5, d)
+    _, _, A = _case(seed=11)
+    Sq, Sk = Xq.T @ Xq / n, Xk.T @ Xk / n
+    res = O.fit_head(Sq, Sk, A, r)
+    Bq, _ = np.linalg.qr(Xq.T)          # orthonormal bases of the ranges
+    Bk, _ = np.linalg.qr(Xk.T)
+    Sqr, Skr = Bq.T @ Sq @ Bq, Bk.T @ Sk @ Bk
+    Lq, Lk = np.linalg.cholesky(Sqr), np.linalg.cholesky(Skr)
+    U, s, Vt = np.linalg.svd(Lq.T @ (Bq.T @ A @ Bk) @ Lk)
+    X = np.linalg.solve(Lq.T, (U[:, :r] * s[:r]) @ Vt[:r]) @ np.linalg.inv(Lk)
+    M_ref = Bq @ X @ Bk.T
+    np.testing.assert_allclose(res["M"], M_ref, atol=1e-8 * np.abs(M_ref).max())
+    assert abs(O.score_loss(res["M"], A, Sq, Sk) - res["loss"]) < 1e-9 * max(res["loss"], 1)
+
+
+# ------------------------------------------------------------ moments, rounding
+def test_moments_match_numpy_cov():
+    rng = np.random.default_rng(3)
+    X = rng.standard_normal((300, 7)) + np.arange(7)
+    S, mu = O.moments(X, center=True)
+    np.testing.assert_allclose(S, np.cov(X.T, bias=True), atol=1e-12)
+    np.testing.assert_allclose(mu, np.average(X, axis=0), atol=1e-12)
+    S0, mu0 = O.moments(X, center=False)
+    ref = sum(np.outer(x, x) for x in X) / len(X)
+    np.testing.assert_allclose(S0, ref, atol=1e-12)
+    assert not np.any(mu0)
+
+
+def test_bf16_rounding_golden_cases():
+    for c in _gold("bf16_rounding.json")["cases"]:
+        got = float(O.round_bf16(np.array([c["x"]]))[0])
+        assert got == c["bf16"], c
+
+
+def test_bf16_rounding_matches_torch_on_fp32_values():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(4)
+    x = np.concatenate([rng.standard_normal(20000) * 10.0 ** rng.integers(-6, 6, 20000),
+                        (1 + (2 * rng.integers(0, 128, 2000) + 1) * 2.0 ** -8)]).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.round_bf16(x.astype(np.float64)), ref)
+
+
+# ------------------------------------------------------------ selection, recall
+def test_topk_against_brute_force_with_ties():
+    rng = np.random.default_rng(5)
+    for n in (1, 5, 63, 64, 65, 200):
+        s = rng.integers(-5, 5, n).astype(float)     # many exact ties
+        for k in (1, 8, 64):
+            idx, val = O.topk(s, k)
+            ref = sorted(range(n), key=lambda j: (-s[j], j))[:k]
+            assert list(idx[:len(ref)]) == ref
+            assert np.all(idx[len(ref):] == -1) and np.all(np.isneginf(val[len(ref):]))
+            np.testing.assert_array_equal(val[:len(ref)], s[ref])
+
+
+def test_recall_golden_example():
+    g = _gold("hand_examples.json")["recall_example"]
+    rows = O.recall_rows(np.array(g["idx_approx"]), np.array(g["idx_exact"]),
+                         np.array(g["q_visible"]), g["min_visible"], g["k"])
+    for got, want in zip(rows, g["row_recall"]):
+        assert (np.isnan(got) and want is None) or got == want
+    h = O.head_recall(np.array([g["idx_approx"]]), np.array([g["idx_exact"]]),
+                      np.array(g["q_visible"]), g["min_visible"], g["k"])
+    assert h[0] == g["head_recall"]
+    assert O.median_over_heads([0.2, 0.9, 0.5, 0.7]) == 0.6
+
+
+def test_margin_condition_guarantees_exact_top_k():
+    """Prop. 2: |s - s_hat| <= eps for all j and 2 eps < gamma_k => same top-k set;
+    at 2 eps > gamma_k a perturbation exists that swaps the boundary pair."""
+    rng = np.random.default_rng(6)
+    k = 8
+    for _ in range(200):
+        s = rng.standard_normal(60)
+        srt = np.sort(s)[::-1]
+        gamma = srt[k - 1] - srt[k]
+        eps = 0.49 * gamma
+        s_hat = s + rng.uniform(-eps, eps, s.shape)
+        assert set(O.topk(s, k)[0]) == set(O.topk(s_hat, k)[0])
+    s = np.array([5.0, 4.0, 3.0, 2.9, 1.0])
+    gamma, eps = 0.1, 0.06
+    s_hat = s.copy()
+    s_hat[2] -= eps
+    s_hat[3] += eps
+    assert set(O.topk(s, 3)[0]) != set(O.topk(s_hat, 3)[0])
+
+
+# ------------------------------------------------------- index and scores
+def test_full_rank_index_reproduces_exact_scores_with_centering():
+    """r = d: codes c_j = R^T (k_j - mu) and s_hat = u.c + q^T A mu equal q^T A k."""
+    d = 16
+    Sq, Sk, A = _case(d=d, seed=12)
+    rng = np.random.default_rng(7)
+    kc = rng.standard_normal((300, d)) + 2.0
+    qc = rng.standard_normal((300, d))
+    res = O.fit(qc[None], kc[None], A[None], d, center=True)
+    K = rng.standard_normal((1, 40, d)) + 2.0
+    q = rng.standard_normal(d)
+    codes = O.build_index(K, res["R"], res["mu"], "f32", 1)
+    s_hat = O.approx_scores(q, res["L"][0], codes[0]) + q @ res["nu"][0]
+    np.testing.assert_allclose(s_hat, O.exact_scores(q, A, K[0]), rtol=2e-5, atol=2e-5)
+
+
+def test_exact_scores_by_double_loop():
+    rng = np.random.default_rng(8)
+    d = 5
+    A = rng.standard_normal((d, d))
+    K = rng.standard_normal((7, d))
+    q = rng.standard_normal(d)
+    ref = [sum(q[a] * A[a, b] * K[j, b] for a in range(d) for b in range(d)) for j in range(7)]
+    np.testing.assert_allclose(O.exact_scores(q, A, K), ref, rtol=1e-12)
+
+
+def test_predicted_mse_reduction_matches_independent_draws():
+    """Remark 2 / App. C: with independent q ~ N(0,Sq), k ~ N(0,Sk) the measured
+    score-MSE reduction equals 1 - sum_{i>r} sigma^2 / sum sigma^2 up to
+    sampling noise (E s^2 = ||C||_F^2 and E (s - s_hat)^2 = L(M_r))."""
+    w = synth.Workload("pin", 1, 1, head_dim=16, spikes=(3, 3), seed=13)
+    f = synth.head_factors(w)
+    Sq, Sk, A = f.Fq[0] @ f.Fq[0].T, f.Fk[0] @ f.Fk[0].T, f.A[0].astype(float)
+    r = 4
+    res = O.fit_head(Sq, Sk, A, r)
+    pred = 1 - res["loss"] / np.sum(res["sigma"] ** 2)
+    rng = np.random.default_rng(9)
+    n = 400000
+    q = rng.standard_normal((n, 16)) @ f.Fq[0].T
+    k = rng.standard_normal((n, 16)) @ f.Fk[0].T
+    s = np.einsum("ni,ij,nj->n", q, A, k)
+    e = s - np.einsum("ni,ij,nj->n", q, res["M"], k)
+    meas = 1 - np.mean(e ** 2) / np.mean(s ** 2)
+    # relative std of a mean of squared Gaussian bilinear forms is ~3/sqrt(n)
+    tol = 5 * 3 / math.sqrt(n) * (1 - pred + 0.05)
+    assert abs(meas - pred) < tol, (meas, pred, tol)
