@@ -1,0 +1,387 @@
+"""Throughput of the SAKI hot path on one GB300 (or N, as independent replicas).
+
+A step is one pass of the whole path over one synthetic batch of the workload:
+calibration moments + closed-form fit (saki_fit), key codes (saki_build_index),
+fused low-rank score + top-k (saki_score_topk) and exact top-k + recall
+(saki_recall).  The metric is scored keys per second: (head, query, visible key)
+triples ranked by the index per second of step time.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+`--impl reference` times the CPU oracle (the plain fp64 restatement of the
+paper) on a bounded sample of the same workload; under torchrun only rank 0
+runs it.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_03228_gb300 import synth  # noqa: E402
+
+METRIC = "scored keys/sec (head x query x key) of fused low-rank score+top-64; % HBM/tensor peak"
+UNIT = "scored keys/s"
+D = 128
+
+
+def peaks():
+    p = dict(hbm_gbs=6800.0, bf16_tflops=1900.0, bf16_tflops_sustained=1700.0, sm_max_mhz=2070.0, source="fallback")
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            m = json.load(f)
+        p.update({k: float(m[k]) for k in ("hbm_gbs", "bf16_tflops", "bf16_tflops_sustained", "sm_max_mhz") if k in m})
+        p["source"] = "measured"
+    except (OSError, ValueError, KeyError):
+        pass
+    # fp32 CUDA-core FMA peak from unit counts: 152 SMs x 128 lanes x 2 flop x max clock
+    p["fp32_tflops"] = 152 * 128 * 2 * p["sm_max_mhz"] * 1e6 / 1e12
+    return p
+
+
+def visible_pairs(w) -> int:
+    _, _, q_vis, _ = synth.seq_layout(w)
+    return int(q_vis.sum()) * w.num_q_heads
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines: list[str] = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ GPU arm
+class GpuPath:
+    """Device buffers and the four library calls of one step."""
+
+    def __init__(self, w, dev, seed_offset=0):
+        import torch
+        from paper_2608_03228_gb300 import saki
+        self.torch, self.saki, self.w, self.dev = torch, saki, w, dev
+        data = synth.make_torch(w, dev, seed_offset)
+        self.data = data
+        Hq, Hk, r, k = w.num_q_heads, w.num_kv_heads, w.rank, w.topk
+        self.cfg = saki.make_config(Hq, Hk, r, k, w.dtype, center=w.center)
+        self.lay = saki.HostLayout(data["seq_offsets"], data["q_seq"], data["q_visible"])
+        T, N = len(data["q_seq"]), self.lay.total_keys
+        dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+        f = dict(device=dev, dtype=torch.float32)
+        self.L, self.R = torch.empty((Hq, D, r), **f), torch.empty((Hq, D, r), **f)
+        self.mu, self.nu = torch.empty((Hk, D), **f), torch.empty((Hq, D), **f)
+        self.sigma, self.loss = torch.empty((Hq, D), **f), torch.empty((Hq,), **f)
+        self.sketch = torch.empty((Hq, N, r), device=dev, dtype=dt)
+        self.idx = torch.empty((Hq, T, k), device=dev, dtype=torch.int32)
+        self.idx_exact = torch.empty((Hq, T, k), device=dev, dtype=torch.int32)
+        self.recall = torch.empty((Hq,), **f)
+        S = saki
+        ws = max(S.saki_workspace_size(self.cfg, S.SAKI_OP_FIT, n_calib=w.n_calib),
+                 S.saki_workspace_size(self.cfg, S.SAKI_OP_BUILD_INDEX, total_keys=N),
+                 S.saki_workspace_size(self.cfg, S.SAKI_OP_SCORE_TOPK, self.lay),
+                 S.saki_workspace_size(self.cfg, S.SAKI_OP_RECALL, self.lay))
+        self.ws = torch.empty(ws, device=dev, dtype=torch.uint8)
+        self.T, self.N = T, N
+
+    def step(self, events=None, inputs=None):
+        S, d = self.saki, inputs or self.data
+        ev = events or [None] * 5
+        if ev[0] is not None:
+            ev[0].record()
+        S.saki_fit(self.cfg, d["q_calib"], d["k_calib"], d["A"], self.L, self.R, mu=self.mu, nu=self.nu,
+                   sigma=self.sigma, loss=self.loss, workspace=self.ws)
+        if ev[1] is not None:
+            ev[1].record()
+        S.saki_build_index(self.cfg, d["K"], self.R, self.sketch, mu=self.mu, workspace=self.ws)
+        if ev[2] is not None:
+            ev[2].record()
+        S.saki_score_topk(self.cfg, self.lay, d["Q"], self.L, self.sketch, self.idx, workspace=self.ws)
+        if ev[3] is not None:
+            ev[3].record()
+        S.saki_recall(self.cfg, self.lay, self.w.topk + 1, d["Q"], d["A"], d["K"], self.idx, self.recall,
+                      idx_exact=self.idx_exact, workspace=self.ws)
+        if ev[4] is not None:
+            ev[4].record()
+
+    def launches_per_step(self) -> int:
+        # saki_fit: moments (+ key means), factors, fit; build: 1; score: 1 (+ split merge);
+        # recall: exact top-k (+ split merge), recall, finish
+        plan_splits = 0   # configs run here plan no splits for the batched causal workloads
+        return (3 + self.w.center) + 1 + (1 + plan_splits) + (3 + plan_splits)
+
+
+def run_ours(args, w):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    g = GpuPath(w, dev, seed_offset=rank)
+    for _ in range(args.warmup):
+        g.step()
+    torch.cuda.synchronize()
+
+    nstage = 4
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nstage + 1)] for _ in range(args.steps)]
+    clocks = ClockSampler(dev.index)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for s in range(args.steps):
+        g.step(evs[s])
+    t1.record()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    ms = t0.elapsed_time(t1)
+    if dist:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    stage_ms = np.array([[evs[s][i].elapsed_time(evs[s][i + 1]) for i in range(nstage)] for s in range(args.steps)])
+    stage_ms = stage_ms.mean(axis=0)
+    pairs = visible_pairs(w)
+    ms_step = ms / args.steps
+    value = pairs * world / (ms_step / 1e3)
+
+    # end to end through the public API with host buffers (pinned), copies timed
+    e2e = run_e2e(g, args, torch)
+
+    pk = peaks()
+    names = ["fit", "build_index", "score_topk", "recall"]
+    roof = roofline(w, pk, dict(zip(names, stage_ms)), g)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if w.dtype == "bf16" else "f32",
+        "data": "synthetic: seeded spiked-covariance queries/keys and power-law non-normal score operators",
+        "config": {"workload": w.name, "query_heads": w.num_q_heads, "kv_heads": w.num_kv_heads,
+                   "layers": w.layers, "T": g.T, "N": g.N, "rank": w.rank, "topk": w.topk, "n_calib": w.n_calib,
+                   "parallelism": f"{world} independent replicas" if world > 1 else "single GPU",
+                   "l2": "inputs larger than L2 (calibration + eval tensors %.1f GB per step)" % (input_bytes(g) / 1e9)},
+        "clocks": clk, "e2e": e2e, "gpu_launches": g.launches_per_step() * args.steps,
+        "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
+        "score_topk_keys_per_s": pairs / (stage_ms[2] / 1e3),
+        "roofline": roof["dominant"], "roofline_score_topk": roof["score_topk"],
+        "recall_median": float(np.median(g.recall.cpu().numpy())),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def input_bytes(g) -> int:
+    return sum(int(g.data[k].numel() * g.data[k].element_size()) for k in ("q_calib", "k_calib", "A", "Q", "K"))
+
+
+def run_e2e(g, args, torch):
+    keys = ("q_calib", "k_calib", "A", "Q", "K")
+    host = {k: g.data[k].cpu().pin_memory() for k in keys}
+    dev = {k: torch.empty_like(g.data[k]) for k in keys}
+    out_host = torch.empty((g.w.num_q_heads,), dtype=torch.float32).pin_memory()
+    steps = max(2, min(args.steps, 5))
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        for k in keys:
+            dev[k].copy_(host[k], non_blocking=True)
+        g.step(inputs=dev)
+        out_host.copy_(g.recall, non_blocking=True)
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / steps
+    h2d = sum(int(host[k].numel() * host[k].element_size()) for k in keys)
+    return {"value": visible_pairs(g.w) / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "steps": steps,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": int(out_host.numel() * 4)}
+
+
+def roofline(w, pk, stage_ms, g):
+    pairs = visible_pairs(w)
+    N, Hq, Hk = g.N, w.num_q_heads, w.num_kv_heads
+    eb = 2 if w.dtype == "bf16" else 4
+    # score_topk on CUDA cores: 2 r flop per visible pair (fp32 FMA)
+    sc = {"kernel": "score_topk", "bound": "alu", "achieved": 2 * w.rank * pairs / (stage_ms["score_topk"] / 1e3) / 1e12,
+          "peak": pk["fp32_tflops"], "unit": "TFLOP/s", "traffic": None,
+          "note": "fp32 CUDA-core FMA peak from 152 SMs x 128 lanes x 2 x max SM clock"}
+    sc["frac"] = sc["achieved"] / sc["peak"]
+    ex = {"kernel": "recall (exact q^T A k top-k)", "bound": "alu",
+          "achieved": 2 * D * pairs / (stage_ms["recall"] / 1e3) / 1e12, "peak": pk["fp32_tflops"],
+          "unit": "TFLOP/s", "traffic": None}
+    ex["frac"] = ex["achieved"] / ex["peak"]
+    fit_flop = 2 * w.n_calib * D * D * (Hq + Hk)   # moments (the Jacobi sweeps are data-dependent)
+    ft = {"kernel": "fit (moments + Jacobi SVD)", "bound": "alu",
+          "achieved": fit_flop / (stage_ms["fit"] / 1e3) / 1e12, "peak": pk["fp32_tflops"], "unit": "TFLOP/s",
+          "traffic": None}
+    ft["frac"] = ft["achieved"] / ft["peak"]
+    bi_bytes = Hk * N * D * eb + Hq * N * w.rank * eb
+    bi = {"kernel": "build_index", "bound": "hbm", "achieved": bi_bytes / (stage_ms["build_index"] / 1e3) / 1e9,
+          "peak": pk["hbm_gbs"], "unit": "GB/s", "traffic": None}
+    bi["frac"] = bi["achieved"] / bi["peak"]
+    by_stage = {"fit": ft, "build_index": bi, "score_topk": sc, "recall": ex}
+    dom = max(stage_ms, key=lambda k: stage_ms[k])
+    for v in by_stage.values():
+        v["peak_source"] = pk["source"]
+    return {"dominant": dict(by_stage[dom], stage=dom), "score_topk": sc}
+
+
+# ------------------------------------------------------------------ CPU oracle
+def oracle_head_step(w, data, h_local):
+    """The oracle's pass over one query head of the workload: fit, codes, top-k,
+    exact top-k and recall for every query of that head."""
+    from oracle import saki_oracle as O
+    G = w.group
+    q_cal = data["q_calib"][h_local:h_local + 1]
+    k_cal = data["k_calib"][0:1]
+    res = O.fit(q_cal, k_cal, data["A"][h_local:h_local + 1], w.rank, center=bool(w.center))
+    sketch = O.build_index(data["K"][0:1], res["R"], res["mu"] if w.center else None, w.dtype, 1)
+    Q = data["Q"][h_local:h_local + 1]
+    ia, _ = O.score_topk(Q, res["L"], sketch, data["seq_offsets"], data["q_seq"], data["q_visible"], w.topk)
+    ie, _ = O.exact_topk(Q, data["A"][h_local:h_local + 1], data["K"][0:1], data["seq_offsets"], data["q_seq"],
+                         data["q_visible"], w.topk, 1)
+    return O.head_recall(ia, ie, data["q_visible"], w.topk + 1, w.topk)
+
+
+def _oracle_sample_data(w, h):
+    # one query head with its KV head, as the oracle consumes it (host fp32 values on the bf16 grid)
+    return synth.make_numpy(w, heads=(h,))
+
+
+def cpu_baseline(w, budget_s=20.0) -> dict:
+    cores = len(os.sched_getaffinity(0))
+    heads = [0, w.num_q_heads // 2 + 1, w.num_q_heads - 1]
+    _, _, q_vis, _ = synth.seq_layout(w)
+    per_head_pairs = int(q_vis.sum())
+    done, elapsed, pairs = 0, 0.0, 0
+    for h in heads:
+        data = _oracle_sample_data(w, h)
+        t = time.perf_counter()
+        oracle_head_step(w, data, 0)
+        elapsed += time.perf_counter() - t
+        pairs += per_head_pairs
+        done += 1
+        if elapsed > budget_s:
+            break
+    return {"value": pairs / elapsed, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{done} of {w.num_q_heads} query heads, every query of each (fit, codes, top-{w.topk}, "
+                      f"exact top-{w.topk}, recall); {elapsed:.1f} s; numpy fp64, BLAS threads = cores"}
+
+
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    _, _, q_vis, _ = synth.seq_layout(w)
+    per_head_pairs = int(q_vis.sum())
+    heads = [(i * 37) % w.num_q_heads for i in range(args.warmup + args.steps)]
+    cache = {}
+    times = []
+    for i, h in enumerate(heads):
+        if h not in cache:
+            cache[h] = _oracle_sample_data(w, h)
+        t = time.perf_counter()
+        oracle_head_step(w, cache[h], 0)
+        dt = time.perf_counter() - t
+        if i >= args.warmup:
+            times.append(dt)
+    ms = 1e3 * sum(times) / len(times)
+    value = per_head_pairs / (ms / 1e3)
+    cores = len(os.sched_getaffinity(0))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 0, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic (same generator as the GPU arm)",
+            "config": {"workload": w.name, "step": "one query head of the workload, every query"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": "one query head per step (fit, codes, top-k, exact top-k, recall)"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="llama31_8b_t4096_r32", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-seconds", type=float, default=20.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    w = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

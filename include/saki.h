@@ -1,0 +1,177 @@
+/*
+ * saki.h -- C ABI of the GB300 (sm_103a) SAKI score-map retrieval library.
+ *
+ * SAKI (arXiv 2608.03228) indexes a KV cache with a per-head rank-r score map.
+ * For query head h reading KV head g(h) = h / (Hq / Hk):
+ *   - fit (Prop. 1, Eq. 3; Sec. 5; App. A): from calibration moments Sq (queries,
+ *     uncentered) and Sk, mu (keys), form C = Sq^{1/2} A_h Sk^{1/2}, take its
+ *     truncated SVD C_r = U_r Lambda_r V_r^T and fold M_r = Sq^{-1/2} C_r Sk^{-1/2}
+ *     into L_h = Sq^{-1/2} U_r Lambda_r^{1/2} and R_h = Sk^{-1/2} V_r Lambda_r^{1/2};
+ *   - index (Sec. 5): key codes c_j = R_h^T (k_j - mu_g);
+ *   - select (Sec. 1, Sec. 5): s_hat_j = (L_h^T q)^T c_j over the keys a query
+ *     can see, keep the k largest;
+ *   - evaluate (Sec. 3 protocol): exact s_j = q^T A_h k_j, its top-k, recall@k.
+ *
+ * Conventions shared by every entry point
+ *   Pointers.  Tensor arguments are DEVICE pointers on the current CUDA device,
+ *     16-byte aligned, row-major with the last listed dimension fastest.  The
+ *     layout description (saki_layout) is HOST memory.  The caller owns every
+ *     buffer, including the workspace; the library keeps no state between calls
+ *     and allocates no device memory.
+ *   Streams.  Work is enqueued on `stream` (NULL = legacy default stream).
+ *     saki_fit synchronises the stream once to report numeric status;
+ *     saki_score_topk and saki_recall copy their small host-side work list into
+ *     the workspace with cudaMemcpyAsync from pageable memory, which orders
+ *     them after earlier work on the stream.  Other calls return at once.
+ *   Errors.  Arguments are checked before any launch; on SAKI_ERR_INVALID_ARGUMENT,
+ *     SAKI_ERR_UNSUPPORTED or SAKI_ERR_WORKSPACE nothing is launched and no
+ *     output is touched.  SAKI_ERR_CUDA reports a failed launch or copy (the
+ *     CUDA error is left for cudaGetLastError()).
+ *   dtype.  SAKI_F32 or SAKI_BF16 applies to queries, keys, calibration data and
+ *     key codes; A, L, R, mu, nu, sigma, loss and scores are always float32.
+ *   GQA.  Query head h uses KV head h / (num_q_heads / num_kv_heads).
+ */
+#ifndef SAKI_H_
+#define SAKI_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SAKI_API __attribute__((visibility("default")))
+#else
+#define SAKI_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* saki_stream; /* same handle as cudaStream_t */
+
+typedef enum saki_status {
+  SAKI_OK = 0,
+  SAKI_ERR_INVALID_ARGUMENT = 1, /* bad pointer, size, shape or flag */
+  SAKI_ERR_UNSUPPORTED = 2,      /* valid request outside what this build implements */
+  SAKI_ERR_CUDA = 3,             /* a CUDA launch or copy failed */
+  SAKI_ERR_NUMERIC = 4,          /* non-finite calibration data or moments */
+  SAKI_ERR_NOT_CONVERGED = 5,    /* Jacobi sweep limit reached for some head */
+  SAKI_ERR_WORKSPACE = 6,        /* workspace smaller than saki_workspace_size() */
+  SAKI_ERR_TIMEOUT = 7           /* a bounded device-side wait gave up */
+} saki_status;
+
+typedef enum saki_dtype { SAKI_F32 = 0, SAKI_BF16 = 1 } saki_dtype;
+
+/* saki_config.flags */
+#define SAKI_FLAG_SORTED 1 /* top-k lists in descending score (ties: lower index) */
+
+typedef struct saki_config {
+  int32_t num_q_heads;   /* Hq >= 1 */
+  int32_t num_kv_heads;  /* Hk >= 1, Hq % Hk == 0 */
+  int32_t head_dim;      /* d; this build supports d = 128 */
+  int32_t rank;          /* r, 1 <= r <= d */
+  int32_t topk;          /* k, 1 <= k <= 128 */
+  int32_t dtype;         /* saki_dtype */
+  int32_t center;        /* 1: centered keys (Sk centered, codes of k - mu); 0: mu = 0 */
+  float eig_floor_rel;   /* eigenvalues below eig_floor_rel * lambda_max count as zero
+                            (App. A, "Singular covariances"); the paper uses 1e-6 */
+  int32_t max_sweeps;    /* Jacobi sweep limit of the fit; 0 selects 40 */
+  int32_t flags;         /* SAKI_FLAG_* */
+} saki_config;
+
+/* Which keys each query may rank (HOST memory).  Keys of sequence s are rows
+ * seq_offsets[s] .. seq_offsets[s+1]-1 of the key / code tensors; query t belongs
+ * to sequence q_seq[t] and sees its first q_visible[t] keys (causal prefill: t+1;
+ * decode: the whole sequence).  Returned key indices are sequence-local. */
+typedef struct saki_layout {
+  int32_t num_seqs;            /* S >= 1 */
+  const int64_t* seq_offsets;  /* [S+1], non-decreasing, seq_offsets[0] == 0 */
+  int64_t num_queries;         /* T >= 0 */
+  const int32_t* q_seq;        /* [T], values in [0, S) */
+  const int64_t* q_visible;    /* [T], 0 <= q_visible[t] <= length of its sequence */
+} saki_layout;
+
+/* Operation codes for saki_workspace_size */
+#define SAKI_OP_FIT 0
+#define SAKI_OP_BUILD_INDEX 1
+#define SAKI_OP_SCORE_TOPK 2
+#define SAKI_OP_RECALL 3
+
+/* Bytes of device workspace `op` needs.  FIT uses n_calib; BUILD_INDEX uses
+ * total_keys; SCORE_TOPK and RECALL use the layout.  Returns 0 if the arguments
+ * are invalid. */
+SAKI_API size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout* layout,
+                           int64_t n_calib, int64_t total_keys);
+
+/* saki_fit -- Prop. 1 (Eq. 3), Sec. 5 and App. A: calibration moments, the exact
+ * rank-r minimiser of the score distortion of Eq. (1), folded into factors.
+ *   q_calib [Hq][n][d] dtype   calibration queries of each query head
+ *   k_calib [Hk][n][d] dtype   calibration keys of each KV head
+ *   A       [Hq][d][d] f32     score operator, s = q^T A k
+ * Outputs (float32):
+ *   L [Hq][d][r], R [Hq][d][r]  factors with L R^T = M_r; each column pair is
+ *                               signed so that the largest-|.| entry of R[:, c]
+ *                               is positive; columns follow descending sigma
+ *   mu [Hk][d]      key means (required when center = 1, may be NULL otherwise)
+ *   nu [Hq][d]      A_h mu_g, the exact mean term q^T nu (NULL = skip)
+ *   sigma [Hq][d]   singular values of C, descending (NULL = skip)
+ *   loss [Hq]       optimum sum_{i>r} sigma_i^2 (NULL = skip)
+ * Moments are normalised by 1/n.  Synchronises `stream`; returns SAKI_ERR_NUMERIC
+ * if a moment is not finite and SAKI_ERR_NOT_CONVERGED if a head's Jacobi SVD
+ * reached max_sweeps (outputs are then still written from the last sweep). */
+SAKI_API saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_calib,
+                     const void* k_calib, const float* A, float* L, float* R, float* mu,
+                     float* nu, float* sigma, float* loss, void* workspace,
+                     size_t workspace_bytes, saki_stream stream);
+
+/* saki_build_index -- Sec. 5 key codes c_j = R_h^T (k_j - mu_g) for every query
+ * head h and every key row j (all sequences at once).
+ *   K      [Hk][total_keys][d] dtype
+ *   R      [Hq][d][r] f32
+ *   mu     [Hk][d] f32, read only when center = 1 (then required)
+ *   sketch [Hq][total_keys][r] dtype, written; rounded to nearest-even. */
+SAKI_API saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const void* K,
+                             const float* R, const float* mu, void* sketch, void* workspace,
+                             size_t workspace_bytes, saki_stream stream);
+
+/* saki_score_topk -- Sec. 5 selection: per (head h, query t) the k keys of the
+ * visible prefix with the largest s_hat = (L_h^T q_t)^T c_j, never forming the
+ * T x N score matrix.
+ *   Q      [Hq][T][d] dtype      queries
+ *   L      [Hq][d][r] f32
+ *   sketch [Hq][total_keys][r] dtype, total_keys = seq_offsets[S]
+ *   nu     [Hq][d] f32 or NULL   adds q^T nu to reported scores (not to ranking)
+ *   idx    [Hq][T][k] int32      sequence-local key indices, -1 where fewer than
+ *                                k keys are visible
+ *   score  [Hq][T][k] f32 or NULL   s_hat (+ q^T nu) of each idx entry, -inf pad
+ * Ranking is by descending s_hat with equal scores ordered by the lower index.
+ * Without SAKI_FLAG_SORTED the k entries of a row come in unspecified order. */
+SAKI_API saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, const void* Q,
+                            const float* L, const void* sketch, const float* nu, int32_t* idx,
+                            float* score, void* workspace, size_t workspace_bytes,
+                            saki_stream stream);
+
+/* saki_recall -- Sec. 3 protocol: exact top-k by s = q^T A_h k over the visible
+ * keys, and recall@k = |approx set & exact set| / k averaged over the queries of
+ * each head with at least min_visible visible keys (the paper uses k + 1).
+ *   Q [Hq][T][d] dtype, A [Hq][d][d] f32, K [Hk][total_keys][d] dtype
+ *   idx_approx [Hq][T][k] int32   e.g. the output of saki_score_topk
+ *   idx_exact  [Hq][T][k] int32 or NULL (then kept in the workspace)
+ *   recall     [Hq] f32, NaN for a head with no qualifying query
+ * Medians across heads (Tab. 1) are left to the caller. */
+SAKI_API saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64_t min_visible,
+                        const void* Q, const float* A, const void* K, const int32_t* idx_approx,
+                        int32_t* idx_exact, float* recall, void* workspace,
+                        size_t workspace_bytes, saki_stream stream);
+
+/* Static description of a status code. */
+SAKI_API const char* saki_status_string(saki_status status);
+
+/* Library version as "major.minor.patch". */
+SAKI_API const char* saki_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SAKI_H_ */

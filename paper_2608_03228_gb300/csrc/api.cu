@@ -1,0 +1,329 @@
+// C-ABI entry points (include/saki.h): argument checks, workspace carving, the
+// host-side work plan of the selection kernels, and launches.  No device
+// memory is allocated here; every buffer belongs to the caller.
+#include <algorithm>
+#include <climits>
+#include <cstring>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace saki;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr int kNumSMs = 152;
+inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+inline bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline int kp_of(int k) { return k <= 64 ? 64 : 128; }
+
+saki_status check_cfg(const saki_config* c) {
+  if (!c) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->num_q_heads < 1 || c->num_kv_heads < 1 || c->num_q_heads % c->num_kv_heads) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->num_q_heads > 65535) return SAKI_ERR_UNSUPPORTED;
+  if (c->head_dim < 1) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->head_dim != kD) return SAKI_ERR_UNSUPPORTED;
+  if (c->rank < 1 || c->rank > c->head_dim) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->topk < 1) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->topk > 128) return SAKI_ERR_UNSUPPORTED;
+  if (c->dtype != SAKI_F32 && c->dtype != SAKI_BF16) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->center != 0 && c->center != 1) return SAKI_ERR_INVALID_ARGUMENT;
+  if (!(c->eig_floor_rel >= 0.f && c->eig_floor_rel < 1.f)) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->max_sweeps < 0) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->flags & ~SAKI_FLAG_SORTED) return SAKI_ERR_INVALID_ARGUMENT;
+  return SAKI_OK;
+}
+
+saki_status check_layout(const saki_layout* L, int64_t* total_keys) {
+  if (!L || L->num_seqs < 1 || !L->seq_offsets || L->num_queries < 0) return SAKI_ERR_INVALID_ARGUMENT;
+  if (L->num_queries > INT32_MAX) return SAKI_ERR_UNSUPPORTED;
+  if (L->num_queries > 0 && (!L->q_seq || !L->q_visible)) return SAKI_ERR_INVALID_ARGUMENT;
+  if (L->seq_offsets[0] != 0) return SAKI_ERR_INVALID_ARGUMENT;
+  for (int s = 0; s < L->num_seqs; ++s) {
+    const int64_t len = L->seq_offsets[s + 1] - L->seq_offsets[s];
+    if (len < 0) return SAKI_ERR_INVALID_ARGUMENT;
+    if (len > INT32_MAX - 1) return SAKI_ERR_UNSUPPORTED;
+  }
+  for (int64_t t = 0; t < L->num_queries; ++t) {
+    const int32_t s = L->q_seq[t];
+    if (s < 0 || s >= L->num_seqs) return SAKI_ERR_INVALID_ARGUMENT;
+    const int64_t v = L->q_visible[t];
+    if (v < 0 || v > L->seq_offsets[s + 1] - L->seq_offsets[s]) return SAKI_ERR_INVALID_ARGUMENT;
+  }
+  *total_keys = L->seq_offsets[L->num_seqs];
+  return SAKI_OK;
+}
+
+// ------------------------------------------------------------------ work plan
+struct Plan {
+  std::vector<ScoreItem> items;
+  std::vector<MergeItem> merges;
+  std::vector<int32_t> vis;
+  int64_t cand_slots = 0;
+  // workspace offsets (bytes)
+  size_t off_items = 0, off_merges = 0, off_vis = 0, off_cand = 0, bytes = 0, staged = 0;
+};
+
+// Groups of up to kGroupQ consecutive queries of one sequence; a group's visible
+// range is cut into splits so that the grid has several CTAs per SM.
+Plan make_plan(const saki_layout* L, int Hq, int kp) {
+  Plan p;
+  const int64_t T = L->num_queries;
+  struct G { int32_t b, n; int64_t vmax; int32_t seq; };
+  std::vector<G> groups;
+  int64_t work = 0;
+  for (int64_t t = 0; t < T;) {
+    G g{(int32_t)t, 0, 0, L->q_seq[t]};
+    while (t < T && L->q_seq[t] == g.seq && g.n < kGroupQ) {
+      g.vmax = std::max(g.vmax, L->q_visible[t]);
+      ++g.n;
+      ++t;
+    }
+    work += g.vmax;
+    groups.push_back(g);
+  }
+  const int64_t target_per_head = std::max<int64_t>(1, (int64_t)8 * kNumSMs / Hq);
+  int64_t chunk = std::max<int64_t>(2048, (work + target_per_head - 1) / target_per_head);
+  chunk = (chunk + 255) / 256 * 256;
+  for (const G& g : groups) {
+    const int64_t base = L->seq_offsets[g.seq];
+    const int32_t S = g.vmax > 0 ? (int32_t)((g.vmax + chunk - 1) / chunk) : 1;
+    if (S == 1) {
+      p.items.push_back(ScoreItem{g.b, g.n, 0, (int32_t)g.vmax, base, -1, 0, 0});
+      continue;
+    }
+    const int64_t slot0 = p.cand_slots;
+    p.cand_slots += (int64_t)g.n * S;
+    for (int32_t s = 0; s < S; ++s) {
+      const int64_t lo = s * chunk, hi = std::min<int64_t>(g.vmax, lo + chunk);
+      p.items.push_back(ScoreItem{g.b, g.n, (int32_t)lo, (int32_t)hi, base, slot0 + s, S, 0});
+    }
+    for (int32_t b = 0; b < g.n; ++b) p.merges.push_back(MergeItem{g.b + b, S, slot0 + (int64_t)b * S});
+  }
+  p.vis.resize(T);
+  for (int64_t t = 0; t < T; ++t) p.vis[t] = (int32_t)L->q_visible[t];
+  p.off_items = 0;
+  p.off_merges = align_up(p.items.size() * sizeof(ScoreItem));
+  p.off_vis = p.off_merges + align_up(p.merges.size() * sizeof(MergeItem));
+  p.staged = p.off_vis + p.vis.size() * sizeof(int32_t);
+  p.off_cand = align_up(p.staged);
+  p.bytes = p.off_cand + align_up((size_t)p.cand_slots * Hq * kp * sizeof(uint64_t));
+  return p;
+}
+
+saki_status upload_plan(const Plan& p, char* ws, cudaStream_t s) {
+  if (p.staged == 0) return SAKI_OK;
+  std::vector<char> host(p.staged, 0);
+  if (!p.items.empty()) std::memcpy(host.data() + p.off_items, p.items.data(), p.items.size() * sizeof(ScoreItem));
+  if (!p.merges.empty())
+    std::memcpy(host.data() + p.off_merges, p.merges.data(), p.merges.size() * sizeof(MergeItem));
+  if (!p.vis.empty()) std::memcpy(host.data() + p.off_vis, p.vis.data(), p.vis.size() * sizeof(int32_t));
+  return cudaMemcpyAsync(ws, host.data(), p.staged, cudaMemcpyHostToDevice, s) == cudaSuccess ? SAKI_OK
+                                                                                              : SAKI_ERR_CUDA;
+}
+
+// fit workspace: S, F, G [(Hq+Hk)][d][d], mu [Hk][d], status [Hq+Hk]
+struct FitWs { size_t S, F, G, mu, st, bytes; };
+FitWs fit_ws(const saki_config* c) {
+  const size_t nm = (size_t)c->num_q_heads + c->num_kv_heads;
+  const size_t mat = nm * kD * kD * sizeof(float);
+  FitWs w;
+  w.S = 0;
+  w.F = align_up(mat);
+  w.G = w.F + align_up(mat);
+  w.mu = w.G + align_up(mat);
+  w.st = w.mu + align_up((size_t)c->num_kv_heads * kD * sizeof(float));
+  w.bytes = w.st + align_up(nm * sizeof(int));
+  return w;
+}
+
+size_t recall_extra(const saki_config* c, int64_t T, bool with_idx) {
+  return align_up((size_t)c->num_q_heads * 2 * sizeof(unsigned long long)) +
+         (with_idx ? align_up((size_t)c->num_q_heads * T * c->topk * sizeof(int32_t)) : 0);
+}
+
+inline saki_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* saki_status_string(saki_status s) {
+  switch (s) {
+    case SAKI_OK: return "ok";
+    case SAKI_ERR_INVALID_ARGUMENT: return "invalid argument";
+    case SAKI_ERR_UNSUPPORTED: return "unsupported by this build";
+    case SAKI_ERR_CUDA: return "CUDA launch or copy failed";
+    case SAKI_ERR_NUMERIC: return "non-finite calibration data or moments";
+    case SAKI_ERR_NOT_CONVERGED: return "Jacobi SVD did not converge within max_sweeps";
+    case SAKI_ERR_WORKSPACE: return "workspace too small";
+    case SAKI_ERR_TIMEOUT: return "bounded device wait gave up";
+  }
+  return "unknown status";
+}
+
+const char* saki_version(void) { return "0.1.0"; }
+
+size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout* layout, int64_t n_calib,
+                           int64_t total_keys) {
+  if (check_cfg(cfg) != SAKI_OK) return 0;
+  switch (op) {
+    case SAKI_OP_FIT:
+      return n_calib >= 1 ? fit_ws(cfg).bytes : 0;
+    case SAKI_OP_BUILD_INDEX:
+      return total_keys >= 0 ? kAlign : 0;
+    case SAKI_OP_SCORE_TOPK:
+    case SAKI_OP_RECALL: {
+      int64_t n = 0;
+      if (check_layout(layout, &n) != SAKI_OK) return 0;
+      const Plan p = make_plan(layout, cfg->num_q_heads, kp_of(cfg->topk));
+      size_t b = p.bytes;
+      if (op == SAKI_OP_RECALL) b += recall_extra(cfg, layout->num_queries, true);
+      return b;
+    }
+  }
+  return 0;
+}
+
+saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_calib, const void* k_calib,
+                     const float* A, float* L, float* R, float* mu, float* nu, float* sigma, float* loss,
+                     void* workspace, size_t workspace_bytes, saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  if (n_calib < 1 || !q_calib || !k_calib || !A || !L || !R || !workspace) return SAKI_ERR_INVALID_ARGUMENT;
+  if (cfg->center && !mu) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {q_calib, k_calib, (const void*)A, (const void*)L, (const void*)R, (const void*)mu,
+                        (const void*)nu, (const void*)sigma, (const void*)loss, (const void*)workspace})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  const FitWs w = fit_ws(cfg);
+  if (workspace_bytes < w.bytes) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  const int Hq = cfg->num_q_heads, Hk = cfg->num_kv_heads, nm = Hq + Hk;
+  float* S = reinterpret_cast<float*>(ws + w.S);
+  float* F = reinterpret_cast<float*>(ws + w.F);
+  float* Gm = reinterpret_cast<float*>(ws + w.G);
+  float* muw = mu ? mu : reinterpret_cast<float*>(ws + w.mu);
+  int* status = reinterpret_cast<int*>(ws + w.st);
+  const int sweeps = cfg->max_sweeps > 0 ? cfg->max_sweeps : 40;
+  if ((st = cuda_status(cudaMemsetAsync(status, 0, nm * sizeof(int), s))) != SAKI_OK) return st;
+  if (!cfg->center && mu && (st = cuda_status(cudaMemsetAsync(mu, 0, (size_t)Hk * kD * sizeof(float), s))) != SAKI_OK)
+    return st;
+  if ((st = cuda_status(launch_gram(q_calib, k_calib, n_calib, Hq, Hk, cfg->center, cfg->dtype, S, muw, s))) != SAKI_OK)
+    return st;
+  if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK) return st;
+  if ((st = cuda_status(launch_fit(A, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps, L, R, sigma,
+                                   loss, nu, status, s))) != SAKI_OK)
+    return st;
+  std::vector<int> hst(nm);
+  if ((st = cuda_status(cudaMemcpyAsync(hst.data(), status, nm * sizeof(int), cudaMemcpyDeviceToHost, s))) != SAKI_OK)
+    return st;
+  if ((st = cuda_status(cudaStreamSynchronize(s))) != SAKI_OK) return st;
+  int acc = 0;
+  for (int v : hst) acc |= v;
+  if (acc & kStNonFinite) return SAKI_ERR_NUMERIC;
+  if (acc & kStNotConverged) return SAKI_ERR_NOT_CONVERGED;
+  return SAKI_OK;
+}
+
+saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const void* K, const float* R,
+                             const float* mu, void* sketch, void* workspace, size_t workspace_bytes,
+                             saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  if (total_keys < 0 || (total_keys > 0 && (!K || !R || !sketch))) return SAKI_ERR_INVALID_ARGUMENT;
+  if (cfg->center && !mu) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {K, (const void*)R, (const void*)mu, (const void*)sketch})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  (void)workspace;
+  (void)workspace_bytes;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return cuda_status(launch_build_generic(K, R, cfg->center ? mu : nullptr, sketch, total_keys, cfg->num_q_heads,
+                                          cfg->num_q_heads / cfg->num_kv_heads, cfg->rank, cfg->center,
+                                          cfg->dtype, s));
+}
+
+saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, const void* Q, const float* L,
+                            const void* sketch, const float* nu, int32_t* idx, float* score, void* workspace,
+                            size_t workspace_bytes, saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  int64_t N = 0;
+  if ((st = check_layout(layout, &N)) != SAKI_OK) return st;
+  const int64_t T = layout->num_queries;
+  if (T > 0 && (!Q || !L || !idx || !workspace || (N > 0 && !sketch))) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {Q, (const void*)L, sketch, (const void*)nu, (const void*)idx, (const void*)score,
+                        (const void*)workspace})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  if (T == 0) return SAKI_OK;
+  const int kp = kp_of(cfg->topk);
+  const Plan p = make_plan(layout, cfg->num_q_heads, kp);
+  if (workspace_bytes < p.bytes) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
+  ScoreArgs a{};
+  a.Q = Q; a.X = sketch; a.W = L; a.nu = nu;
+  a.items = reinterpret_cast<const ScoreItem*>(ws + p.off_items);
+  a.merges = reinterpret_cast<const MergeItem*>(ws + p.off_merges);
+  a.vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
+  a.idx = idx; a.score = score;
+  a.cand = reinterpret_cast<uint64_t*>(ws + p.off_cand);
+  a.cand_per_head = p.cand_slots;
+  a.T = T; a.N = N;
+  a.Hq = cfg->num_q_heads; a.G = cfg->num_q_heads / cfg->num_kv_heads; a.P = cfg->rank; a.k = cfg->topk;
+  a.exact = 0;
+  a.n_items = (int32_t)p.items.size();
+  a.n_merges = (int32_t)p.merges.size();
+  if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
+  return cuda_status(launch_merge(a, cfg->dtype, kp, s));
+}
+
+saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64_t min_visible, const void* Q,
+                        const float* A, const void* K, const int32_t* idx_approx, int32_t* idx_exact, float* recall,
+                        void* workspace, size_t workspace_bytes, saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  int64_t N = 0;
+  if ((st = check_layout(layout, &N)) != SAKI_OK) return st;
+  const int64_t T = layout->num_queries;
+  if (!recall || !workspace || (T > 0 && (!Q || !A || !idx_approx || (N > 0 && !K)))) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {Q, (const void*)A, K, (const void*)idx_approx, (const void*)idx_exact, (const void*)recall,
+                        (const void*)workspace})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  const int kp = kp_of(cfg->topk);
+  const Plan p = make_plan(layout, cfg->num_q_heads, kp);
+  const size_t need = p.bytes + recall_extra(cfg, T, idx_exact == nullptr);
+  if (workspace_bytes < need) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  unsigned long long* counters = reinterpret_cast<unsigned long long*>(ws + p.bytes);
+  int32_t* ie = idx_exact ? idx_exact
+                          : reinterpret_cast<int32_t*>(ws + p.bytes + align_up((size_t)cfg->num_q_heads * 2 *
+                                                                               sizeof(unsigned long long)));
+  if (T > 0) {
+    if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
+    ScoreArgs a{};
+    a.Q = Q; a.X = K; a.W = A; a.nu = nullptr;
+    a.items = reinterpret_cast<const ScoreItem*>(ws + p.off_items);
+    a.merges = reinterpret_cast<const MergeItem*>(ws + p.off_merges);
+    a.vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
+    a.idx = ie; a.score = nullptr;
+    a.cand = reinterpret_cast<uint64_t*>(ws + p.off_cand);
+    a.cand_per_head = p.cand_slots;
+    a.T = T; a.N = N;
+    a.Hq = cfg->num_q_heads; a.G = cfg->num_q_heads / cfg->num_kv_heads; a.P = kD; a.k = cfg->topk;
+    a.exact = 1;
+    a.n_items = (int32_t)p.items.size();
+    a.n_merges = (int32_t)p.merges.size();
+    if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
+    if ((st = cuda_status(launch_merge(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
+  }
+  const int32_t* vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
+  return cuda_status(launch_recall(idx_approx, ie, vis, T, cfg->num_q_heads, cfg->topk, min_visible, counters,
+                                   recall, s));
+}
+
+}  // extern "C"

@@ -1,0 +1,369 @@
+// The closed-form fit of Prop. 1 (Eq. 3), Sec. 5 and App. A, one CTA per matrix.
+//
+// factor_kernel: for each moment matrix S (query heads, then KV heads) a factor F
+//   with F F^T = S and G = F^{+T}.  Fast path: Cholesky S = F F^T, G = F^{-T},
+//   taken only when lambda_min(S) >= 1/||F^{-1}||_F^2 >= floor * trace(S) >=
+//   floor * lambda_max(S) proves that the eigenvalue floor of App. A drops
+//   nothing.  Otherwise the floor is applied exactly: eigenpairs of S from a
+//   one-sided Jacobi run on S (S V = V Lambda for a PSD matrix), F = V_+
+//   Lambda_+^{1/2}, G = V_+ Lambda_+^{-1/2} over the kept eigenvalues.
+//   Any factor with F F^T = S yields the same optimum, because
+//   ||F_q^T X F_k||_F^2 = tr(X^T Sq X Sk) for every X.
+//
+// fit_kernel: per query head h with KV head g,
+//   C' = Fq^T A_h Fk (singular values equal those of Sq^{1/2} A_h Sk^{1/2}),
+//   one-sided (Hestenes) Jacobi on C'^T: its columns converge to V Sigma with
+//   V the right singular vectors of C'; then
+//   R = Gk V_r Sigma_r^{1/2}  and  L = Gq (C' V_r) Sigma_r^{-1/2} = Gq U_r Sigma_r^{1/2},
+//   so L R^T = M_r, loss = sum_{i>r} sigma_i^2 and nu = A_h mu_g.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace saki {
+namespace {
+
+constexpr int kFitThreads = 512;
+
+__device__ __forceinline__ void rr_pair(int round, int k, int& pa, int& pb) {
+  // round-robin (circle) schedule of kD players: position 0 fixed, others rotate
+  auto player = [&](int p) { return p == 0 ? 0 : ((p - 1 + round) % (kD - 1)) + 1; };
+  pa = player(k);
+  pb = player(kD - 1 - k);
+}
+
+// One-sided Jacobi on the columns of X (column-major, leading dimension kLdS) until
+// every pair satisfies |x_a . x_b| <= tol ||x_a|| ||x_b||.  Needs kFitThreads
+// threads; returns true on convergence within max_sweeps.
+__device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_counter) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int sweep = 0; sweep < max_sweeps; ++sweep) {
+    if (tid == 0) *s_counter = 0;
+    __syncthreads();
+    int rot = 0;
+    for (int round = 0; round < kD - 1; ++round) {
+#pragma unroll 1
+      for (int q = 0; q < 4; ++q) {
+        int pa, pb;
+        rr_pair(round, warp * 4 + q, pa, pb);
+        float* xa = X + pa * kLdS;
+        float* xb = X + pb * kLdS;
+        float a[4], b[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) { a[u] = xa[lane + 32 * u]; b[u] = xb[lane + 32 * u]; }
+        float al = 0.f, be = 0.f, ga = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          al = fmaf(a[u], a[u], al);
+          be = fmaf(b[u], b[u], be);
+          ga = fmaf(a[u], b[u], ga);
+        }
+        al = warp_sum(al);  // xor butterflies leave identical values in every lane
+        be = warp_sum(be);
+        ga = warp_sum(ga);
+        if (ga != 0.f && fabsf(ga) > tol * sqrtf(al) * sqrtf(be)) {
+          const float zeta = (be - al) / (2.f * ga);
+          const float t = fabsf(zeta) > 1e18f ? 0.5f / zeta
+                                              : copysignf(1.f, zeta) / (fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
+          const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
+          const float s = c * t;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            xa[lane + 32 * u] = c * a[u] - s * b[u];
+            xb[lane + 32 * u] = s * a[u] + c * b[u];
+          }
+          ++rot;
+        }
+      }
+      __syncthreads();
+    }
+    if (lane == 0 && rot) atomicAdd(s_counter, rot);
+    __syncthreads();
+    const int total = *s_counter;
+    __syncthreads();
+    if (total == 0) return true;
+  }
+  return false;
+}
+
+// column norms of X into out[kD] (warp per column)
+__device__ void column_norms(const float* X, float* out) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int c = warp; c < kD; c += kFitThreads / 32) {
+    float v = 0.f;
+    for (int i = lane; i < kD; i += 32) v = fmaf(X[c * kLdS + i], X[c * kLdS + i], v);
+    v = warp_sum(v);
+    if (lane == 0) out[c] = sqrtf(v);
+  }
+}
+
+__global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, float floor_rel, int max_sweeps,
+                                                             float tol, float* Fout, float* Gout, int* status) {
+  extern __shared__ __align__(16) float sm[];
+  float* Sb = sm;               // row-major, lower triangle becomes the Cholesky factor
+  float* Xb = sm + kD * kLdS;   // inverse factor, or the Jacobi matrix
+  __shared__ float lam[kD];
+  __shared__ float red[32];
+  __shared__ int flag, counter;
+  const int m = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* Sm = S + (int64_t)m * kD * kD;
+  float* F = Fout + (int64_t)m * kD * kD;
+  float* G = Gout + (int64_t)m * kD * kD;
+
+  for (int o = tid; o < kD * kD; o += kFitThreads) Sb[(o / kD) * kLdS + (o % kD)] = Sm[o];
+  if (tid == 0) flag = 0;
+  __syncthreads();
+  // trace and finiteness
+  if (warp == 0) {
+    float tr = 0.f;
+    for (int i = lane; i < kD; i += 32) tr += Sb[i * kLdS + i];
+    tr = warp_sum(tr);
+    if (lane == 0) red[0] = tr;
+  }
+  bool bad = false;
+  for (int o = tid; o < kD * kD; o += kFitThreads) bad |= !isfinite(Sm[o]);
+  if (__syncthreads_or(bad)) {
+    for (int o = tid; o < kD * kD; o += kFitThreads) { F[o] = 0.f; G[o] = 0.f; }
+    if (tid == 0) status[m] |= kStNonFinite;
+    return;
+  }
+  const float trace = red[0];
+
+  // Cholesky, right-looking, in place
+  for (int j = 0; j < kD; ++j) {
+    const float piv = Sb[j * kLdS + j];
+    const bool ok = piv > 0.f && isfinite(piv);
+    if (!ok) { if (tid == 0) flag = 1; }
+    __syncthreads();
+    if (flag) break;
+    const float ljj = sqrtf(piv);
+    for (int i = j + 1 + tid; i < kD; i += kFitThreads) Sb[i * kLdS + j] /= ljj;
+    __syncthreads();
+    if (tid == 0) Sb[j * kLdS + j] = ljj;
+    const int mm = kD - j - 1;
+    for (int o = tid; o < mm * mm; o += kFitThreads) {
+      const int i = j + 1 + o / mm, c = j + 1 + o % mm;
+      if (c <= i) Sb[i * kLdS + c] -= Sb[i * kLdS + j] * Sb[c * kLdS + j];
+    }
+    __syncthreads();
+  }
+
+  bool chol_ok = (flag == 0);
+  if (chol_ok) {
+    // Linv = F^{-1}, row by row; thread c owns column c
+    for (int i = 0; i < kD; ++i) {
+      if (tid < kD) {
+        const int c = tid;
+        float v = 0.f;
+        if (c <= i) {
+          float acc = (c == i) ? 1.f : 0.f;
+          for (int p = c; p < i; ++p) acc -= Sb[i * kLdS + p] * Xb[p * kLdS + c];
+          v = acc / Sb[i * kLdS + i];
+        }
+        Xb[i * kLdS + c] = v;
+      }
+      __syncthreads();
+    }
+    float ss = 0.f;
+    for (int o = tid; o < kD * kD; o += kFitThreads) {
+      const float v = Xb[(o / kD) * kLdS + (o % kD)];
+      ss = fmaf(v, v, ss);
+    }
+    ss = warp_sum(ss);
+    if (lane == 0) red[warp] = ss;
+    __syncthreads();
+    if (tid == 0) {
+      float t = 0.f;
+      for (int w = 0; w < kFitThreads / 32; ++w) t += red[w];
+      flag = (isfinite(t) && t > 0.f && 1.f / t >= floor_rel * trace) ? 0 : 2;
+    }
+    __syncthreads();
+    chol_ok = (flag == 0);
+  }
+  if (chol_ok) {
+    for (int o = tid; o < kD * kD; o += kFitThreads) {
+      const int i = o / kD, c = o % kD;
+      F[o] = c <= i ? Sb[i * kLdS + c] : 0.f;
+      G[o] = i <= c ? Xb[c * kLdS + i] : 0.f;   // G = Linv^T
+    }
+    return;
+  }
+
+  // exact floor: eigenpairs from one-sided Jacobi on S itself
+  for (int o = tid; o < kD * kD; o += kFitThreads) Xb[(o % kD) * kLdS + (o / kD)] = Sm[o];
+  __syncthreads();
+  const bool conv = jacobi_columns(Xb, max_sweeps, tol, &counter);
+  if (!conv && tid == 0) status[m] |= kStNotConverged;
+  column_norms(Xb, lam);
+  __syncthreads();
+  if (tid == 0) {
+    float mx = 0.f;
+    for (int i = 0; i < kD; ++i) mx = fmaxf(mx, lam[i]);
+    red[0] = mx;
+  }
+  __syncthreads();
+  const float lmax = red[0];
+  for (int o = tid; o < kD * kD; o += kFitThreads) {
+    const int i = o / kD, c = o % kD;
+    const float l = lam[c];
+    const bool keep = l > 0.f && l >= floor_rel * lmax;
+    const float w = Xb[c * kLdS + i];
+    F[o] = keep ? w / sqrtf(l) : 0.f;          // v sqrt(l),  v = w / l
+    G[o] = keep ? w / (l * sqrtf(l)) : 0.f;    // v / sqrt(l)
+  }
+}
+
+__global__ void __launch_bounds__(kFitThreads) fit_kernel(const float* A, const float* Fm, const float* Gm,
+                                                          const float* mu, int Hq, int Hk, int r, int max_sweeps,
+                                                          float tol, float* L, float* R, float* sigma, float* loss,
+                                                          float* nu, int* status) {
+  extern __shared__ __align__(16) float sm[];
+  float* X = sm;               // column-major, ld kLdS
+  float* Y = sm + kD * kLdS;
+  __shared__ float sig[kD];
+  __shared__ float sgn[kD];
+  __shared__ int perm[kD];
+  __shared__ int counter;
+  const int h = blockIdx.x, g = h / (Hq / Hk);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* Ah = A + (int64_t)h * kD * kD;
+  const float* Fq = Fm + (int64_t)h * kD * kD;
+  const float* Gq = Gm + (int64_t)h * kD * kD;
+  const float* Fk = Fm + (int64_t)(Hq + g) * kD * kD;
+  const float* Gk = Gm + (int64_t)(Hq + g) * kD * kD;
+  float* Lh = L + (int64_t)h * kD * r;
+  float* Rh = R + (int64_t)h * kD * r;
+
+  for (int o = tid; o < kD * kD; o += kFitThreads) Y[(o % kD) * kLdS + (o / kD)] = Ah[o];
+  __syncthreads();
+  const int cc = tid % kD, r0 = (tid / kD) * 32;
+  {  // X = A Fk
+    float acc[32];
+#pragma unroll
+    for (int u = 0; u < 32; ++u) acc[u] = 0.f;
+    for (int p = 0; p < kD; ++p) {
+      const float f = __ldg(Fk + p * kD + cc);
+#pragma unroll
+      for (int u = 0; u < 32; ++u) acc[u] = fmaf(Y[p * kLdS + r0 + u], f, acc[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < 32; ++u) X[cc * kLdS + r0 + u] = acc[u];
+  }
+  __syncthreads();
+  {  // Y = X^T Fq = C'^T
+    float acc[32];
+#pragma unroll
+    for (int u = 0; u < 32; ++u) acc[u] = 0.f;
+    for (int p = 0; p < kD; ++p) {
+      const float f = __ldg(Fq + p * kD + cc);
+#pragma unroll
+      for (int u = 0; u < 32; ++u) acc[u] = fmaf(X[(r0 + u) * kLdS + p], f, acc[u]);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < 32; ++u) Y[cc * kLdS + r0 + u] = acc[u];
+  }
+  __syncthreads();
+  for (int o = tid; o < kD * kLdS; o += kFitThreads) X[o] = Y[o];
+  __syncthreads();
+
+  const bool conv = jacobi_columns(X, max_sweeps, tol, &counter);
+  if (!conv && tid == 0) status[h] |= kStNotConverged;
+  column_norms(X, sig);
+  __syncthreads();
+  if (tid < kD) {  // rank = position in descending order, ties by index
+    const float s = sig[tid];
+    int rk = 0;
+    for (int j = 0; j < kD; ++j) rk += (sig[j] > s) || (sig[j] == s && j < tid);
+    perm[rk] = tid;
+  }
+  __syncthreads();
+  float smax = sig[perm[0]];
+  if (tid == 0 && !isfinite(smax)) status[h] |= kStNonFinite;
+
+  // Z = C' V_r Sigma^{-1} (= U_r) into L as scratch;  Rtmp = Gk V_r Sigma^{1/2} into Y after
+  const int a = tid % kD;
+  for (int c = tid / kD; c < r; c += kFitThreads / kD) {
+    const int i = perm[c];
+    const float s = sig[i];
+    const bool live = s > 0.f && s > smax * 1e-20f;
+    float acc = 0.f;
+    for (int b = 0; b < kD; ++b) acc = fmaf(Y[a * kLdS + b], X[i * kLdS + b], acc);
+    Lh[a * r + c] = live ? acc / (s * s) : 0.f;   // C' x_i / s^2 = u_i (x_i = s v_i)
+  }
+  __syncthreads();
+  for (int c = tid / kD; c < r; c += kFitThreads / kD) {
+    const int i = perm[c];
+    const float s = sig[i];
+    const bool live = s > 0.f && s > smax * 1e-20f;
+    float acc = 0.f;
+    for (int b = 0; b < kD; ++b) acc = fmaf(__ldg(Gk + a * kD + b), X[i * kLdS + b], acc);
+    Y[c * kLdS + a] = live ? acc / sqrtf(s) : 0.f;   // Gk v_i sqrt(s) = Gk x_i / sqrt(s)
+  }
+  __syncthreads();
+  for (int c = warp; c < r; c += kFitThreads / 32) {  // sign: largest-|.| entry of R[:, c] positive
+    float best = -1.f, val = 0.f;
+    int bi = 0;
+    for (int i = lane; i < kD; i += 32) {
+      const float v = Y[c * kLdS + i];
+      if (fabsf(v) > best) { best = fabsf(v); bi = i; val = v; }
+    }
+#pragma unroll
+    for (int m = 16; m > 0; m >>= 1) {
+      const float ob = __shfl_xor_sync(0xffffffffu, best, m);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, m);
+      const float ov = __shfl_xor_sync(0xffffffffu, val, m);
+      if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; val = ov; }
+    }
+    if (lane == 0) sgn[c] = val < 0.f ? -1.f : 1.f;
+  }
+  __syncthreads();
+  for (int o = tid; o < kD * r; o += kFitThreads) {
+    const int i = o / r, c = o % r;
+    Rh[o] = sgn[c] * Y[c * kLdS + i];
+    X[c * kLdS + i] = Lh[o];   // Z back into shared memory (X is free now)
+  }
+  __syncthreads();
+  for (int c = tid / kD; c < r; c += kFitThreads / kD) {
+    const float s = sig[perm[c]];
+    float acc = 0.f;
+    for (int e = 0; e < kD; ++e) acc = fmaf(__ldg(Gq + a * kD + e), X[c * kLdS + e], acc);
+    Lh[a * r + c] = sgn[c] * acc * sqrtf(fmaxf(s, 0.f));   // Gq u_i sqrt(s)
+  }
+  if (tid < kD && sigma) sigma[(int64_t)h * kD + tid] = sig[perm[tid]];
+  if (warp == 0 && loss) {
+    float v = 0.f;
+    for (int c = r + lane; c < kD; c += 32) v = fmaf(sig[perm[c]], sig[perm[c]], v);
+    v = warp_sum(v);
+    if (lane == 0) loss[h] = v;
+  }
+  if (nu && tid < kD) {
+    float v = 0.f;
+    if (mu)
+      for (int b = 0; b < kD; ++b) v = fmaf(__ldg(Ah + tid * kD + b), __ldg(mu + g * kD + b), v);
+    nu[(int64_t)h * kD + tid] = v;
+  }
+}
+
+constexpr float kTol = 1e-6f;
+constexpr size_t kSmem = 2 * sizeof(float) * kD * kLdS;
+}  // namespace
+
+cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps, float* F, float* Gm,
+                          int* status, cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(factor_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+  if (e != cudaSuccess) return e;
+  factor_kernel<<<nmat, kFitThreads, kSmem, s>>>(S, floor_rel, max_sweeps, kTol, F, Gm, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fit(const float* A, const float* F, const float* Gm, const float* mu, int Hq, int Hk, int r,
+                       int max_sweeps, float* L, float* R, float* sigma, float* loss, float* nu, int* status,
+                       cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(fit_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+  if (e != cudaSuccess) return e;
+  fit_kernel<<<Hq, kFitThreads, kSmem, s>>>(A, F, Gm, mu, Hq, Hk, r, max_sweeps, kTol, L, R, sigma, loss, nu,
+                                            status);
+  return cudaGetLastError();
+}
+
+}  // namespace saki

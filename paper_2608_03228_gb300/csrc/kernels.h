@@ -1,0 +1,75 @@
+// Internal interface between the C-ABI layer (api.cu) and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace saki {
+
+// One unit of scoring work: up to kGroupQ consecutive queries of one sequence
+// against keys [key_lo, key_hi) of that sequence (a split of its visible range).
+struct ScoreItem {
+  int32_t q_begin;      // first query row in Q
+  int32_t q_count;      // queries in the group
+  int32_t key_lo;       // sequence-local first key of this split
+  int32_t key_hi;       // sequence-local end of this split
+  int64_t key_base;     // global row of the sequence's key 0
+  int64_t cand;         // -1: write final lists; else candidate slot of (row 0, this split)
+  int32_t cand_stride;  // slots between consecutive rows (= number of splits)
+  int32_t pad;
+};
+
+// Merge of the per-split candidate lists of one query.
+struct MergeItem {
+  int32_t t;        // query row
+  int32_t nsplit;   // number of candidate lists
+  int64_t cand;     // slot of split 0 (lists are consecutive slots)
+};
+
+constexpr int kGroupQ = 8;  // queries per generic work item
+
+struct ScoreArgs {
+  const void* Q;        // [Hq][T][d]
+  const void* X;        // codes [Hq][N][P] (approximate) or keys [Hk][N][d] (exact)
+  const float* W;       // projection [Hq][d][P]: L (approximate) or A (exact)
+  const float* nu;      // [Hq][d] or null
+  const ScoreItem* items;
+  const MergeItem* merges;
+  const int32_t* vis;   // [T] visible keys per query
+  int32_t* idx;         // [Hq][T][k]
+  float* score;         // [Hq][T][k] or null
+  uint64_t* cand;       // candidate lists, kp keys per slot, per head: cand_per_head slots
+  int64_t cand_per_head;
+  int64_t T, N;
+  int32_t Hq, G, P, k, exact, n_items, n_merges;
+};
+
+// generic CUDA-core scoring (any rank, f32 or bf16)
+cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, cudaStream_t s);
+cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s);
+size_t score_generic_smem(int P, int kp);
+
+// calibration moments: S [(Hq+Hk)][d][d] (queries first), mu [Hk][d]
+cudaError_t launch_gram(const void* q_calib, const void* k_calib, int64_t n, int Hq, int Hk,
+                        int center, int dtype, float* S, float* mu, cudaStream_t s);
+
+// factor F (F F^T = S, floor applied) and G = pseudo-inverse transpose of F, per matrix
+cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps,
+                          float* F, float* Gm, int* status, cudaStream_t s);
+
+// per query head: C' = Fq^T A Fk, Jacobi SVD, factors L, R, sigma, loss, nu
+cudaError_t launch_fit(const float* A, const float* F, const float* Gm, const float* mu, int Hq,
+                       int Hk, int r, int max_sweeps, float* L, float* R, float* sigma,
+                       float* loss, float* nu, int* status, cudaStream_t s);
+
+// key codes
+cudaError_t launch_build_generic(const void* K, const float* R, const float* mu, void* sketch,
+                                 int64_t N, int Hq, int G, int r, int center, int dtype,
+                                 cudaStream_t s);
+
+// recall counters [Hq][2] (matches, rows) and final per-head recall
+cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int32_t* vis,
+                          int64_t T, int Hq, int k, int64_t min_visible,
+                          unsigned long long* counters, float* recall, cudaStream_t s);
+
+}  // namespace saki

@@ -1,0 +1,267 @@
+// Generic fused score + top-k on CUDA cores (any rank, f32 or bf16 inputs).
+//
+// Serves the decode-shaped work of the selection step (Sec. 5: s_hat = (L^T q)^T c_j
+// over the visible keys, keep the k largest) and, with W = A and X = K, the
+// exact top-k of the Sec. 3 recall protocol.  A work item is up to kGroupQ
+// queries of one sequence against one split of its keys; each lane scores one
+// key for all queries of the group from 128-bit loads, so every key row is read
+// once per item.  Selection never forms the score matrix: each warp keeps, per
+// query, a shared-memory buffer of candidates above its running k-th best key
+// and re-selects (warp bitonic sort) when the buffer fills; warps are merged at
+// the end, and splits of a long sequence by a second small kernel.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace saki {
+
+namespace {
+constexpr int kWarps = 8;
+constexpr int kThreads = kWarps * 32;
+
+template <typename T> __device__ __forceinline__ float to_f(T v);
+template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+// Keep the KP best of the warp's buffer (sorted, descending) and return the
+// k-th best key as the new acceptance threshold (0 while fewer than k).
+template <int KP>
+__device__ __forceinline__ void reselect(uint64_t* qb, int& cnt, uint64_t& thr, int k) {
+  constexpr int E = 2 * KP / 32;
+  const int lane = threadIdx.x & 31;
+  __syncwarp();
+  uint64_t v[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int i = e * 32 + lane;
+    v[e] = i < cnt ? qb[i] : 0ull;
+  }
+  warp_sort_desc<E>(v);
+  __syncwarp();
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int i = e * 32 + lane;
+    if (i < KP) qb[i] = v[e];
+  }
+  cnt = cnt < KP ? cnt : KP;
+  uint64_t t = 0;
+  const int ke = (k - 1) >> 5;
+#pragma unroll
+  for (int e = 0; e < E; ++e)
+    if (e == ke) t = v[e];
+  t = shfl_u64(t, (k - 1) & 31);
+  thr = cnt >= k ? t : 0ull;
+  __syncwarp();
+}
+
+template <typename Tin, int KP>
+__global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs a) {
+  constexpr int CAP = 2 * KP;
+  constexpr int EK = KP / 32;
+  constexpr int NV = Vec<Tin>::NV;
+  extern __shared__ __align__(16) unsigned char smem[];
+  uint64_t* buf = reinterpret_cast<uint64_t*>(smem);                       // [warps][GQ][CAP]
+  float* qs = reinterpret_cast<float*>(buf + kWarps * kGroupQ * CAP);      // [GQ][d]
+  float* us = qs + kGroupQ * kD;                                           // [GQ][P]
+  float* qnu = us + kGroupQ * a.P;                                         // [GQ]
+  int* visq = reinterpret_cast<int*>(qnu + kGroupQ);                       // [GQ]
+
+  const ScoreItem it = a.items[blockIdx.x];
+  const int h = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int P = a.P;
+  const int nq = it.q_count;
+
+  const Tin* Q = static_cast<const Tin*>(a.Q);
+  for (int o = tid; o < kGroupQ * kD; o += kThreads) {
+    const int b = o / kD;
+    qs[o] = b < nq ? to_f<Tin>(Q[((int64_t)h * a.T + it.q_begin + b) * kD + (o % kD)]) : 0.f;
+  }
+  if (tid < kGroupQ) visq[tid] = tid < nq ? a.vis[it.q_begin + tid] : 0;
+  for (int o = tid; o < kWarps * kGroupQ * CAP; o += kThreads) buf[o] = 0ull;
+  __syncthreads();
+
+  // u_b = W_h^T q_b (fp32), and the mean term q_b^T nu_h
+  const float* W = a.W + (int64_t)h * kD * P;
+  for (int o = tid; o < kGroupQ * P; o += kThreads) {
+    const int b = o / P, p = o % P;
+    float acc = 0.f;
+    for (int i = 0; i < kD; ++i) acc = fmaf(__ldg(W + i * P + p), qs[b * kD + i], acc);
+    us[o] = acc;
+  }
+  if (warp < kGroupQ) {
+    float v = 0.f;
+    if (a.nu)
+      for (int i = lane; i < kD; i += 32) v = fmaf(qs[warp * kD + i], __ldg(a.nu + (int64_t)h * kD + i), v);
+    v = warp_sum(v);
+    if (lane == 0) qnu[warp] = v;
+  }
+  __syncthreads();
+
+  const Tin* X = static_cast<const Tin*>(a.X) +
+                 ((int64_t)(a.exact ? h / a.G : h) * a.N + it.key_base) * P;
+  uint64_t thr[kGroupQ];
+  int cnt[kGroupQ];
+#pragma unroll
+  for (int b = 0; b < kGroupQ; ++b) { thr[b] = 0ull; cnt[b] = 0; }
+  uint64_t* wbuf = buf + warp * kGroupQ * CAP;
+  const int nkeys = it.key_hi - it.key_lo;
+  const bool vec = ((P * (int)sizeof(Tin)) % 16) == 0;
+  const unsigned lt_mask = (1u << lane) - 1u;
+
+  for (int base = warp * 32; base < nkeys; base += kThreads) {
+    const int jl = base + lane;
+    const int j = it.key_lo + jl;
+    float acc[kGroupQ];
+#pragma unroll
+    for (int b = 0; b < kGroupQ; ++b) acc[b] = 0.f;
+    if (jl < nkeys) {
+      const Tin* row = X + (int64_t)j * P;
+      if (vec) {
+        const uint4* r4 = reinterpret_cast<const uint4*>(row);
+        const int nv = P / NV;
+        for (int v = 0; v < nv; ++v) {
+          const uint4 raw = __ldg(r4 + v);
+          float x[NV];
+          Vec<Tin>::unpack(raw, x);
+#pragma unroll
+          for (int b = 0; b < kGroupQ; ++b) {
+            const float4* u4 = reinterpret_cast<const float4*>(us + b * P + v * NV);
+#pragma unroll
+            for (int e4 = 0; e4 < NV / 4; ++e4) {
+              const float4 uu = u4[e4];
+              acc[b] = fmaf(uu.x, x[4 * e4 + 0], acc[b]);
+              acc[b] = fmaf(uu.y, x[4 * e4 + 1], acc[b]);
+              acc[b] = fmaf(uu.z, x[4 * e4 + 2], acc[b]);
+              acc[b] = fmaf(uu.w, x[4 * e4 + 3], acc[b]);
+            }
+          }
+        }
+      } else {
+        for (int p = 0; p < P; ++p) {
+          const float x = to_f<Tin>(row[p]);
+#pragma unroll
+          for (int b = 0; b < kGroupQ; ++b) acc[b] = fmaf(us[b * P + p], x, acc[b]);
+        }
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < kGroupQ; ++b) {
+      if (b < nq) {
+        const bool ok = (jl < nkeys) && (j < visq[b]);
+        const uint64_t key = make_key(acc[b], (uint32_t)j);
+        const bool pass = ok && key > thr[b];
+        const unsigned mask = __ballot_sync(0xffffffffu, pass);
+        if (mask) {
+          uint64_t* qb = wbuf + b * CAP;
+          if (pass) qb[cnt[b] + __popc(mask & lt_mask)] = key;
+          cnt[b] += __popc(mask);
+          if (cnt[b] > CAP - 32) reselect<KP>(qb, cnt[b], thr[b], a.k);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int b = 0; b < kGroupQ; ++b)
+    if (b < nq) reselect<KP>(wbuf + b * CAP, cnt[b], thr[b], a.k);
+  __syncthreads();
+
+  // merge the warps' lists of query `warp`
+  if (warp < nq) {
+    const int b = warp;
+    uint64_t best[EK], other[EK];
+#pragma unroll
+    for (int e = 0; e < EK; ++e) best[e] = buf[(0 * kGroupQ + b) * CAP + e * 32 + lane];
+    for (int w2 = 1; w2 < kWarps; ++w2) {
+#pragma unroll
+      for (int e = 0; e < EK; ++e) other[e] = buf[(w2 * kGroupQ + b) * CAP + e * 32 + lane];
+      warp_merge_top<EK>(best, other);
+    }
+    if (it.cand < 0) {
+      const int64_t row = ((int64_t)h * a.T + it.q_begin + b) * a.k;
+#pragma unroll
+      for (int e = 0; e < EK; ++e) {
+        const int i = e * 32 + lane;
+        if (i < a.k) {
+          a.idx[row + i] = key_index(best[e]);
+          if (a.score) a.score[row + i] = best[e] ? key_score(best[e]) + qnu[b] : -INFINITY;
+        }
+      }
+    } else {
+      uint64_t* c = a.cand + ((int64_t)h * a.cand_per_head + it.cand + (int64_t)b * it.cand_stride) * KP;
+#pragma unroll
+      for (int e = 0; e < EK; ++e) c[e * 32 + lane] = best[e];
+    }
+  }
+}
+
+template <typename Tin, int KP>
+__global__ void __launch_bounds__(128) merge_kernel(const ScoreArgs a) {
+  constexpr int EK = KP / 32;
+  const int lane = threadIdx.x & 31;
+  const int m = blockIdx.x * 4 + (threadIdx.x >> 5);
+  if (m >= a.n_merges) return;
+  const int h = blockIdx.y;
+  const MergeItem mi = a.merges[m];
+  const uint64_t* c = a.cand + ((int64_t)h * a.cand_per_head + mi.cand) * KP;
+  uint64_t best[EK], other[EK];
+#pragma unroll
+  for (int e = 0; e < EK; ++e) best[e] = c[e * 32 + lane];
+  for (int s = 1; s < mi.nsplit; ++s) {
+#pragma unroll
+    for (int e = 0; e < EK; ++e) other[e] = c[(int64_t)s * KP + e * 32 + lane];
+    warp_merge_top<EK>(best, other);
+  }
+  float qnu = 0.f;
+  if (a.nu) {
+    const Tin* q = static_cast<const Tin*>(a.Q) + ((int64_t)h * a.T + mi.t) * kD;
+    for (int i = lane; i < kD; i += 32) qnu = fmaf(to_f<Tin>(q[i]), __ldg(a.nu + (int64_t)h * kD + i), qnu);
+    qnu = warp_sum(qnu);
+  }
+  const int64_t row = ((int64_t)h * a.T + mi.t) * a.k;
+#pragma unroll
+  for (int e = 0; e < EK; ++e) {
+    const int i = e * 32 + lane;
+    if (i < a.k) {
+      a.idx[row + i] = key_index(best[e]);
+      if (a.score) a.score[row + i] = best[e] ? key_score(best[e]) + qnu : -INFINITY;
+    }
+  }
+}
+
+template <typename Tin, int KP>
+cudaError_t launch_score_t(const ScoreArgs& a, cudaStream_t s) {
+  const size_t sm = score_generic_smem(a.P, KP);
+  auto kern = score_generic_kernel<Tin, KP>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+  if (e != cudaSuccess) return e;
+  kern<<<dim3(a.n_items, a.Hq), kThreads, sm, s>>>(a);
+  return cudaGetLastError();
+}
+}  // namespace
+
+size_t score_generic_smem(int P, int kp) {
+  return sizeof(uint64_t) * (size_t)kWarps * kGroupQ * 2 * kp +
+         sizeof(float) * (size_t)(kGroupQ * kD + kGroupQ * P + kGroupQ) + sizeof(int) * kGroupQ;
+}
+
+cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, cudaStream_t s) {
+  if (a.n_items == 0) return cudaSuccess;
+  if (dtype == SAKI_BF16)
+    return kp == 64 ? launch_score_t<__nv_bfloat16, 64>(a, s) : launch_score_t<__nv_bfloat16, 128>(a, s);
+  return kp == 64 ? launch_score_t<float, 64>(a, s) : launch_score_t<float, 128>(a, s);
+}
+
+cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s) {
+  if (a.n_merges == 0) return cudaSuccess;
+  dim3 grid((a.n_merges + 3) / 4, a.Hq);
+  if (dtype == SAKI_BF16) {
+    if (kp == 64) merge_kernel<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(a);
+    else merge_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(a);
+  } else {
+    if (kp == 64) merge_kernel<float, 64><<<grid, 128, 0, s>>>(a);
+    else merge_kernel<float, 128><<<grid, 128, 0, s>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace saki

@@ -1,0 +1,161 @@
+"""Thin ctypes binding of libsaki.so (include/saki.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels.  Device tensors are torch CUDA tensors (PyTorch supplies device memory
+and the current stream); the layout arrays are host numpy arrays.  Importing
+this module loads the library and raises if it has not been built -- there is
+no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libsaki.so")
+if not os.path.exists(_LIB_PATH):
+    raise ImportError(f"{_LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+_lib = ctypes.CDLL(_LIB_PATH)
+
+SAKI_F32, SAKI_BF16 = 0, 1
+SAKI_FLAG_SORTED = 1
+SAKI_OP_FIT, SAKI_OP_BUILD_INDEX, SAKI_OP_SCORE_TOPK, SAKI_OP_RECALL = 0, 1, 2, 3
+STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED", 3: "SAKI_ERR_CUDA",
+          4: "SAKI_ERR_NUMERIC", 5: "SAKI_ERR_NOT_CONVERGED", 6: "SAKI_ERR_WORKSPACE", 7: "SAKI_ERR_TIMEOUT"}
+EXPORTS = ("saki_workspace_size", "saki_fit", "saki_build_index", "saki_score_topk", "saki_recall",
+           "saki_status_string", "saki_version")
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("rank", ctypes.c_int32), ("topk", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("center", ctypes.c_int32), ("eig_floor_rel", ctypes.c_float), ("max_sweeps", ctypes.c_int32),
+                ("flags", ctypes.c_int32)]
+
+
+class Layout(ctypes.Structure):
+    _fields_ = [("num_seqs", ctypes.c_int32), ("seq_offsets", ctypes.c_void_p), ("num_queries", ctypes.c_int64),
+                ("q_seq", ctypes.c_void_p), ("q_visible", ctypes.c_void_p)]
+
+
+_vp, _i64, _i32, _sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_size_t
+_lib.saki_workspace_size.restype = _sz
+_lib.saki_workspace_size.argtypes = [ctypes.POINTER(Config), _i32, ctypes.POINTER(Layout), _i64, _i64]
+_lib.saki_fit.restype = ctypes.c_int
+_lib.saki_fit.argtypes = [ctypes.POINTER(Config), _i64] + [_vp] * 10 + [_sz, _vp]
+_lib.saki_build_index.restype = ctypes.c_int
+_lib.saki_build_index.argtypes = [ctypes.POINTER(Config), _i64] + [_vp] * 5 + [_sz, _vp]
+_lib.saki_score_topk.restype = ctypes.c_int
+_lib.saki_score_topk.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout)] + [_vp] * 7 + [_sz, _vp]
+_lib.saki_recall.restype = ctypes.c_int
+_lib.saki_recall.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout), _i64] + [_vp] * 7 + [_sz, _vp]
+_lib.saki_status_string.restype = ctypes.c_char_p
+_lib.saki_status_string.argtypes = [ctypes.c_int]
+_lib.saki_version.restype = ctypes.c_char_p
+
+
+class SakiError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS.get(status, status)} ({_lib.saki_status_string(status).decode()})")
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def make_config(num_q_heads, num_kv_heads, rank, topk, dtype="bf16", center=0, eig_floor_rel=1e-6,
+                max_sweeps=0, flags=0, head_dim=128) -> Config:
+    dt = {"f32": SAKI_F32, "bf16": SAKI_BF16}.get(dtype, dtype)
+    return Config(num_q_heads, num_kv_heads, head_dim, rank, topk, dt, center, eig_floor_rel, max_sweeps, flags)
+
+
+class HostLayout:
+    """Holds the host arrays of a saki_layout alive while a call uses them."""
+
+    def __init__(self, seq_offsets, q_seq, q_visible):
+        self.seq_offsets = np.ascontiguousarray(seq_offsets, np.int64)
+        self.q_seq = np.ascontiguousarray(q_seq, np.int32)
+        self.q_visible = np.ascontiguousarray(q_visible, np.int64)
+        self.c = Layout(len(self.seq_offsets) - 1, self.seq_offsets.ctypes.data, len(self.q_seq),
+                        self.q_seq.ctypes.data if len(self.q_seq) else None,
+                        self.q_visible.ctypes.data if len(self.q_visible) else None)
+
+    @property
+    def total_keys(self) -> int:
+        return int(self.seq_offsets[-1])
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is not None:
+        return stream if isinstance(stream, int) else stream.cuda_stream
+    import torch
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise SakiError(status, where)
+
+
+def _workspace(nbytes: int, device):
+    import torch
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def saki_status_string(status: int) -> str:
+    return _lib.saki_status_string(status).decode()
+
+
+def saki_version() -> str:
+    return _lib.saki_version().decode()
+
+
+def saki_workspace_size(cfg: Config, op: int, layout: HostLayout | None = None, n_calib: int = 0,
+                        total_keys: int = 0) -> int:
+    return int(_lib.saki_workspace_size(ctypes.byref(cfg), op, ctypes.byref(layout.c) if layout else None,
+                                        n_calib, total_keys))
+
+
+def saki_fit(cfg: Config, q_calib, k_calib, A, L, R, mu=None, nu=None, sigma=None, loss=None, workspace=None,
+             stream=None):
+    """Prop. 1 fit; all arguments are CUDA tensors laid out as in saki.h."""
+    n = q_calib.shape[1]
+    need = saki_workspace_size(cfg, SAKI_OP_FIT, n_calib=n)
+    ws = workspace if workspace is not None else _workspace(need, q_calib.device)
+    _check(_lib.saki_fit(ctypes.byref(cfg), n, _ptr(q_calib), _ptr(k_calib), _ptr(A), _ptr(L), _ptr(R), _ptr(mu),
+                         _ptr(nu), _ptr(sigma), _ptr(loss), _ptr(ws), ws.numel(), _stream(stream)), "saki_fit")
+
+
+def saki_build_index(cfg: Config, K, R, sketch, mu=None, workspace=None, stream=None):
+    N = K.shape[1]
+    need = saki_workspace_size(cfg, SAKI_OP_BUILD_INDEX, total_keys=N)
+    ws = workspace if workspace is not None else _workspace(need, K.device)
+    _check(_lib.saki_build_index(ctypes.byref(cfg), N, _ptr(K), _ptr(R), _ptr(mu), _ptr(sketch), _ptr(ws),
+                                 ws.numel(), _stream(stream)), "saki_build_index")
+
+
+def saki_score_topk(cfg: Config, layout: HostLayout, Q, L, sketch, idx, score=None, nu=None, workspace=None,
+                    stream=None):
+    need = saki_workspace_size(cfg, SAKI_OP_SCORE_TOPK, layout)
+    ws = workspace if workspace is not None else _workspace(need, Q.device)
+    _check(_lib.saki_score_topk(ctypes.byref(cfg), ctypes.byref(layout.c), _ptr(Q), _ptr(L), _ptr(sketch), _ptr(nu),
+                                _ptr(idx), _ptr(score), _ptr(ws), ws.numel(), _stream(stream)), "saki_score_topk")
+
+
+def saki_recall(cfg: Config, layout: HostLayout, min_visible: int, Q, A, K, idx_approx, recall, idx_exact=None,
+                workspace=None, stream=None):
+    need = saki_workspace_size(cfg, SAKI_OP_RECALL, layout)
+    ws = workspace if workspace is not None else _workspace(need, Q.device)
+    _check(_lib.saki_recall(ctypes.byref(cfg), ctypes.byref(layout.c), min_visible, _ptr(Q), _ptr(A), _ptr(K),
+                            _ptr(idx_approx), _ptr(idx_exact), _ptr(recall), _ptr(ws), ws.numel(), _stream(stream)),
+           "saki_recall")

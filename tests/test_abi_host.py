@@ -1,0 +1,130 @@
+"""Host-side checks of the C ABI: the library builds and loads without a GPU,
+exports every symbol include/saki.h declares, the ctypes structs match the C
+layout, and invalid arguments are rejected before any device work."""
+import ctypes
+import os
+import re
+import subprocess
+import tempfile
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "saki.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_03228_gb300 import _build
+    if not os.path.exists(_build.LIB):
+        _build.build()
+    from paper_2608_03228_gb300 import saki
+    return saki
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"SAKI_API\s+[\w\s\*]+?\b(saki_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_four_path_calls():
+    syms = declared_symbols()
+    for s in ("saki_fit", "saki_build_index", "saki_score_topk", "saki_recall"):
+        assert s in syms
+
+
+def test_every_declared_symbol_is_exported(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", lib.library_path()], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (saki_\w+)", out))
+    missing = [s for s in declared_symbols() if s not in exported]
+    assert not missing, missing
+    for s in declared_symbols():
+        assert hasattr(lib._lib, s)
+
+
+def test_ctypes_layout_matches_c(lib, tmp_path):
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "saki.h"\nint main(void){'
+                   'printf("%zu %zu %zu %zu %zu\\n", sizeof(saki_config), offsetof(saki_config, eig_floor_rel),'
+                   ' offsetof(saki_config, flags), sizeof(saki_layout), offsetof(saki_layout, q_visible));return 0;}')
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    vals = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True).stdout.split()]
+    assert vals == [ctypes.sizeof(lib.Config), lib.Config.eig_floor_rel.offset, lib.Config.flags.offset,
+                    ctypes.sizeof(lib.Layout), lib.Layout.q_visible.offset]
+
+
+def test_status_strings(lib):
+    for code in range(8):
+        assert lib.saki_status_string(code)
+    assert lib.saki_version().count(".") == 2
+
+
+FAKE = 1 << 20   # aligned, never dereferenced: every call below fails before any device work
+
+
+def _cfg(lib, **kw):
+    base = dict(num_q_heads=8, num_kv_heads=2, rank=32, topk=64, dtype="bf16")
+    base.update(kw)
+    return lib.make_config(**base)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(num_kv_heads=3), 1), (dict(rank=0), 1), (dict(rank=129), 1), (dict(topk=0), 1), (dict(topk=129), 2),
+    (dict(head_dim=64), 2), (dict(dtype=7), 1), (dict(center=2), 1), (dict(eig_floor_rel=-1.0), 1),
+    (dict(max_sweeps=-1), 1), (dict(flags=4), 1),
+])
+def test_config_validation(lib, kw, code):
+    cfg = _cfg(lib, **kw)
+    st = lib._lib.saki_fit(ctypes.byref(cfg), 16, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, None, None, FAKE,
+                           1 << 40, None)
+    assert st == code
+    assert lib.saki_workspace_size(cfg, lib.SAKI_OP_FIT, n_calib=16) == 0
+
+
+def test_fit_argument_checks(lib):
+    cfg = _cfg(lib)
+    call = lambda *p: lib._lib.saki_fit(ctypes.byref(cfg), *p)
+    assert call(16, None, FAKE, FAKE, FAKE, FAKE, None, None, None, None, FAKE, 1 << 40, None) == 1
+    assert call(0, FAKE, FAKE, FAKE, FAKE, FAKE, None, None, None, None, FAKE, 1 << 40, None) == 1
+    assert call(16, FAKE + 2, FAKE, FAKE, FAKE, FAKE, None, None, None, None, FAKE, 1 << 40, None) == 1
+    need = lib.saki_workspace_size(cfg, lib.SAKI_OP_FIT, n_calib=16)
+    assert need >= 10 * 128 * 128 * 4 * 3
+    assert call(16, FAKE, FAKE, FAKE, FAKE, FAKE, None, None, None, None, FAKE, need - 1, None) == 6
+    cfg.center = 1   # centered keys need the mu output
+    assert call(16, FAKE, FAKE, FAKE, FAKE, FAKE, None, None, None, None, FAKE, need, None) == 1
+
+
+def _layout(lib, lens, q_seq, q_vis):
+    off = np.zeros(len(lens) + 1, np.int64)
+    off[1:] = np.cumsum(lens)
+    return lib.HostLayout(off, q_seq, q_vis)
+
+
+def test_layout_validation(lib):
+    cfg = _cfg(lib)
+    good = _layout(lib, [100, 50], [0, 0, 1], [100, 3, 50])
+    assert lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_TOPK, good) > 0
+    for lay in (_layout(lib, [100], [1], [5]),          # sequence id out of range
+                _layout(lib, [100], [0], [101]),        # sees more keys than its sequence holds
+                _layout(lib, [100], [0], [-1])):
+        assert lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_TOPK, lay) == 0
+        st = lib._lib.saki_score_topk(ctypes.byref(cfg), ctypes.byref(lay.c), FAKE, FAKE, FAKE, None, FAKE, None,
+                                      FAKE, 1 << 40, None)
+        assert st == 1
+    st = lib._lib.saki_score_topk(ctypes.byref(cfg), ctypes.byref(good.c), FAKE, FAKE, FAKE, None, FAKE, None, FAKE,
+                                  16, None)
+    assert st == 6
+    st = lib._lib.saki_recall(ctypes.byref(cfg), ctypes.byref(good.c), 65, FAKE, FAKE, FAKE, FAKE, None, None,
+                              FAKE, 1 << 40, None)
+    assert st == 1   # recall output missing
+
+
+def test_workspace_grows_with_splits(lib):
+    """A long decode sequence is split across CTAs; the split lists need room."""
+    cfg = _cfg(lib, num_q_heads=32, num_kv_heads=8)
+    short = _layout(lib, [4096], [0] * 8, [4096] * 8)
+    long_ = _layout(lib, [1 << 20], [0] * 8, [1 << 20] * 8)
+    assert lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_TOPK, long_) > \
+        lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_TOPK, short)

@@ -1,0 +1,287 @@
+"""GPU parity: every step of the path through the C ABI against the fp64 oracle
+on the same seeded inputs (stage by stage, then end to end)."""
+import numpy as np
+import pytest
+
+from oracle import saki_oracle as O
+from paper_2608_03228_gb300 import synth
+from tests.parity import (GAP_REL, MAP_REL, RECALL_ABS, check_topk_rows, f32, map_rel_err, to_dev)
+
+pytestmark = pytest.mark.gpu
+D = 128
+
+
+def _torch():
+    import torch
+    assert torch.cuda.is_available(), "GPU test without a GPU"
+    return torch
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    w = synth.WORKLOADS["tiny_f32_t512"]
+    data = synth.make_numpy(w)
+    ref = O.fit(data["q_calib"], data["k_calib"], data["A"], w.rank, center=bool(w.center))
+    return w, data, ref
+
+
+def _gpu_fit(lib, w, data, center=None, rank=None):
+    torch = _torch()
+    center = w.center if center is None else center
+    r = w.rank if rank is None else rank
+    cfg = lib.make_config(w.num_q_heads, w.num_kv_heads, r, w.topk, w.dtype, center=center)
+    Hq, Hk = w.num_q_heads, w.num_kv_heads
+    L = torch.empty((Hq, D, r), device="cuda")
+    R = torch.empty((Hq, D, r), device="cuda")
+    mu = torch.empty((Hk, D), device="cuda")
+    nu = torch.empty((Hq, D), device="cuda")
+    sig = torch.empty((Hq, D), device="cuda")
+    loss = torch.empty((Hq,), device="cuda")
+    ws = torch.empty(lib.saki_workspace_size(cfg, lib.SAKI_OP_FIT, n_calib=w.n_calib), dtype=torch.uint8,
+                     device="cuda")
+    lib.saki_fit(cfg, to_dev(data["q_calib"], w.dtype), to_dev(data["k_calib"], w.dtype), f32(data["A"]), L, R,
+                 mu=mu, nu=nu, sigma=sig, loss=loss, workspace=ws)
+    torch.cuda.synchronize()
+    nm = Hq + Hk
+    S = ws[: nm * D * D * 4].view(torch.float32).reshape(nm, D, D).cpu().numpy()
+    return dict(L=L.cpu().numpy(), R=R.cpu().numpy(), mu=mu.cpu().numpy(), nu=nu.cpu().numpy(),
+                sigma=sig.cpu().numpy(), loss=loss.cpu().numpy(), S=S, cfg=cfg)
+
+
+def _rel_gap(sig, r):
+    return (sig[r - 1] - sig[r]) / sig[0] if r < len(sig) else 1.0
+
+
+# ------------------------------------------------------------------- a1 + a2
+@pytest.mark.parametrize("center", [0, 1])
+def test_fit_tiny(lib, tiny, center):
+    w, data, _ = tiny
+    ref = O.fit(data["q_calib"], data["k_calib"], data["A"], w.rank, center=bool(center))
+    g = _gpu_fit(lib, w, data, center=center)
+    Hq = w.num_q_heads
+    for h in range(Hq):   # moments (Sec. 5): fp32 accumulation of n products
+        assert np.linalg.norm(g["S"][h] - ref["Sq"][h]) <= 1e-5 * np.linalg.norm(ref["Sq"][h])
+    for gk in range(w.num_kv_heads):
+        assert np.linalg.norm(g["S"][Hq + gk] - ref["Sk"][gk]) <= 1e-5 * np.linalg.norm(ref["Sk"][gk])
+        np.testing.assert_allclose(g["mu"][gk], ref["mu"][gk], atol=1e-5)
+    for h in range(Hq):
+        s_ref = ref["sigma"][h]
+        np.testing.assert_allclose(g["sigma"][h], s_ref, atol=1e-4 * s_ref[0], rtol=0)
+        assert abs(g["loss"][h] - ref["loss"][h]) <= 1e-4 * np.sum(s_ref ** 2)
+        if _rel_gap(s_ref, w.rank) >= 1e-3:
+            assert map_rel_err(g["L"][h], g["R"][h], ref["M"][h]) <= MAP_REL
+        np.testing.assert_allclose(g["nu"][h], ref["nu"][h], atol=1e-4 * max(1.0, np.abs(ref["nu"][h]).max()))
+
+
+def test_fit_full_rank_and_rank_one(lib, tiny):
+    w, data, _ = tiny
+    for r in (1, D):
+        ref = O.fit(data["q_calib"], data["k_calib"], data["A"], r, center=False)
+        g = _gpu_fit(lib, w, data, rank=r)
+        for h in range(w.num_q_heads):
+            if _rel_gap(ref["sigma"][h], r) >= 1e-3:
+                assert map_rel_err(g["L"][h], g["R"][h], ref["M"][h]) <= MAP_REL, (r, h)
+            if r == D:   # M_d = A (Prop. 1 with nothing discarded)
+                A = data["A"][h].astype(np.float64)
+                assert np.linalg.norm(g["L"][h] @ g["R"][h].T - A) <= 1e-4 * np.linalg.norm(A)
+
+
+def test_fit_singular_calibration(lib):
+    """n < d: rank-deficient moments take the exact eigenvalue-floor path."""
+    w = synth.Workload("sing", 2, 1, rank=8, dtype="f32", n_calib=40, seq_lens=(64,), spikes=(4, 4), seed=7)
+    data = synth.make_numpy(w)
+    ref = O.fit(data["q_calib"], data["k_calib"], data["A"], w.rank, center=False)
+    g = _gpu_fit(lib, w, data)
+    for h in range(w.num_q_heads):
+        if _rel_gap(ref["sigma"][h], w.rank) >= 1e-3:
+            assert map_rel_err(g["L"][h], g["R"][h], ref["M"][h]) <= 1e-3
+        np.testing.assert_allclose(g["sigma"][h][:20], ref["sigma"][h][:20], atol=1e-3 * ref["sigma"][h][0])
+
+
+def test_fit_rejects_nonfinite(lib, tiny):
+    torch = _torch()
+    w, data, _ = tiny
+    q = data["q_calib"].copy()
+    q[1, 3, 5] = np.nan
+    cfg = lib.make_config(w.num_q_heads, w.num_kv_heads, w.rank, w.topk, w.dtype)
+    L = torch.empty((w.num_q_heads, D, w.rank), device="cuda")
+    R = torch.empty_like(L)
+    with pytest.raises(lib.SakiError) as e:
+        lib.saki_fit(cfg, to_dev(q, w.dtype), to_dev(data["k_calib"], w.dtype), f32(data["A"]), L, R)
+    assert e.value.status == 4
+
+
+# ------------------------------------------------------------------------ a3
+def _build(lib, w, K, R, mu=None, center=0):
+    torch = _torch()
+    cfg = lib.make_config(w.num_q_heads, w.num_kv_heads, R.shape[2], w.topk, w.dtype, center=center)
+    N = K.shape[1]
+    sk = torch.empty((w.num_q_heads, N, R.shape[2]), dtype=torch.bfloat16 if w.dtype == "bf16" else torch.float32,
+                     device="cuda")
+    lib.saki_build_index(cfg, to_dev(K, w.dtype), f32(R), sk, mu=None if mu is None else f32(mu))
+    return sk.float().cpu().numpy()
+
+
+@pytest.mark.parametrize("dtype,r,center", [("f32", 16, 0), ("bf16", 32, 0), ("bf16", 64, 1), ("f32", 5, 1)])
+def test_build_index(lib, dtype, r, center):
+    w = synth.Workload("bi", 8, 2, rank=r, dtype=dtype, n_calib=256, seq_lens=(1000,), spikes=(6, 6), seed=3)
+    data = synth.make_numpy(w)
+    ref = O.fit(data["q_calib"], data["k_calib"], data["A"], r, center=bool(center))
+    R = ref["R"].astype(np.float32)
+    mu = ref["mu"].astype(np.float32)
+    got = _build(lib, w, data["K"], R, mu if center else None, center)
+    exact = np.array([(data["K"][h // w.group].astype(np.float64) - (mu[h // w.group] if center else 0))
+                      @ R[h].astype(np.float64) for h in range(w.num_q_heads)])
+    if dtype == "f32":
+        bound = np.array([np.abs(data["K"][h // w.group].astype(np.float64) - (mu[h // w.group] if center else 0))
+                          @ np.abs(R[h].astype(np.float64)) for h in range(w.num_q_heads)])
+        assert np.all(np.abs(got - exact) <= 2e-6 * bound + 1e-30)
+    else:
+        rne = O.round_bf16(exact)
+        # faithful rounding (within one bf16 step) everywhere, round-to-nearest almost everywhere
+        assert np.all(np.abs(got - exact) <= 2.0 ** -7 * np.abs(exact) + 1e-38)
+        assert np.mean(got == rne) >= 0.999
+
+
+# ------------------------------------------------------------------ a4 + a5
+def _layout_arrays(lens, queries):
+    off = np.zeros(len(lens) + 1, np.int64)
+    off[1:] = np.cumsum(lens)
+    q_seq, q_vis = [], []
+    for s, (L, qs) in enumerate(zip(lens, queries)):
+        for v in qs:
+            q_seq.append(s)
+            q_vis.append(min(v, L) if v >= 0 else L)
+    return off, np.array(q_seq, np.int32), np.array(q_vis, np.int64)
+
+
+def _score_case(lib, Hq, Hk, r, k, dtype, lens, queries, seed=0, center=0, flags=1):
+    torch = _torch()
+    rng = np.random.default_rng(seed)
+    off, q_seq, q_vis = _layout_arrays(lens, queries)
+    N, T = int(off[-1]), len(q_seq)
+    G = Hq // Hk
+    cast = (lambda a: synth.round_to_bf16_grid(a)) if dtype == "bf16" else (lambda a: a.astype(np.float32))
+    Q = cast(rng.standard_normal((Hq, T, D)).astype(np.float32))
+    L = (rng.standard_normal((Hq, D, r)) / np.sqrt(D)).astype(np.float32)
+    sketch = O.round_to(dtype, rng.standard_normal((Hq, N, r))).astype(np.float32)
+    nu = rng.standard_normal((Hq, D)).astype(np.float32) if center else None
+    cfg = lib.make_config(Hq, Hk, r, k, dtype, center=center, flags=flags)
+    lay = lib.HostLayout(off, q_seq, q_vis)
+    idx = torch.empty((Hq, T, k), dtype=torch.int32, device="cuda")
+    sc = torch.empty((Hq, T, k), dtype=torch.float32, device="cuda")
+    lib.saki_score_topk(cfg, lay, to_dev(Q, dtype), f32(L), to_dev(sketch, dtype), idx, score=sc,
+                        nu=None if nu is None else f32(nu))
+    idx, sc = idx.cpu().numpy(), sc.cpu().numpy()
+    for h in range(Hq):
+        rows = []
+        for t in range(T):
+            b = off[q_seq[t]]
+            rows.append(O.approx_scores(Q[h, t], L[h], sketch[h, b:b + q_vis[t]]))
+        qnu = [float(Q[h, t].astype(np.float64) @ nu[h]) if nu is not None else 0.0 for t in range(T)]
+        check_topk_rows(idx[h], rows, k, gpu_scores=sc[h] - np.array(qnu, np.float32)[:, None], label=f"h{h}")
+        if flags & 1:   # sorted: descending scores
+            for t in range(T):
+                v = sc[h, t][idx[h, t] >= 0]
+                assert np.all(np.diff(v) <= 0)
+    return idx, sc
+
+
+def test_score_topk_tiny_causal(lib, tiny):
+    """Stage parity on the tiny workload: oracle L and codes in, top-64 out."""
+    torch = _torch()
+    w, data, ref = tiny
+    L = ref["L"].astype(np.float32)
+    sketch = O.build_index(data["K"], ref["R"].astype(np.float32), None, "f32", w.group).astype(np.float32)
+    cfg = lib.make_config(w.num_q_heads, w.num_kv_heads, w.rank, w.topk, w.dtype, flags=1)
+    lay = lib.HostLayout(data["seq_offsets"], data["q_seq"], data["q_visible"])
+    T = len(data["q_seq"])
+    idx = torch.empty((w.num_q_heads, T, w.topk), dtype=torch.int32, device="cuda")
+    sc = torch.empty_like(idx, dtype=torch.float32)
+    lib.saki_score_topk(cfg, lay, to_dev(data["Q"], "f32"), f32(L), f32(sketch), idx, score=sc)
+    idx, sc = idx.cpu().numpy(), sc.cpu().numpy()
+    waived = 0
+    for h in range(w.num_q_heads):
+        rows = [O.approx_scores(data["Q"][h, t], L[h], sketch[h, :data["q_visible"][t]]) for t in range(T)]
+        waived += check_topk_rows(idx[h], rows, w.topk, gpu_scores=sc[h], label=f"h{h}")[1]
+    assert waived <= 2
+
+
+@pytest.mark.parametrize("case", [
+    # Hq, Hk, r, k, dtype, lens, queries per sequence (-1 = whole sequence)
+    (4, 1, 32, 64, "bf16", (3000,), ([-1] * 8,)),                          # decode, one group
+    (4, 2, 16, 64, "bf16", (10000,), ([-1, 9999, 5000, 100, 64, 65, 1, 0],)),  # splits + merge, mixed visibility
+    (2, 1, 1, 1, "f32", (300,), (list(range(0, 300, 7)),)),                 # r = 1 (scalar path), k = 1
+    (2, 2, 128, 100, "f32", (500, 90), ([-1, 250, 99], [-1, 3])),          # r = d, k > 64 (wide buffers)
+    (8, 2, 64, 64, "bf16", (40, 17, 6000, 64), ([-1, 20], [-1], [-1] * 4, [-1, 63])),  # ragged, short seqs
+    (4, 1, 24, 32, "bf16", (2500,), (list(range(2400, 2500)),)),            # many groups of one sequence
+])
+def test_score_topk_layouts(lib, case):
+    Hq, Hk, r, k, dtype, lens, queries = case
+    _score_case(lib, Hq, Hk, r, k, dtype, lens, queries, seed=int(sum(lens)) % 1000 + r)
+
+
+def test_score_topk_mean_term(lib):
+    _score_case(lib, 4, 1, 32, 64, "bf16", (700,), ([-1, 300],), center=1)
+
+
+def test_score_topk_unsorted_flag(lib):
+    _score_case(lib, 2, 1, 32, 64, "bf16", (900,), ([-1, 500],), flags=0)
+
+
+# ------------------------------------------------------------------ a6 + a7
+def test_recall_tiny(lib, tiny):
+    torch = _torch()
+    w, data, ref = tiny
+    G = w.group
+    L = ref["L"].astype(np.float32)
+    sketch = O.build_index(data["K"], ref["R"].astype(np.float32), None, "f32", G)
+    ia, _ = O.score_topk(data["Q"], L, sketch, data["seq_offsets"], data["q_seq"], data["q_visible"], w.topk)
+    ie, _ = O.exact_topk(data["Q"], data["A"], data["K"], data["seq_offsets"], data["q_seq"], data["q_visible"],
+                         w.topk, G)
+    cfg = lib.make_config(w.num_q_heads, w.num_kv_heads, w.rank, w.topk, w.dtype, flags=1)
+    lay = lib.HostLayout(data["seq_offsets"], data["q_seq"], data["q_visible"])
+    T = len(data["q_seq"])
+    idx_e = torch.empty((w.num_q_heads, T, w.topk), dtype=torch.int32, device="cuda")
+    rec = torch.empty((w.num_q_heads,), device="cuda")
+    lib.saki_recall(cfg, lay, w.topk + 1, to_dev(data["Q"], "f32"), f32(data["A"]), to_dev(data["K"], "f32"),
+                    torch.from_numpy(ia.astype(np.int32)).cuda(), rec, idx_exact=idx_e)
+    idx_e = idx_e.cpu().numpy()
+    waived = 0
+    for h in range(w.num_q_heads):
+        rows = [O.exact_scores(data["Q"][h, t], data["A"][h], data["K"][h // G, :data["q_visible"][t]])
+                for t in range(T)]
+        waived += check_topk_rows(idx_e[h], rows, w.topk, label=f"exact h{h}")[1]
+    ref_rec = O.head_recall(ia, ie, data["q_visible"], w.topk + 1, w.topk)
+    np.testing.assert_allclose(rec.cpu().numpy(), ref_rec, atol=RECALL_ABS + waived / (w.topk * (T - w.topk)))
+
+
+# --------------------------------------------------------------- end to end
+def test_end_to_end_tiny(lib, tiny):
+    """fit -> index -> select -> recall, all on the GPU, against the oracle chain."""
+    torch = _torch()
+    w, data, ref = tiny
+    G, T = w.group, len(data["q_seq"])
+    g = _gpu_fit(lib, w, data)
+    cfg = g["cfg"]
+    cfg.flags = 1
+    sk = torch.empty((w.num_q_heads, data["K"].shape[1], w.rank), device="cuda")
+    Kd = to_dev(data["K"], "f32")
+    lib.saki_build_index(cfg, Kd, f32(g["R"]), sk)
+    lay = lib.HostLayout(data["seq_offsets"], data["q_seq"], data["q_visible"])
+    idx = torch.empty((w.num_q_heads, T, w.topk), dtype=torch.int32, device="cuda")
+    Qd = to_dev(data["Q"], "f32")
+    lib.saki_score_topk(cfg, lay, Qd, f32(g["L"]), sk, idx)
+    rec = torch.empty((w.num_q_heads,), device="cuda")
+    lib.saki_recall(cfg, lay, w.topk + 1, Qd, f32(data["A"]), Kd, idx, rec)
+    sketch = O.build_index(data["K"], ref["R"], None, "f32", G)
+    ia, _ = O.score_topk(data["Q"], ref["L"], sketch, data["seq_offsets"], data["q_seq"], data["q_visible"], w.topk)
+    ie, _ = O.exact_topk(data["Q"], data["A"], data["K"], data["seq_offsets"], data["q_seq"], data["q_visible"],
+                         w.topk, G)
+    ref_rec = O.head_recall(ia, ie, data["q_visible"], w.topk + 1, w.topk)
+    np.testing.assert_allclose(rec.cpu().numpy(), ref_rec, atol=RECALL_ABS)
+    # the selected sets agree wherever the oracle's margin is clear
+    idx = idx.cpu().numpy()
+    for h in range(w.num_q_heads):
+        rows = [O.approx_scores(data["Q"][h, t], ref["L"][h], sketch[h, :data["q_visible"][t]]) for t in range(T)]
+        check_topk_rows(idx[h], rows, w.topk, label=f"e2e h{h}")
