@@ -23,9 +23,9 @@ template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
 template <> __device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
 
 // Keep the KP best of the warp's buffer (sorted, descending) and return the
-// k-th best key as the new acceptance threshold (0 while fewer than k).
+// k-th best key (0 while fewer than k are held).
 template <int KP>
-__device__ __forceinline__ void reselect(uint64_t* qb, int& cnt, uint64_t& thr, int k) {
+__device__ __forceinline__ uint64_t reselect(uint64_t* qb, int& cnt, int k) {
   constexpr int E = 2 * KP / 32;
   const int lane = threadIdx.x & 31;
   __syncwarp();
@@ -49,8 +49,31 @@ __device__ __forceinline__ void reselect(uint64_t* qb, int& cnt, uint64_t& thr, 
   for (int e = 0; e < E; ++e)
     if (e == ke) t = v[e];
   t = shfl_u64(t, (k - 1) & 31);
-  thr = cnt >= k ? t : 0ull;
   __syncwarp();
+  return cnt >= k ? t : 0ull;
+}
+
+// Rare path, kept out of line: append the passing keys of this 32-key batch to
+// the warp's buffer of one query, re-select when it is nearly full, publish the
+// warp's k-th best as a CTA-wide lower bound, and return the new threshold.
+template <int KP>
+__device__ __noinline__ uint64_t append_keys(uint64_t* qb, int* cnt_s, unsigned long long* cta_thr, uint64_t key,
+                                             bool pass, unsigned mask, uint64_t thr, int k) {
+  constexpr int CAP = 2 * KP;
+  const int lane = threadIdx.x & 31;
+  int cnt = *cnt_s;
+  if (pass) qb[cnt + __popc(mask & ((1u << lane) - 1u))] = key;
+  cnt += __popc(mask);
+  if (cnt > CAP - 32) {
+    const uint64_t t = reselect<KP>(qb, cnt, k);
+    if (t > thr) thr = t;
+    if (lane == 0 && t) atomicMax(cta_thr, (unsigned long long)t);
+  }
+  __syncwarp();
+  if (lane == 0) *cnt_s = cnt;
+  __syncwarp();
+  const uint64_t c = *cta_thr;
+  return c > thr ? c : thr;
 }
 
 template <typename Tin, int KP>
@@ -64,6 +87,8 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
   float* us = qs + kGroupQ * kD;                                           // [GQ][P]
   float* qnu = us + kGroupQ * a.P;                                         // [GQ]
   int* visq = reinterpret_cast<int*>(qnu + kGroupQ);                       // [GQ]
+  int* cnt_s = visq + kGroupQ;                                             // [warps][GQ]
+  __shared__ unsigned long long cta_thr[kGroupQ];
 
   const ScoreItem it = a.items[blockIdx.x];
   const int h = blockIdx.y;
@@ -76,7 +101,11 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
     const int b = o / kD;
     qs[o] = b < nq ? to_f<Tin>(Q[((int64_t)h * a.T + it.q_begin + b) * kD + (o % kD)]) : 0.f;
   }
-  if (tid < kGroupQ) visq[tid] = tid < nq ? a.vis[it.q_begin + tid] : 0;
+  if (tid < kGroupQ) {
+    visq[tid] = tid < nq ? a.vis[it.q_begin + tid] : 0;
+    cta_thr[tid] = 0ull;
+  }
+  if (tid < kWarps * kGroupQ) cnt_s[tid] = 0;
   for (int o = tid; o < kWarps * kGroupQ * CAP; o += kThreads) buf[o] = 0ull;
   __syncthreads();
 
@@ -100,13 +129,12 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
   const Tin* X = static_cast<const Tin*>(a.X) +
                  ((int64_t)(a.exact ? h / a.G : h) * a.N + it.key_base) * P;
   uint64_t thr[kGroupQ];
-  int cnt[kGroupQ];
 #pragma unroll
-  for (int b = 0; b < kGroupQ; ++b) { thr[b] = 0ull; cnt[b] = 0; }
+  for (int b = 0; b < kGroupQ; ++b) thr[b] = 0ull;
   uint64_t* wbuf = buf + warp * kGroupQ * CAP;
+  int* wcnt = cnt_s + warp * kGroupQ;
   const int nkeys = it.key_hi - it.key_lo;
   const bool vec = ((P * (int)sizeof(Tin)) % 16) == 0;
-  const unsigned lt_mask = (1u << lane) - 1u;
 
   for (int base = warp * 32; base < nkeys; base += kThreads) {
     const int jl = base + lane;
@@ -151,18 +179,14 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
         const uint64_t key = make_key(acc[b], (uint32_t)j);
         const bool pass = ok && key > thr[b];
         const unsigned mask = __ballot_sync(0xffffffffu, pass);
-        if (mask) {
-          uint64_t* qb = wbuf + b * CAP;
-          if (pass) qb[cnt[b] + __popc(mask & lt_mask)] = key;
-          cnt[b] += __popc(mask);
-          if (cnt[b] > CAP - 32) reselect<KP>(qb, cnt[b], thr[b], a.k);
-        }
+        if (mask) thr[b] = append_keys<KP>(wbuf + b * CAP, wcnt + b, cta_thr + b, key, pass, mask, thr[b], a.k);
       }
     }
   }
-#pragma unroll
-  for (int b = 0; b < kGroupQ; ++b)
-    if (b < nq) reselect<KP>(wbuf + b * CAP, cnt[b], thr[b], a.k);
+  for (int b = 0; b < nq; ++b) {
+    int c = wcnt[b];
+    reselect<KP>(wbuf + b * CAP, c, a.k);
+  }
   __syncthreads();
 
   // merge the warps' lists of query `warp`
@@ -241,7 +265,7 @@ cudaError_t launch_score_t(const ScoreArgs& a, cudaStream_t s) {
 
 size_t score_generic_smem(int P, int kp) {
   return sizeof(uint64_t) * (size_t)kWarps * kGroupQ * 2 * kp +
-         sizeof(float) * (size_t)(kGroupQ * kD + kGroupQ * P + kGroupQ) + sizeof(int) * kGroupQ;
+         sizeof(float) * (size_t)(kGroupQ * kD + kGroupQ * P + kGroupQ) + sizeof(int) * (kGroupQ + kWarps * kGroupQ);
 }
 
 cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, cudaStream_t s) {
