@@ -164,6 +164,32 @@ SAKI_API saki_status saki_recall(const saki_config* cfg, const saki_layout* layo
                         int32_t* idx_exact, float* recall, void* workspace,
                         size_t workspace_bytes, saki_stream stream);
 
+/* Bytes of the static device scratch array behind saki_score_topk_noalloc. */
+#define SAKI_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/* saki_score_topk_noalloc -- the paper has no counterpart; this is a library
+ * convenience.  Same arguments, semantics and results as saki_score_topk, minus
+ * the workspace, for callers that cannot call cudaMalloc: for example a plugin
+ * running inside a serving framework whose allocator owns all device memory, or
+ * a decode loop that must not allocate because cudaMalloc can synchronise the
+ * device.  Its scratch is a static device array of SAKI_NOALLOC_SCRATCH_BYTES
+ * inside the library, held by every GPU that loads the library until the
+ * process exits; nothing is allocated per call.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ *   - A layout whose work plan needs more than SAKI_NOALLOC_SCRATCH_BYTES
+ *     (saki_workspace_size with SAKI_OP_SCORE_TOPK reports the need) is rejected
+ *     with SAKI_ERR_WORKSPACE before any launch.
+ *   - Every call shares the one array and it keeps the last call's contents;
+ *     each call rewrites everything it later reads, so nothing needs clearing,
+ *     but calls that overlap on the GPU (other streams, other host threads)
+ *     race on it: serialise them. */
+SAKI_API saki_status saki_score_topk_noalloc(const saki_config* cfg, const saki_layout* layout,
+                                             const void* Q, const float* L, const void* sketch,
+                                             const float* nu, int32_t* idx, float* score,
+                                             saki_stream stream);
+
 /* Static description of a status code. */
 SAKI_API const char* saki_status_string(saki_status status);
 

@@ -24,7 +24,8 @@ SAKI_OP_FIT, SAKI_OP_BUILD_INDEX, SAKI_OP_SCORE_TOPK, SAKI_OP_RECALL = 0, 1, 2, 
 STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED", 3: "SAKI_ERR_CUDA",
           4: "SAKI_ERR_NUMERIC", 5: "SAKI_ERR_NOT_CONVERGED", 6: "SAKI_ERR_WORKSPACE", 7: "SAKI_ERR_TIMEOUT"}
 EXPORTS = ("saki_workspace_size", "saki_fit", "saki_build_index", "saki_score_topk", "saki_recall",
-           "saki_status_string", "saki_version")
+           "saki_status_string", "saki_version", "saki_score_topk_noalloc")
+SAKI_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 class Config(ctypes.Structure):
@@ -50,6 +51,8 @@ _lib.saki_score_topk.restype = ctypes.c_int
 _lib.saki_score_topk.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout)] + [_vp] * 7 + [_sz, _vp]
 _lib.saki_recall.restype = ctypes.c_int
 _lib.saki_recall.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout), _i64] + [_vp] * 7 + [_sz, _vp]
+_lib.saki_score_topk_noalloc.restype = ctypes.c_int
+_lib.saki_score_topk_noalloc.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout)] + [_vp] * 6 + [_vp]
 _lib.saki_status_string.restype = ctypes.c_char_p
 _lib.saki_status_string.argtypes = [ctypes.c_int]
 _lib.saki_version.restype = ctypes.c_char_p
@@ -159,3 +162,11 @@ def saki_recall(cfg: Config, layout: HostLayout, min_visible: int, Q, A, K, idx_
     _check(_lib.saki_recall(ctypes.byref(cfg), ctypes.byref(layout.c), min_visible, _ptr(Q), _ptr(A), _ptr(K),
                             _ptr(idx_approx), _ptr(idx_exact), _ptr(recall), _ptr(ws), ws.numel(), _stream(stream)),
            "saki_recall")
+
+
+def saki_score_topk_noalloc(cfg: Config, layout: HostLayout, Q, L, sketch, idx, score=None, nu=None, stream=None):
+    """saki_score_topk without a workspace: the library's static device scratch
+    serves instead (for callers that cannot allocate device memory)."""
+    _check(_lib.saki_score_topk_noalloc(ctypes.byref(cfg), ctypes.byref(layout.c), _ptr(Q), _ptr(L), _ptr(sketch),
+                                        _ptr(nu), _ptr(idx), _ptr(score), _stream(stream)),
+           "saki_score_topk_noalloc")
