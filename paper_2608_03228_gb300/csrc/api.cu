@@ -16,6 +16,7 @@ namespace {
 constexpr size_t kAlign = 256;
 constexpr int kNumSMs = 152;
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+inline saki_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA; }
 inline bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline int kp_of(int k) { return k <= 64 ? 64 : 128; }
 
@@ -124,6 +125,108 @@ saki_status upload_plan(const Plan& p, char* ws, cudaStream_t s) {
                                                                                               : SAKI_ERR_CUDA;
 }
 
+// Tensor-core plan: tiles of up to 128 consecutive queries of one sequence,
+// heaviest first; the workspace holds the tiles, the visible counts, the error
+// word, the exact three-way bf16 split of the projection and the mean terms.
+struct TcPlan {
+  std::vector<TcTile> tiles;
+  std::vector<int32_t> vis;
+  size_t off_vis = 0, off_err = 0, staged = 0, off_w = 0, off_qnu = 0, bytes = 0;
+};
+
+TcPlan make_tc_plan(const saki_layout* L, int Hq, int P, bool with_qnu) {
+  TcPlan p;
+  const int64_t T = L->num_queries;
+  for (int64_t t = 0; t < T;) {
+    TcTile tl{(int32_t)t, 0, L->seq_offsets[L->q_seq[t]], 0, 0};
+    const int32_t seq = L->q_seq[t];
+    while (t < T && L->q_seq[t] == seq && tl.nrows < 128) {
+      tl.vis_max = std::max<int32_t>(tl.vis_max, (int32_t)L->q_visible[t]);
+      ++tl.nrows;
+      ++t;
+    }
+    p.tiles.push_back(tl);
+  }
+  std::stable_sort(p.tiles.begin(), p.tiles.end(),
+                   [](const TcTile& a, const TcTile& b) { return a.vis_max > b.vis_max; });
+  p.vis.resize(T);
+  for (int64_t t = 0; t < T; ++t) p.vis[t] = (int32_t)L->q_visible[t];
+  p.off_vis = align_up(p.tiles.size() * sizeof(TcTile));
+  p.off_err = p.off_vis + align_up(p.vis.size() * sizeof(int32_t));
+  p.staged = p.off_err + sizeof(int);
+  p.off_w = align_up(p.staged);
+  p.off_qnu = p.off_w + align_up((size_t)Hq * 3 * P * kD * 2);
+  p.bytes = p.off_qnu + (with_qnu ? align_up((size_t)Hq * T * sizeof(float)) : 0);
+  return p;
+}
+
+// The tensor-core kernel serves bf16 data, K widths 16/32/64/128, k <= 64, and
+// layouts whose query tiles average at least 32 rows (prefill-like); decode-like
+// layouts (a few queries per sequence) go to the CUDA-core kernel.
+bool use_tc(const saki_config* c, const saki_layout* L, int P) {
+  if (c->dtype != SAKI_BF16 || !tc_supported(P) || c->topk > 64 || L->num_queries == 0) return false;
+  int64_t tiles = 0;
+  for (int64_t t = 0; t < L->num_queries;) {
+    const int32_t seq = L->q_seq[t];
+    int n = 0;
+    while (t < L->num_queries && L->q_seq[t] == seq && n < 128) { ++n; ++t; }
+    ++tiles;
+  }
+  return L->num_queries >= 32 * tiles;
+}
+
+saki_status upload_tc_plan(const TcPlan& p, char* ws, cudaStream_t s) {
+  std::vector<char> host(p.staged, 0);
+  if (!p.tiles.empty()) std::memcpy(host.data(), p.tiles.data(), p.tiles.size() * sizeof(TcTile));
+  if (!p.vis.empty()) std::memcpy(host.data() + p.off_vis, p.vis.data(), p.vis.size() * sizeof(int32_t));
+  return cudaMemcpyAsync(ws, host.data(), p.staged, cudaMemcpyHostToDevice, s) == cudaSuccess ? SAKI_OK
+                                                                                              : SAKI_ERR_CUDA;
+}
+
+int num_sms() {
+  int dev = 0, n = kNumSMs;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : kNumSMs;
+}
+
+// Run the tensor-core selection: W is L (approximate, X = codes) or A (exact, X = keys).
+saki_status run_tc(const saki_config* cfg, const saki_layout* layout, const TcPlan& p, int P, bool exact,
+                   const void* Q, const float* W, const void* X, const float* nu, int32_t* idx, float* score,
+                   char* ws, cudaStream_t s) {
+  saki_status st = upload_tc_plan(p, ws, s);
+  if (st != SAKI_OK) return st;
+  void* wsplit = ws + p.off_w;
+  if (launch_pack_w(W, cfg->num_q_heads, P, wsplit, s) != cudaSuccess) return SAKI_ERR_CUDA;
+  float* qnu = nullptr;
+  if (nu && score) {
+    qnu = reinterpret_cast<float*>(ws + p.off_qnu);
+    if (launch_qnu(Q, nu, layout->num_queries, cfg->num_q_heads, qnu, s) != cudaSuccess) return SAKI_ERR_CUDA;
+  }
+  TcLaunch L{};
+  L.Q = Q;
+  L.X = X;
+  L.Wsplit = wsplit;
+  L.P = P;
+  L.Hk = cfg->num_kv_heads;
+  L.num_sms = num_sms();
+  TcArgs& a = L.args;
+  a.tiles = reinterpret_cast<const TcTile*>(ws);
+  a.vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
+  a.qnu = qnu;
+  a.idx = idx;
+  a.score = score;
+  a.err = reinterpret_cast<int*>(ws + p.off_err);
+  a.T = layout->num_queries;
+  a.N = layout->seq_offsets[layout->num_seqs];
+  a.n_items = (int32_t)(p.tiles.size() * cfg->num_q_heads);
+  a.Hq = cfg->num_q_heads;
+  a.G = cfg->num_q_heads / cfg->num_kv_heads;
+  a.k = cfg->topk;
+  a.exact = exact ? 1 : 0;
+  a.sorted = (cfg->flags & SAKI_FLAG_SORTED) ? 1 : 0;
+  return cuda_status(launch_score_tc(L, s));
+}
+
 // fit workspace: S, F, G [(Hq+Hk)][d][d], mu [Hk][d], status [Hq+Hk]
 struct FitWs { size_t S, F, G, mu, st, bytes; };
 FitWs fit_ws(const saki_config* c) {
@@ -143,8 +246,6 @@ size_t recall_extra(const saki_config* c, int64_t T, bool with_idx) {
   return align_up((size_t)c->num_q_heads * 2 * sizeof(unsigned long long)) +
          (with_idx ? align_up((size_t)c->num_q_heads * T * c->topk * sizeof(int32_t)) : 0);
 }
-
-inline saki_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA; }
 
 }  // namespace
 
@@ -178,8 +279,12 @@ size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout
     case SAKI_OP_RECALL: {
       int64_t n = 0;
       if (check_layout(layout, &n) != SAKI_OK) return 0;
-      const Plan p = make_plan(layout, cfg->num_q_heads, kp_of(cfg->topk));
-      size_t b = p.bytes;
+      const int P = op == SAKI_OP_RECALL ? kD : cfg->rank;
+      size_t b;
+      if (use_tc(cfg, layout, P))
+        b = make_tc_plan(layout, cfg->num_q_heads, P, op == SAKI_OP_SCORE_TOPK).bytes;
+      else
+        b = make_plan(layout, cfg->num_q_heads, kp_of(cfg->topk)).bytes;
       if (op == SAKI_OP_RECALL) b += recall_extra(cfg, layout->num_queries, true);
       return b;
     }
@@ -258,11 +363,16 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
                         (const void*)workspace})
     if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
   if (T == 0) return SAKI_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  if (use_tc(cfg, layout, cfg->rank)) {
+    const TcPlan tp = make_tc_plan(layout, cfg->num_q_heads, cfg->rank, true);
+    if (workspace_bytes < tp.bytes) return SAKI_ERR_WORKSPACE;
+    return run_tc(cfg, layout, tp, cfg->rank, false, Q, L, sketch, nu, idx, score, ws, s);
+  }
   const int kp = kp_of(cfg->topk);
   const Plan p = make_plan(layout, cfg->num_q_heads, kp);
   if (workspace_bytes < p.bytes) return SAKI_ERR_WORKSPACE;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  char* ws = static_cast<char*>(workspace);
   if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
   ScoreArgs a{};
   a.Q = Q; a.X = sketch; a.W = L; a.nu = nu;
@@ -294,15 +404,23 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
                         (const void*)workspace})
     if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
   const int kp = kp_of(cfg->topk);
-  const Plan p = make_plan(layout, cfg->num_q_heads, kp);
-  const size_t need = p.bytes + recall_extra(cfg, T, idx_exact == nullptr);
+  const bool tc = use_tc(cfg, layout, kD);
+  const Plan p = tc ? Plan{} : make_plan(layout, cfg->num_q_heads, kp);
+  const TcPlan tp = tc ? make_tc_plan(layout, cfg->num_q_heads, kD, false) : TcPlan{};
+  const size_t base = tc ? tp.bytes : p.bytes;
+  const size_t need = base + recall_extra(cfg, T, idx_exact == nullptr);
   if (workspace_bytes < need) return SAKI_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
-  unsigned long long* counters = reinterpret_cast<unsigned long long*>(ws + p.bytes);
+  unsigned long long* counters = reinterpret_cast<unsigned long long*>(ws + base);
   int32_t* ie = idx_exact ? idx_exact
-                          : reinterpret_cast<int32_t*>(ws + p.bytes + align_up((size_t)cfg->num_q_heads * 2 *
-                                                                               sizeof(unsigned long long)));
+                          : reinterpret_cast<int32_t*>(ws + base + align_up((size_t)cfg->num_q_heads * 2 *
+                                                                            sizeof(unsigned long long)));
+  if (tc) {
+    if ((st = run_tc(cfg, layout, tp, kD, true, Q, A, K, nullptr, ie, nullptr, ws, s)) != SAKI_OK) return st;
+    return cuda_status(launch_recall(idx_approx, ie, reinterpret_cast<const int32_t*>(ws + tp.off_vis), T,
+                                     cfg->num_q_heads, cfg->topk, min_visible, counters, recall, s));
+  }
   if (T > 0) {
     if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
     ScoreArgs a{};

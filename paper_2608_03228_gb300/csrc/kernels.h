@@ -72,4 +72,39 @@ cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int3
                           int64_t T, int Hq, int k, int64_t min_visible,
                           unsigned long long* counters, float* recall, cudaStream_t s);
 
+// ---------------------------------------------------------------- tensor-core path
+// A tile: up to 128 consecutive queries of one sequence, ranked against that
+// sequence's first vis_max keys (each row against its own visible prefix).
+struct TcTile {
+  int32_t q0;
+  int32_t nrows;
+  int64_t key_base;
+  int32_t vis_max;
+  int32_t pad;
+};
+
+struct TcArgs {
+  const TcTile* tiles;
+  const int32_t* vis;   // [T]
+  const float* qnu;     // [Hq][T] mean term added to reported scores, or null
+  int32_t* idx;         // [Hq][T][k]
+  float* score;         // [Hq][T][k] or null
+  int* err;             // set to 1 if a bounded wait gave up
+  int64_t T, N;
+  int32_t n_items, Hq, G, k, exact, sorted;
+};
+
+struct TcLaunch {
+  const void* Q;        // [Hq][T][d] bf16
+  const void* X;        // codes [Hq][N][P] (approximate) or keys [Hk][N][d] (exact), bf16
+  const void* Wsplit;   // [Hq][3][P][d] bf16 from launch_pack_w
+  int P, Hk, num_sms;
+  TcArgs args;
+};
+
+bool tc_supported(int P);
+cudaError_t launch_pack_w(const float* W, int Hq, int P, void* out, cudaStream_t s);
+cudaError_t launch_qnu(const void* Q, const float* nu, int64_t T, int Hq, float* out, cudaStream_t s);
+cudaError_t launch_score_tc(const TcLaunch& L, cudaStream_t s);
+
 }  // namespace saki
