@@ -160,11 +160,13 @@ TcPlan make_tc_plan(const saki_layout* L, int Hq, int P, bool with_qnu) {
   return p;
 }
 
-// The tensor-core kernel serves bf16 data, K widths 16/32/64/128, k <= 64, and
-// layouts whose query tiles average at least 32 rows (prefill-like); decode-like
-// layouts (a few queries per sequence) go to the CUDA-core kernel.
+// The tensor-core kernel serves bf16 data, K widths 16/32/64/128, k <= 64, queries
+// that see at most 65535 keys, and layouts whose query tiles average at least 32
+// rows (prefill-like); everything else goes to the CUDA-core kernel.
 bool use_tc(const saki_config* c, const saki_layout* L, int P) {
   if (c->dtype != SAKI_BF16 || !tc_supported(P) || c->topk > 64 || L->num_queries == 0) return false;
+  for (int64_t t = 0; t < L->num_queries; ++t)
+    if (L->q_visible[t] > 65535) return false;   // candidate lists hold 16-bit key offsets
   int64_t tiles = 0;
   for (int64_t t = 0; t < L->num_queries;) {
     const int32_t seq = L->q_seq[t];

@@ -38,7 +38,7 @@ template <int P>
 struct TcCfg {
   static constexpr int NT = P == 128 ? 128 : 256;            // keys per tile (MMA N)
   static constexpr int STAGES = P <= 32 ? 4 : 2;
-  static constexpr int CAP = P == 128 ? 96 : 128;             // candidate slots per row
+  static constexpr int CAP = P == 128 ? 128 : (P == 16 ? 208 : 168);   // candidate slots per row
   static constexpr int KB = P == 128 ? 2 : 1;                 // 64-wide K blocks
   static constexpr int KW = P == 128 ? 64 : P;                // K width of one block
   static constexpr int KK = KW / 16;                          // MMA K steps per block
@@ -47,7 +47,7 @@ struct TcCfg {
   static constexpr int A_PART = 128 * P * 2;                  // u_hi (or u_lo) bytes
   static constexpr int A_BYTES = 2 * A_PART > 32768 ? 2 * A_PART : 32768;  // also holds the 128x128 query tile
   static constexpr int STAGE_BYTES = NT * P * 2;
-  static constexpr int CAND_BYTES = CAP * kLdc * 4 * 2;
+  static constexpr int CAND_BYTES = CAP * kLdc * 4 + ((CAP * kLdc * 2 + 15) & ~15);
   static constexpr int TMEM_COLS = 2 * NT;
   static constexpr int OFF_STAGE = A_BYTES;
   static constexpr int OFF_CAND = OFF_STAGE + STAGES * STAGE_BYTES;
@@ -60,38 +60,105 @@ struct TcCfg {
 __device__ __forceinline__ float fmax3(float a, float b, float c) { return fmaxf(a, fmaxf(b, c)); }
 
 // ---------------------------------------------------------------- selection
+// A row's candidate column: scores (fp32) and key indices (16-bit; the host only
+// sends sequences of at most 65535 keys here).
 struct Col {
   float* bs;
-  int* bi;
+  uint16_t* bi;
   int row;
   __device__ __forceinline__ float s(int i) const { return bs[i * kLdc + row]; }
   __device__ __forceinline__ int j(int i) const { return bi[i * kLdc + row]; }
   __device__ __forceinline__ void put(int i, float v, int k) const {
     bs[i * kLdc + row] = v;
-    bi[i * kLdc + row] = k;
+    bi[i * kLdc + row] = (uint16_t)k;
   }
 };
 
+// The passes below keep eight independent shared-memory loads in flight per
+// thread: a row's column is scanned with no other parallelism, so latency, not
+// bandwidth, bounds them.
+
+// Number of entries scoring >= p.
+__device__ __forceinline__ int count_ge(const Col& c, int cnt, float p) {
+  int n0 = 0, n1 = 0, i = 0;
+  for (; i + 8 <= cnt; i += 8) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = c.s(i + u);
+#pragma unroll
+    for (int u = 0; u < 8; u += 2) {
+      n0 += v[u] >= p;
+      n1 += v[u + 1] >= p;
+    }
+  }
+  for (; i < cnt; ++i) n0 += c.s(i) >= p;
+  return n0 + n1;
+}
+
+// Keep the entries scoring >= p (in place, order preserved); returns their count.
+__device__ __forceinline__ int compact_ge(const Col& c, int cnt, float p) {
+  int w = 0, i = 0;
+  for (; i + 8 <= cnt; i += 8) {
+    float v[8];
+    int j[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      v[u] = c.s(i + u);
+      j[u] = c.j(i + u);
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (v[u] >= p) {
+        c.put(w, v[u], j[u]);
+        ++w;
+      }
+  }
+  for (; i < cnt; ++i) {
+    const float v = c.s(i);
+    if (v >= p) {
+      c.put(w, v, c.j(i));
+      ++w;
+    }
+  }
+  return w;
+}
+
+// (score, index) worse-than: lower score, or equal score and higher index.
+__device__ __forceinline__ bool worse(float a, int ja, float b, int jb) { return a < b || (a == b && ja > jb); }
+
 // Remove the worst entry (lowest score, then highest index); raise thr to its score.
 __device__ __forceinline__ void remove_worst(const Col& c, int& cnt, float& thr) {
-  int w = 0;
-  float ws = c.s(0);
-  int wj = c.j(0);
-  for (int i = 1; i < cnt; ++i) {
+  float ws[4];
+  int wj[4], wp[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) { ws[u] = INFINITY; wj[u] = -1; wp[u] = 0; }
+  int i = 0;
+  for (; i + 4 <= cnt; i += 4) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float v = c.s(i + u);
+      const int jj = c.j(i + u);
+      if (worse(v, jj, ws[u], wj[u])) { ws[u] = v; wj[u] = jj; wp[u] = i + u; }
+    }
+  }
+  for (; i < cnt; ++i) {
     const float v = c.s(i);
     const int jj = c.j(i);
-    if (v < ws || (v == ws && jj > wj)) { ws = v; wj = jj; w = i; }
+    if (worse(v, jj, ws[0], wj[0])) { ws[0] = v; wj[0] = jj; wp[0] = i; }
   }
+#pragma unroll
+  for (int u = 1; u < 4; ++u)
+    if (worse(ws[u], wj[u], ws[0], wj[0])) { ws[0] = ws[u]; wj[0] = wj[u]; wp[0] = wp[u]; }
   --cnt;
-  c.put(w, c.s(cnt), c.j(cnt));
-  thr = fmaxf(thr, ws);
+  c.put(wp[0], c.s(cnt), c.j(cnt));
+  thr = fmaxf(thr, ws[0]);
 }
 
 // Keep every entry scoring >= a sampled pivot p, provided at least k and at most
 // tmax remain; the threshold becomes p (all later keys have higher indices, so a
 // key scoring exactly p loses to all kept entries).  Returns false if no tried
 // pivot qualifies.
-__device__ __noinline__ bool pivot_round(const Col& c, int& cnt, float& thr, int k, int aim, int tmax) {
+__device__ __forceinline__ bool pivot_round(const Col& c, int& cnt, float& thr, int k, int aim, int tmax) {
   float s[8];
 #pragma unroll
   for (int u = 0; u < 8; ++u) s[u] = c.s(((2 * u + 1) * cnt) >> 4);
@@ -115,18 +182,9 @@ __device__ __noinline__ bool pivot_round(const Col& c, int& cnt, float& thr, int
 #pragma unroll
     for (int u = 1; u < 8; ++u)
       if (u == q) p = s[u];
-    int n = 0;
-    for (int i = 0; i < cnt; ++i) n += c.s(i) >= p;
+    const int n = count_ge(c, cnt, p);
     if (n >= k && n <= tmax) {
-      int w = 0;
-      for (int i = 0; i < cnt; ++i) {
-        const float v = c.s(i);
-        if (v >= p) {
-          c.put(w, v, c.j(i));
-          ++w;
-        }
-      }
-      cnt = w;
+      cnt = compact_ge(c, cnt, p);
       thr = fmaxf(thr, p);
       return true;
     }
@@ -141,25 +199,34 @@ __device__ __noinline__ bool pivot_round(const Col& c, int& cnt, float& thr, int
   return false;
 }
 
-// Make room: bring cnt down to at most tmax (>= k) without losing the row's top k.
-__device__ __noinline__ void shrink(const Col& c, int& cnt, float& thr, int k, int tmax) {
-  if (!pivot_round(c, cnt, thr, k, (k + tmax) >> 1, tmax))
-    while (cnt > tmax) remove_worst(c, cnt, thr);
+// Warp-wide room making, run at a convergent point whenever any lane of the warp
+// has more than tmax candidates: every lane holding more than lo = (k + tmax)/2
+// shrinks at the same time (one pivot round for the whole warp instead of one per
+// lane, and the lanes' fill levels stay in step).  Lanes above tmax are brought
+// to at most tmax in every case; the row's top k is never dropped.
+__device__ __forceinline__ void shrink_warp(const Col& c, int& cnt, float& thr, int k, int tmax) {
+  const int lo = (k + tmax) >> 1;
+  if (cnt > lo) {
+    if (!pivot_round(c, cnt, thr, k, k + ((tmax - k) >> 3), lo) && cnt > tmax)
+      while (cnt > tmax) remove_worst(c, cnt, thr);
+  }
 }
 
 // Exactly the k best (or all, if fewer).
-__device__ __noinline__ void finalize(const Col& c, int& cnt, float& thr, int k) {
+__device__ __forceinline__ void finalize(const Col& c, int& cnt, float& thr, int k) {
   for (int guard = 0; cnt - k > 12 && guard < 4; ++guard)
     if (!pivot_round(c, cnt, thr, k, k + 4, cnt - 1)) break;
   while (cnt > k) remove_worst(c, cnt, thr);
 }
 
-// 16 scores of one row: mask keys the row cannot see, append the ones above thr.
-template <int CAP>
-__device__ __forceinline__ void take16(const uint32_t* r, int j0, int vis, const Col& c, int& cnt, float& thr, int k) {
+// 16 scores of one row (register offset OFF of a 32-score load): mask the keys
+// the row cannot see and append the ones above thr (lanes diverge here).
+template <int OFF>
+__device__ __forceinline__ void append16(const uint32_t (&r)[32], int j0, int vis, const Col& c, int& cnt,
+                                         float thr) {
   float v[16];
 #pragma unroll
-  for (int u = 0; u < 16; ++u) v[u] = __uint_as_float(r[u]);
+  for (int u = 0; u < 16; ++u) v[u] = __uint_as_float(r[OFF + u]);
   if (j0 + 16 > vis) {
 #pragma unroll
     for (int u = 0; u < 16; ++u)
@@ -168,15 +235,24 @@ __device__ __forceinline__ void take16(const uint32_t* r, int j0, int vis, const
   const float m = fmaxf(fmax3(fmax3(v[0], v[1], v[2]), fmax3(v[3], v[4], v[5]), fmax3(v[6], v[7], v[8])),
                         fmax3(fmax3(v[9], v[10], v[11]), fmax3(v[12], v[13], v[14]), v[15]));
   if (m > thr) {
+    // branch-free: write every key at the next free slot, advance only past
+    // the ones above thr (the slot stays in bounds: cnt <= CAP - 16 on entry)
 #pragma unroll
     for (int u = 0; u < 16; ++u) {
-      if (v[u] > thr) {
-        c.put(cnt, v[u], j0 + u);
-        ++cnt;
-      }
+      c.put(cnt, v[u], j0 + u);
+      cnt += v[u] > thr ? 1 : 0;
     }
-    if (cnt > CAP - 16) shrink(c, cnt, thr, k, CAP - 16);
   }
+}
+
+// 32 scores of one row; the capacity check runs with the whole warp converged.
+template <int CAP>
+__device__ __forceinline__ void take32(const uint32_t (&r)[32], int j0, int vis, const Col& c, int& cnt, float& thr,
+                                       int k) {
+  append16<0>(r, j0, vis, c, cnt, thr);
+  if (__any_sync(0xffffffffu, cnt > CAP - 16)) shrink_warp(c, cnt, thr, k, CAP - 16);
+  append16<16>(r, j0 + 16, vis, c, cnt, thr);
+  if (__any_sync(0xffffffffu, cnt > CAP - 16)) shrink_warp(c, cnt, thr, k, CAP - 16);
 }
 
 template <int P>
@@ -239,11 +315,13 @@ __global__ void __launch_bounds__(192, 1)
                     const __grid_constant__ CUtensorMap tmX, const TcArgs a) {
   using C = TcCfg<P>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // align by pointer arithmetic on the shared array, so the compiler keeps
+  // treating every derived pointer as shared memory
+  uint8_t* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
   uint8_t* sA = smem;
   uint8_t* sStage = smem + C::OFF_STAGE;
   float* bs = reinterpret_cast<float*>(smem + C::OFF_CAND);
-  int* bi = reinterpret_cast<int*>(smem + C::OFF_CAND + C::CAP * kLdc * 4);
+  uint16_t* bi = reinterpret_cast<uint16_t*>(smem + C::OFF_CAND + C::CAP * kLdc * 4);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* empty = full + C::STAGES;
   uint64_t* accf = empty + C::STAGES;
@@ -441,8 +519,7 @@ __global__ void __launch_bounds__(192, 1)
             tc::mbar_arrive(acce + buf);
           }
           const int j0 = i * C::NT + c * 32;
-          take16<C::CAP>(r, j0, vis, col, cnt, thr, a.k);
-          take16<C::CAP>(r + 16, j0 + 16, vis, col, cnt, thr, a.k);
+          take32<C::CAP>(r, j0, vis, col, cnt, thr, a.k);
         }
         ++ac;
       }
