@@ -229,6 +229,27 @@ saki_status run_tc(const saki_config* cfg, const saki_layout* layout, const TcPl
   return cuda_status(launch_score_tc(L, s));
 }
 
+// Index build on the tensor cores: bf16 data, uncentered keys (codes of centered
+// keys keep the CUDA-core path, which subtracts mu before the products), r a
+// multiple of 16 dividing 128.  Items: (KV head, 128-column block, 32 key tiles).
+struct BuildWs { std::vector<BuildItem> items; size_t off_err, off_w, bytes; bool tc; };
+BuildWs build_ws(const saki_config* c, int64_t N) {
+  BuildWs w{};
+  const int G = c->num_q_heads / c->num_kv_heads;
+  w.tc = c->dtype == SAKI_BF16 && !c->center && build_tc_supported(c->rank, G) && N > 0;
+  if (!w.tc) { w.bytes = kAlign; return w; }
+  const int ncb = (G * c->rank + 127) / 128;
+  const int64_t tiles = (N + 127) / 128;
+  for (int g = 0; g < c->num_kv_heads; ++g)
+    for (int cb = 0; cb < ncb; ++cb)
+      for (int64_t t = 0; t < tiles; t += 32)
+        w.items.push_back(BuildItem{g, cb, (int32_t)t, (int32_t)std::min<int64_t>(tiles, t + 32)});
+  w.off_err = align_up(w.items.size() * sizeof(BuildItem));
+  w.off_w = w.off_err + kAlign;
+  w.bytes = w.off_w + align_up(build_tc_workspace(c->num_q_heads, c->rank));
+  return w;
+}
+
 // fit workspace: S, F, G [(Hq+Hk)][d][d], mu [Hk][d], status [Hq+Hk]
 struct FitWs { size_t S, F, G, mu, st, bytes; };
 FitWs fit_ws(const saki_config* c) {
@@ -276,7 +297,7 @@ size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout
     case SAKI_OP_FIT:
       return n_calib >= 1 ? fit_ws(cfg).bytes : 0;
     case SAKI_OP_BUILD_INDEX:
-      return total_keys >= 0 ? kAlign : 0;
+      return total_keys >= 0 ? build_ws(cfg, total_keys).bytes : 0;
     case SAKI_OP_SCORE_TOPK:
     case SAKI_OP_RECALL: {
       int64_t n = 0;
@@ -344,9 +365,21 @@ saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const v
   if (cfg->center && !mu) return SAKI_ERR_INVALID_ARGUMENT;
   for (const void* p : {K, (const void*)R, (const void*)mu, (const void*)sketch})
     if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
-  (void)workspace;
-  (void)workspace_bytes;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const BuildWs w = build_ws(cfg, total_keys);
+  if (w.tc) {
+    if (!workspace) return SAKI_ERR_INVALID_ARGUMENT;
+    if (workspace_bytes < w.bytes) return SAKI_ERR_WORKSPACE;
+    char* ws = static_cast<char*>(workspace);
+    std::vector<char> host(w.off_w, 0);
+    std::memcpy(host.data(), w.items.data(), w.items.size() * sizeof(BuildItem));
+    if ((st = cuda_status(cudaMemcpyAsync(ws, host.data(), host.size(), cudaMemcpyHostToDevice, s))) != SAKI_OK)
+      return st;
+    return cuda_status(launch_build_tc(K, R, sketch, total_keys, cfg->num_q_heads,
+                                       cfg->num_q_heads / cfg->num_kv_heads, cfg->rank,
+                                       reinterpret_cast<const BuildItem*>(ws), (int)w.items.size(), ws + w.off_w,
+                                       reinterpret_cast<int*>(ws + w.off_err), num_sms(), s));
+  }
   return cuda_status(launch_build_generic(K, R, cfg->center ? mu : nullptr, sketch, total_keys, cfg->num_q_heads,
                                           cfg->num_q_heads / cfg->num_kv_heads, cfg->rank, cfg->center,
                                           cfg->dtype, s));

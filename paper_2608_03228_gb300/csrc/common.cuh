@@ -45,6 +45,12 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(f
   return __float2bfloat16_rn(v);
 }
 
+// Two floats rounded to bf16 (nearest even), packed low element first.
+__device__ __forceinline__ uint32_t pack_bf16_pair(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
 // ---------------------------------------------------------------- ranking keys
 // A 64-bit key orders candidates by (score descending, index ascending): the high
 // word is an order-preserving image of the float score (with -0 folded onto +0),

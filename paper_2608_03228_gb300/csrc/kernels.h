@@ -107,4 +107,16 @@ cudaError_t launch_pack_w(const float* W, int Hq, int P, void* out, cudaStream_t
 cudaError_t launch_qnu(const void* Q, const float* nu, int64_t T, int Hq, float* out, cudaStream_t s);
 cudaError_t launch_score_tc(const TcLaunch& L, cudaStream_t s);
 
+// ---------------------------------------------------------------- tensor-core index build
+// A build item: KV head g, block cb of <= 128 output columns (heads hl*r+c of the
+// group), key tiles [t0, t1) of 128 keys.
+struct BuildItem {
+  int32_t g, cb, t0, t1;
+};
+bool build_tc_supported(int r, int G);
+size_t build_tc_workspace(int Hq, int r);
+cudaError_t launch_build_tc(const void* K, const float* R, void* sketch, int64_t N, int Hq, int G, int r,
+                            const BuildItem* items, int n_items, void* wsplit, int* err, int num_sms,
+                            cudaStream_t s);
+
 }  // namespace saki

@@ -122,9 +122,14 @@ def _build(lib, w, K, R, mu=None, center=0):
     return sk.float().cpu().numpy()
 
 
-@pytest.mark.parametrize("dtype,r,center", [("f32", 16, 0), ("bf16", 32, 0), ("bf16", 64, 1), ("f32", 5, 1)])
-def test_build_index(lib, dtype, r, center):
-    w = synth.Workload("bi", 8, 2, rank=r, dtype=dtype, n_calib=256, seq_lens=(1000,), spikes=(6, 6), seed=3)
+@pytest.mark.parametrize("dtype,r,center,hq,hk,n", [
+    ("f32", 16, 0, 8, 2, 1000), ("bf16", 32, 0, 8, 2, 1000), ("bf16", 64, 1, 8, 2, 1000), ("f32", 5, 1, 8, 2, 1000),
+    ("bf16", 16, 0, 8, 2, 300),       # tensor-core build, one 64-column block, ragged last key tile
+    ("bf16", 64, 0, 8, 2, 777),       # two 128-column blocks per KV head
+    ("bf16", 32, 0, 14, 2, 513),      # GQA 7: blocks of 128 and 96 columns
+])
+def test_build_index(lib, dtype, r, center, hq, hk, n):
+    w = synth.Workload("bi", hq, hk, rank=r, dtype=dtype, n_calib=256, seq_lens=(n,), spikes=(6, 6), seed=3)
     data = synth.make_numpy(w)
     ref = O.fit(data["q_calib"], data["k_calib"], data["A"], r, center=bool(center))
     R = ref["R"].astype(np.float32)
