@@ -59,6 +59,7 @@ saki_status check_layout(const saki_layout* L, int64_t* total_keys) {
 
 // ------------------------------------------------------------------ work plan
 struct Plan {
+  int nq = 1;   // launch width: smallest power of two >= the largest group
   std::vector<ScoreItem> items;
   std::vector<MergeItem> merges;
   std::vector<int32_t> vis;
@@ -83,6 +84,7 @@ Plan make_plan(const saki_layout* L, int Hq, int kp) {
       ++t;
     }
     work += g.vmax;
+    while (p.nq < g.n) p.nq *= 2;
     groups.push_back(g);
   }
   const int64_t target_per_head = std::max<int64_t>(1, (int64_t)8 * kNumSMs / Hq);
@@ -422,7 +424,7 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
   a.exact = 0;
   a.n_items = (int32_t)p.items.size();
   a.n_merges = (int32_t)p.merges.size();
-  if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
+  if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, p.nq, s))) != SAKI_OK) return st;
   return cuda_status(launch_merge(a, cfg->dtype, kp, s));
 }
 
@@ -471,7 +473,7 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
     a.exact = 1;
     a.n_items = (int32_t)p.items.size();
     a.n_merges = (int32_t)p.merges.size();
-    if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
+    if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, p.nq, s))) != SAKI_OK) return st;
     if ((st = cuda_status(launch_merge(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
   }
   const int32_t* vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);

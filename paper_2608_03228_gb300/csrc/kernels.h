@@ -45,9 +45,10 @@ struct ScoreArgs {
 };
 
 // generic CUDA-core scoring (any rank, f32 or bf16)
-cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, cudaStream_t s);
+// nq: query-group width of the launch (1, 2, 4 or 8), at least every item's q_count
+cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, cudaStream_t s);
 cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s);
-size_t score_generic_smem(int P, int kp);
+size_t score_generic_smem(int P, int kp, int nq);
 
 // calibration moments: S [(Hq+Hk)][d][d] (queries first), mu [Hk][d]
 cudaError_t launch_gram(const void* q_calib, const void* k_calib, int64_t n, int Hq, int Hk,

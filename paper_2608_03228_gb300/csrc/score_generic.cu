@@ -76,11 +76,25 @@ __device__ __noinline__ uint64_t append_keys(uint64_t* qb, int* cnt_s, unsigned 
   return c > thr ? c : thr;
 }
 
-template <typename Tin, int KP>
+// Packed fp32x2 fused multiply-add: (acc.x, acc.y) += (a.x, a.y) * (b.x, b.y).
+__device__ __forceinline__ void ffma2(unsigned long long& acc, unsigned long long x, unsigned long long y) {
+  asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc) : "l"(x), "l"(y));
+}
+__device__ __forceinline__ unsigned long long pk2(float lo, float hi) {
+  return ((unsigned long long)__float_as_uint(hi) << 32) | __float_as_uint(lo);
+}
+__device__ __forceinline__ float sum2(unsigned long long v) {
+  return __uint_as_float((uint32_t)v) + __uint_as_float((uint32_t)(v >> 32));
+}
+
+// NQ: compile-time width of the query group (1, 2, 4 or 8); the host launches the
+// smallest width that holds every group of the call.
+template <typename Tin, int KP, int NQ>
 __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs a) {
   constexpr int CAP = 2 * KP;
   constexpr int EK = KP / 32;
   constexpr int NV = Vec<Tin>::NV;
+  constexpr int kGroupQ = NQ;
   extern __shared__ __align__(16) unsigned char smem[];
   uint64_t* buf = reinterpret_cast<uint64_t*>(smem);                       // [warps][GQ][CAP]
   float* qs = reinterpret_cast<float*>(buf + kWarps * kGroupQ * CAP);      // [GQ][d]
@@ -129,8 +143,9 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
   const Tin* X = static_cast<const Tin*>(a.X) +
                  ((int64_t)(a.exact ? h / a.G : h) * a.N + it.key_base) * P;
   uint64_t thr[kGroupQ];
+  float thr_f[kGroupQ];   // score part of thr: a key can only pass if its score is >= thr_f
 #pragma unroll
-  for (int b = 0; b < kGroupQ; ++b) thr[b] = 0ull;
+  for (int b = 0; b < kGroupQ; ++b) { thr[b] = 0ull; thr_f[b] = -INFINITY; }
   uint64_t* wbuf = buf + warp * kGroupQ * CAP;
   int* wcnt = cnt_s + warp * kGroupQ;
   const int nkeys = it.key_hi - it.key_lo;
@@ -145,6 +160,9 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
     if (jl < nkeys) {
       const Tin* row = X + (int64_t)j * P;
       if (vec) {
+        unsigned long long a2[kGroupQ];
+#pragma unroll
+        for (int b = 0; b < kGroupQ; ++b) a2[b] = 0ull;
         const uint4* r4 = reinterpret_cast<const uint4*>(row);
         const int nv = P / NV;
         for (int v = 0; v < nv; ++v) {
@@ -153,17 +171,17 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
           Vec<Tin>::unpack(raw, x);
 #pragma unroll
           for (int b = 0; b < kGroupQ; ++b) {
-            const float4* u4 = reinterpret_cast<const float4*>(us + b * P + v * NV);
+            const ulonglong2* u2 = reinterpret_cast<const ulonglong2*>(us + b * P + v * NV);
 #pragma unroll
             for (int e4 = 0; e4 < NV / 4; ++e4) {
-              const float4 uu = u4[e4];
-              acc[b] = fmaf(uu.x, x[4 * e4 + 0], acc[b]);
-              acc[b] = fmaf(uu.y, x[4 * e4 + 1], acc[b]);
-              acc[b] = fmaf(uu.z, x[4 * e4 + 2], acc[b]);
-              acc[b] = fmaf(uu.w, x[4 * e4 + 3], acc[b]);
+              const ulonglong2 uu = u2[e4];
+              ffma2(a2[b], uu.x, pk2(x[4 * e4 + 0], x[4 * e4 + 1]));
+              ffma2(a2[b], uu.y, pk2(x[4 * e4 + 2], x[4 * e4 + 3]));
             }
           }
         }
+#pragma unroll
+        for (int b = 0; b < kGroupQ; ++b) acc[b] = sum2(a2[b]);
       } else {
         for (int p = 0; p < P; ++p) {
           const float x = to_f<Tin>(row[p]);
@@ -175,11 +193,16 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
 #pragma unroll
     for (int b = 0; b < kGroupQ; ++b) {
       if (b < nq) {
-        const bool ok = (jl < nkeys) && (j < visq[b]);
-        const uint64_t key = make_key(acc[b], (uint32_t)j);
-        const bool pass = ok && key > thr[b];
-        const unsigned mask = __ballot_sync(0xffffffffu, pass);
-        if (mask) thr[b] = append_keys<KP>(wbuf + b * CAP, wcnt + b, cta_thr + b, key, pass, mask, thr[b], a.k);
+        const bool ok = (jl < nkeys) && (j < visq[b]) && acc[b] >= thr_f[b];
+        if (__ballot_sync(0xffffffffu, ok)) {
+          const uint64_t key = make_key(acc[b], (uint32_t)j);
+          const bool pass = ok && key > thr[b];
+          const unsigned mask = __ballot_sync(0xffffffffu, pass);
+          if (mask) {
+            thr[b] = append_keys<KP>(wbuf + b * CAP, wcnt + b, cta_thr + b, key, pass, mask, thr[b], a.k);
+            thr_f[b] = key_score(thr[b]);
+          }
+        }
       }
     }
   }
@@ -252,10 +275,10 @@ __global__ void __launch_bounds__(128) merge_kernel(const ScoreArgs a) {
   }
 }
 
-template <typename Tin, int KP>
+template <typename Tin, int KP, int NQ>
 cudaError_t launch_score_t(const ScoreArgs& a, cudaStream_t s) {
-  const size_t sm = score_generic_smem(a.P, KP);
-  auto kern = score_generic_kernel<Tin, KP>;
+  const size_t sm = score_generic_smem(a.P, KP, NQ);
+  auto kern = score_generic_kernel<Tin, KP, NQ>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
   kern<<<dim3(a.n_items, a.Hq), kThreads, sm, s>>>(a);
@@ -263,16 +286,28 @@ cudaError_t launch_score_t(const ScoreArgs& a, cudaStream_t s) {
 }
 }  // namespace
 
-size_t score_generic_smem(int P, int kp) {
-  return sizeof(uint64_t) * (size_t)kWarps * kGroupQ * 2 * kp +
-         sizeof(float) * (size_t)(kGroupQ * kD + kGroupQ * P + kGroupQ) + sizeof(int) * (kGroupQ + kWarps * kGroupQ);
+size_t score_generic_smem(int P, int kp, int nq) {
+  return sizeof(uint64_t) * (size_t)kWarps * nq * 2 * kp +
+         sizeof(float) * (size_t)(nq * kD + nq * P + nq) + sizeof(int) * (nq + kWarps * nq);
 }
 
-cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, cudaStream_t s) {
+namespace {
+template <typename Tin, int KP>
+cudaError_t launch_nq(const ScoreArgs& a, int nq, cudaStream_t s) {
+  switch (nq) {
+    case 1: return launch_score_t<Tin, KP, 1>(a, s);
+    case 2: return launch_score_t<Tin, KP, 2>(a, s);
+    case 4: return launch_score_t<Tin, KP, 4>(a, s);
+    default: return launch_score_t<Tin, KP, 8>(a, s);
+  }
+}
+}  // namespace
+
+cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, cudaStream_t s) {
   if (a.n_items == 0) return cudaSuccess;
   if (dtype == SAKI_BF16)
-    return kp == 64 ? launch_score_t<__nv_bfloat16, 64>(a, s) : launch_score_t<__nv_bfloat16, 128>(a, s);
-  return kp == 64 ? launch_score_t<float, 64>(a, s) : launch_score_t<float, 128>(a, s);
+    return kp == 64 ? launch_nq<__nv_bfloat16, 64>(a, nq, s) : launch_nq<__nv_bfloat16, 128>(a, nq, s);
+  return kp == 64 ? launch_nq<float, 64>(a, nq, s) : launch_nq<float, 128>(a, nq, s);
 }
 
 cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s) {
