@@ -252,8 +252,8 @@ BuildWs build_ws(const saki_config* c, int64_t N) {
   return w;
 }
 
-// fit workspace: S, F, G [(Hq+Hk)][d][d], mu [Hk][d], status [Hq+Hk]
-struct FitWs { size_t S, F, G, mu, st, bytes; };
+// fit workspace: S, F, G [(Hq+Hk)][d][d], mu [Hk][d], status [Hq+Hk], C'^T scratch [Hq][d][d]
+struct FitWs { size_t S, F, G, mu, st, C, bytes; };
 FitWs fit_ws(const saki_config* c) {
   const size_t nm = (size_t)c->num_q_heads + c->num_kv_heads;
   const size_t mat = nm * kD * kD * sizeof(float);
@@ -263,7 +263,8 @@ FitWs fit_ws(const saki_config* c) {
   w.G = w.F + align_up(mat);
   w.mu = w.G + align_up(mat);
   w.st = w.mu + align_up((size_t)c->num_kv_heads * kD * sizeof(float));
-  w.bytes = w.st + align_up(nm * sizeof(int));
+  w.C = w.st + align_up(nm * sizeof(int));
+  w.bytes = w.C + align_up((size_t)c->num_q_heads * kD * kD * sizeof(float));
   return w;
 }
 
@@ -344,8 +345,8 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
   if ((st = cuda_status(launch_gram(q_calib, k_calib, n_calib, Hq, Hk, cfg->center, cfg->dtype, S, muw, s))) != SAKI_OK)
     return st;
   if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK) return st;
-  if ((st = cuda_status(launch_fit(A, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps, L, R, sigma,
-                                   loss, nu, status, s))) != SAKI_OK)
+  if ((st = cuda_status(launch_fit(A, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
+                                   reinterpret_cast<float*>(ws + w.C), L, R, sigma, loss, nu, status, s))) != SAKI_OK)
     return st;
   std::vector<int> hst(nm);
   if ((st = cuda_status(cudaMemcpyAsync(hst.data(), status, nm * sizeof(int), cudaMemcpyDeviceToHost, s))) != SAKI_OK)

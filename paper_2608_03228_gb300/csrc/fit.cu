@@ -212,13 +212,14 @@ __global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, flo
   }
 }
 
-__global__ void __launch_bounds__(kFitThreads) fit_kernel(const float* A, const float* Fm, const float* Gm,
-                                                          const float* mu, int Hq, int Hk, int r, int max_sweeps,
-                                                          float tol, float* L, float* R, float* sigma, float* loss,
-                                                          float* nu, int* status) {
+// Shared memory holds only the Jacobi matrix (66 KB), so two CTAs share an SM;
+// C'^T is kept in a global scratch slice (L2-resident) for the steps after the SVD.
+__global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, const float* Fm, const float* Gm,
+                                                             const float* mu, int Hq, int Hk, int r, int max_sweeps,
+                                                             float tol, float* Cws, float* L, float* R, float* sigma,
+                                                             float* loss, float* nu, int* status) {
   extern __shared__ __align__(16) float sm[];
   float* X = sm;               // column-major, ld kLdS
-  float* Y = sm + kD * kLdS;
   __shared__ float sig[kD];
   __shared__ float sgn[kD];
   __shared__ int perm[kD];
@@ -230,26 +231,25 @@ __global__ void __launch_bounds__(kFitThreads) fit_kernel(const float* A, const 
   const float* Gq = Gm + (int64_t)h * kD * kD;
   const float* Fk = Fm + (int64_t)(Hq + g) * kD * kD;
   const float* Gk = Gm + (int64_t)(Hq + g) * kD * kD;
+  float* Ct = Cws + (int64_t)h * kD * kD;   // C'^T, column-major: (row, col) at [col * d + row]
   float* Lh = L + (int64_t)h * kD * r;
   float* Rh = R + (int64_t)h * kD * r;
 
-  for (int o = tid; o < kD * kD; o += kFitThreads) Y[(o % kD) * kLdS + (o / kD)] = Ah[o];
-  __syncthreads();
   const int cc = tid % kD, r0 = (tid / kD) * 32;
-  {  // X = A Fk
+  {  // X = A Fk   (A rows broadcast from L1, Fk columns coalesced)
     float acc[32];
 #pragma unroll
     for (int u = 0; u < 32; ++u) acc[u] = 0.f;
     for (int p = 0; p < kD; ++p) {
       const float f = __ldg(Fk + p * kD + cc);
 #pragma unroll
-      for (int u = 0; u < 32; ++u) acc[u] = fmaf(Y[p * kLdS + r0 + u], f, acc[u]);
+      for (int u = 0; u < 32; ++u) acc[u] = fmaf(__ldg(Ah + (r0 + u) * kD + p), f, acc[u]);
     }
 #pragma unroll
     for (int u = 0; u < 32; ++u) X[cc * kLdS + r0 + u] = acc[u];
   }
   __syncthreads();
-  {  // Y = X^T Fq = C'^T
+  {  // C'^T = X^T Fq -> global scratch
     float acc[32];
 #pragma unroll
     for (int u = 0; u < 32; ++u) acc[u] = 0.f;
@@ -258,12 +258,11 @@ __global__ void __launch_bounds__(kFitThreads) fit_kernel(const float* A, const 
 #pragma unroll
       for (int u = 0; u < 32; ++u) acc[u] = fmaf(X[(r0 + u) * kLdS + p], f, acc[u]);
     }
-    __syncthreads();
 #pragma unroll
-    for (int u = 0; u < 32; ++u) Y[cc * kLdS + r0 + u] = acc[u];
+    for (int u = 0; u < 32; ++u) Ct[cc * kD + r0 + u] = acc[u];
   }
   __syncthreads();
-  for (int o = tid; o < kD * kLdS; o += kFitThreads) X[o] = Y[o];
+  for (int o = tid; o < kD * kD; o += kFitThreads) X[(o / kD) * kLdS + (o % kD)] = Ct[o];
   __syncthreads();
 
   const bool conv = jacobi_columns(X, max_sweeps, tol, &counter);
@@ -277,34 +276,31 @@ __global__ void __launch_bounds__(kFitThreads) fit_kernel(const float* A, const 
     perm[rk] = tid;
   }
   __syncthreads();
-  float smax = sig[perm[0]];
+  const float smax = sig[perm[0]];
   if (tid == 0 && !isfinite(smax)) status[h] |= kStNonFinite;
 
-  // Z = C' V_r Sigma^{-1} (= U_r) into L as scratch;  Rtmp = Gk V_r Sigma^{1/2} into Y after
+  // Z = C' V_r Sigma^{-1} (= U_r) into L as scratch; R = Gk V_r Sigma^{1/2} (unsigned) into R
   const int a = tid % kD;
   for (int c = tid / kD; c < r; c += kFitThreads / kD) {
     const int i = perm[c];
     const float s = sig[i];
     const bool live = s > 0.f && s > smax * 1e-20f;
-    float acc = 0.f;
-    for (int b = 0; b < kD; ++b) acc = fmaf(Y[a * kLdS + b], X[i * kLdS + b], acc);
-    Lh[a * r + c] = live ? acc / (s * s) : 0.f;   // C' x_i / s^2 = u_i (x_i = s v_i)
-  }
-  __syncthreads();
-  for (int c = tid / kD; c < r; c += kFitThreads / kD) {
-    const int i = perm[c];
-    const float s = sig[i];
-    const bool live = s > 0.f && s > smax * 1e-20f;
-    float acc = 0.f;
-    for (int b = 0; b < kD; ++b) acc = fmaf(__ldg(Gk + a * kD + b), X[i * kLdS + b], acc);
-    Y[c * kLdS + a] = live ? acc / sqrtf(s) : 0.f;   // Gk v_i sqrt(s) = Gk x_i / sqrt(s)
+    float z = 0.f, q = 0.f;
+    const float* ct = Ct + a * kD;   // column a of C'^T = row a of C'
+    for (int b = 0; b < kD; ++b) {
+      const float x = X[i * kLdS + b];
+      z = fmaf(__ldg(ct + b), x, z);
+      q = fmaf(__ldg(Gk + a * kD + b), x, q);
+    }
+    Lh[a * r + c] = live ? z / (s * s) : 0.f;    // C' x_i / s^2 = u_i (x_i = s v_i)
+    Rh[a * r + c] = live ? q / sqrtf(s) : 0.f;   // Gk v_i sqrt(s) = Gk x_i / sqrt(s)
   }
   __syncthreads();
   for (int c = warp; c < r; c += kFitThreads / 32) {  // sign: largest-|.| entry of R[:, c] positive
     float best = -1.f, val = 0.f;
     int bi = 0;
     for (int i = lane; i < kD; i += 32) {
-      const float v = Y[c * kLdS + i];
+      const float v = Rh[i * r + c];
       if (fabsf(v) > best) { best = fabsf(v); bi = i; val = v; }
     }
 #pragma unroll
@@ -319,8 +315,8 @@ __global__ void __launch_bounds__(kFitThreads) fit_kernel(const float* A, const 
   __syncthreads();
   for (int o = tid; o < kD * r; o += kFitThreads) {
     const int i = o / r, c = o % r;
-    Rh[o] = sgn[c] * Y[c * kLdS + i];
-    X[c * kLdS + i] = Lh[o];   // Z back into shared memory (X is free now)
+    Rh[o] *= sgn[c];
+    X[c * kLdS + i] = Lh[o];   // Z back into shared memory (the Jacobi matrix is no longer needed)
   }
   __syncthreads();
   for (int c = tid / kD; c < r; c += kFitThreads / kD) {
@@ -345,7 +341,8 @@ __global__ void __launch_bounds__(kFitThreads) fit_kernel(const float* A, const 
 }
 
 constexpr float kTol = 1e-6f;
-constexpr size_t kSmem = 2 * sizeof(float) * kD * kLdS;
+constexpr size_t kSmem = 2 * sizeof(float) * kD * kLdS;     // factor kernel: S and its inverse factor
+constexpr size_t kFitSmem = sizeof(float) * kD * kLdS;      // fit kernel: the Jacobi matrix
 }  // namespace
 
 cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps, float* F, float* Gm,
@@ -357,12 +354,12 @@ cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_swe
 }
 
 cudaError_t launch_fit(const float* A, const float* F, const float* Gm, const float* mu, int Hq, int Hk, int r,
-                       int max_sweeps, float* L, float* R, float* sigma, float* loss, float* nu, int* status,
-                       cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(fit_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+                       int max_sweeps, float* Cws, float* L, float* R, float* sigma, float* loss, float* nu,
+                       int* status, cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(fit_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFitSmem);
   if (e != cudaSuccess) return e;
-  fit_kernel<<<Hq, kFitThreads, kSmem, s>>>(A, F, Gm, mu, Hq, Hk, r, max_sweeps, kTol, L, R, sigma, loss, nu,
-                                            status);
+  fit_kernel<<<Hq, kFitThreads, kFitSmem, s>>>(A, F, Gm, mu, Hq, Hk, r, max_sweeps, kTol, Cws, L, R, sigma, loss,
+                                               nu, status);
   return cudaGetLastError();
 }
 

@@ -59,8 +59,9 @@ cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_swe
                           float* F, float* Gm, int* status, cudaStream_t s);
 
 // per query head: C' = Fq^T A Fk, Jacobi SVD, factors L, R, sigma, loss, nu
+// Cws: scratch [Hq][d][d] (C'^T per head)
 cudaError_t launch_fit(const float* A, const float* F, const float* Gm, const float* mu, int Hq,
-                       int Hk, int r, int max_sweeps, float* L, float* R, float* sigma,
+                       int Hk, int r, int max_sweeps, float* Cws, float* L, float* R, float* sigma,
                        float* loss, float* nu, int* status, cudaStream_t s);
 
 // key codes

@@ -12,12 +12,13 @@
 //      (codes, or raw keys for the exact scores) into a ring of shared-memory
 //      stages; one thread issues tcgen05.mma (M = 128 queries, N = NT keys,
 //      K = P, twice: u_hi and u_lo) into one of two TMEM accumulators;
-//   3. four epilogue warps own one query row per thread (TMEM lane = row): they
-//      pull 32 scores at a time with tcgen05.ld, mask the causal edge, skip any
-//      16-score half whose maximum does not beat the row's threshold, and append
-//      the others to the row's candidate column in shared memory; when a column
-//      fills, a sampled pivot shrinks it to a set that still holds the row's top
-//      k and raises the threshold.  The T x N score matrix is never stored.
+//   3. four epilogue warps own one query row per thread (TMEM lane = row) and
+//      select in two passes over the same scores (the key tiles are multiplied
+//      twice; the tensor core has ample headroom): pass 1 keeps per-row maxima
+//      of 128 key groups and derives a certified lower bound tau on the row's
+//      k-th best score; pass 2 appends the visible keys scoring >= tau to the
+//      row's candidate column in shared memory.  The T x N score matrix is never
+//      stored.
 //   4. exact top-k of the remaining candidates per row, written coalesced.
 // Roles: warp 0 = TMA producer, warp 1 = TMEM owner + MMA issuer, warps 2-5 =
 // epilogue.  Every mbarrier wait is bounded (tc.cuh); a timed-out CTA drains its
@@ -33,12 +34,14 @@ namespace saki {
 namespace {
 
 constexpr int kLdc = 129;   // candidate column stride (words): conflict-free per-row scans and row reads
+constexpr int kGroups = 64;   // pass-1 key groups per row (key offset mod 64); two maxima kept per group
+constexpr int kScr = 36;      // per-row scratch stride (words): 32 scores + pad, conflict-free 16-byte stores
 
 template <int P>
 struct TcCfg {
   static constexpr int NT = P == 128 ? 128 : 256;            // keys per tile (MMA N)
   static constexpr int STAGES = P <= 32 ? 4 : 2;
-  static constexpr int CAP = P == 128 ? 128 : (P == 16 ? 208 : 168);   // candidate slots per row
+  static constexpr int CAP = P == 128 ? 104 : 128;            // candidate slots per row (multiple of 8)
   static constexpr int KB = P == 128 ? 2 : 1;                 // 64-wide K blocks
   static constexpr int KW = P == 128 ? 64 : P;                // K width of one block
   static constexpr int KK = KW / 16;                          // MMA K steps per block
@@ -48,18 +51,32 @@ struct TcCfg {
   static constexpr int A_BYTES = 2 * A_PART > 32768 ? 2 * A_PART : 32768;  // also holds the 128x128 query tile
   static constexpr int STAGE_BYTES = NT * P * 2;
   static constexpr int CAND_BYTES = CAP * kLdc * 4 + ((CAP * kLdc * 2 + 15) & ~15);
+  static constexpr int SCR_BYTES = 128 * kScr * 4;
   static constexpr int TMEM_COLS = 2 * NT;
   static constexpr int OFF_STAGE = A_BYTES;
   static constexpr int OFF_CAND = OFF_STAGE + STAGES * STAGE_BYTES;
-  static constexpr int OFF_BAR = OFF_CAND + CAND_BYTES;
+  static constexpr int OFF_SCR = OFF_CAND + CAND_BYTES;
+  static constexpr int OFF_BAR = OFF_SCR + SCR_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
   static_assert(STAGE_BYTES >= P * 128, "a projection chunk must fit a stage");
+  static_assert(CAP % 8 == 0 && CAP >= 64 + 32, "candidate capacity: k + one chunk of appends");
+  static_assert(NT % 64 == 0, "a key tile covers whole key groups");
   static_assert(SMEM <= 232448, "shared memory budget");
 };
 
-__device__ __forceinline__ float fmax3(float a, float b, float c) { return fmaxf(a, fmaxf(b, c)); }
-
 // ---------------------------------------------------------------- selection
+// Selection of a row's top k runs in two passes over the same tensor-core scores.
+//   Pass 1 keeps, per row, the two highest scores of each of 64 key groups (key
+//   offset mod 64).  These 128 values are scores of distinct keys, so any value
+//   tau with at least k of them >= tau is a certified lower bound on the row's
+//   k-th best score: no key of the top k scores below tau.
+//   Pass 2 appends only the keys scoring >= tau to the row's candidate column
+//   (about 75 per row for independent scores with k = 64, against ~5 k ln(n/k)
+//   for a streaming threshold), and a final exact cut leaves the top k.
+// Every helper runs with the warp converged: loops over candidate slots run to
+// the warp's largest count with per-lane predicates, so the 32 rows of a warp
+// never split into separately executed paths.
+
 // A row's candidate column: scores (fp32) and key indices (16-bit; the host only
 // sends sequences of at most 65535 keys here).
 struct Col {
@@ -74,31 +91,63 @@ struct Col {
   }
 };
 
-// The passes below keep eight independent shared-memory loads in flight per
-// thread: a row's column is scanned with no other parallelism, so latency, not
-// bandwidth, bounds them.
+__device__ __forceinline__ int warp_max(int v) { return __reduce_max_sync(0xffffffffu, v); }
 
-// Number of entries scoring >= p.
-__device__ __forceinline__ int count_ge(const Col& c, int cnt, float p) {
-  int n0 = 0, n1 = 0, i = 0;
-  for (; i + 8 <= cnt; i += 8) {
+// Largest float below t (appending "score > below(tau)" keeps every score >= tau).
+__device__ __forceinline__ float below(float t) {
+  if (t == -INFINITY) return t;
+  const uint32_t b = __float_as_uint(t);
+  if ((b & 0x7fffffffu) == 0) return __uint_as_float(0x80000001u);
+  return __uint_as_float((b & 0x80000000u) ? b + 1 : b - 1);
+}
+
+// Bitonic sort of a register array into descending order (compile-time indices).
+template <int N>
+__device__ __forceinline__ void sort_desc(float (&s)[N]) {
+#pragma unroll
+  for (int size = 2; size <= N; size <<= 1)
+#pragma unroll
+    for (int j = size >> 1; j > 0; j >>= 1)
+#pragma unroll
+      for (int i = 0; i < N; ++i) {
+        const int l = i ^ j;
+        if (l > i) {
+          const float a = s[i], b = s[l];
+          const bool desc = (i & size) == 0;
+          s[i] = desc ? fmaxf(a, b) : fminf(a, b);
+          s[l] = desc ? fminf(a, b) : fmaxf(a, b);
+        }
+      }
+}
+
+template <int N>
+__device__ __forceinline__ float pick(const float (&s)[N], int q) {
+  float p = s[0];
+#pragma unroll
+  for (int u = 1; u < N; ++u) p = (u == q) ? s[u] : p;
+  return p;
+}
+
+// Entries scoring >= p among the lane's first cnt (slots read up to the warp's cmax).
+__device__ __forceinline__ int count_ge(const Col& c, int cnt, int cmax, float p) {
+  int n0 = 0, n1 = 0;
+  for (int i = 0; i < cmax; i += 8) {
     float v[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) v[u] = c.s(i + u);
 #pragma unroll
     for (int u = 0; u < 8; u += 2) {
-      n0 += v[u] >= p;
-      n1 += v[u + 1] >= p;
+      n0 += (i + u < cnt && v[u] >= p) ? 1 : 0;
+      n1 += (i + u + 1 < cnt && v[u + 1] >= p) ? 1 : 0;
     }
   }
-  for (; i < cnt; ++i) n0 += c.s(i) >= p;
   return n0 + n1;
 }
 
-// Keep the entries scoring >= p (in place, order preserved); returns their count.
-__device__ __forceinline__ int compact_ge(const Col& c, int cnt, float p) {
-  int w = 0, i = 0;
-  for (; i + 8 <= cnt; i += 8) {
+// Lanes with `on` keep their entries scoring >= p (in place, order preserved).
+__device__ __forceinline__ int compact_ge(const Col& c, int cnt, int cmax, float p, bool on) {
+  int w = 0;
+  for (int i = 0; i < cmax; i += 8) {
     float v[8];
     int j[8];
 #pragma unroll
@@ -107,152 +156,307 @@ __device__ __forceinline__ int compact_ge(const Col& c, int cnt, float p) {
       j[u] = c.j(i + u);
     }
 #pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (v[u] >= p) {
-        c.put(w, v[u], j[u]);
-        ++w;
-      }
-  }
-  for (; i < cnt; ++i) {
-    const float v = c.s(i);
-    if (v >= p) {
-      c.put(w, v, c.j(i));
-      ++w;
+    for (int u = 0; u < 8; ++u) {
+      const bool keep = on && i + u < cnt && v[u] >= p;
+      if (keep) c.put(w, v[u], j[u]);
+      w += keep ? 1 : 0;
     }
   }
-  return w;
+  return on ? w : cnt;
 }
 
 // (score, index) worse-than: lower score, or equal score and higher index.
 __device__ __forceinline__ bool worse(float a, int ja, float b, int jb) { return a < b || (a == b && ja > jb); }
 
-// Remove the worst entry (lowest score, then highest index); raise thr to its score.
-__device__ __forceinline__ void remove_worst(const Col& c, int& cnt, float& thr) {
+// Lanes with `on` drop their worst entry (lowest score, then highest index) and
+// raise thr to its score.
+__device__ __forceinline__ void remove_worst(const Col& c, int& cnt, int cmax, float& thr, bool on) {
   float ws[4];
   int wj[4], wp[4];
 #pragma unroll
   for (int u = 0; u < 4; ++u) { ws[u] = INFINITY; wj[u] = -1; wp[u] = 0; }
-  int i = 0;
-  for (; i + 4 <= cnt; i += 4) {
+  for (int i = 0; i < cmax; i += 4) {
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const float v = c.s(i + u);
       const int jj = c.j(i + u);
-      if (worse(v, jj, ws[u], wj[u])) { ws[u] = v; wj[u] = jj; wp[u] = i + u; }
+      if (i + u < cnt && worse(v, jj, ws[u], wj[u])) { ws[u] = v; wj[u] = jj; wp[u] = i + u; }
     }
-  }
-  for (; i < cnt; ++i) {
-    const float v = c.s(i);
-    const int jj = c.j(i);
-    if (worse(v, jj, ws[0], wj[0])) { ws[0] = v; wj[0] = jj; wp[0] = i; }
   }
 #pragma unroll
   for (int u = 1; u < 4; ++u)
     if (worse(ws[u], wj[u], ws[0], wj[0])) { ws[0] = ws[u]; wj[0] = wj[u]; wp[0] = wp[u]; }
-  --cnt;
-  c.put(wp[0], c.s(cnt), c.j(cnt));
-  thr = fmaxf(thr, ws[0]);
+  if (on && cnt > 0) {
+    --cnt;
+    const float ls = c.s(cnt);
+    const int lj = c.j(cnt);
+    c.put(wp[0], ls, lj);
+    thr = fmaxf(thr, ws[0]);
+  }
 }
 
-// Keep every entry scoring >= a sampled pivot p, provided at least k and at most
-// tmax remain; the threshold becomes p (all later keys have higher indices, so a
-// key scoring exactly p loses to all kept entries).  Returns false if no tried
-// pivot qualifies.
-__device__ __forceinline__ bool pivot_round(const Col& c, int& cnt, float& thr, int k, int aim, int tmax) {
+// Lanes with `on` cut their column to the entries scoring >= a sampled pivot p,
+// for a pivot leaving between k and tmax entries; thr becomes p (every later key
+// has a higher index, so a later key scoring exactly p loses to all kept ones).
+// Lanes for which no tried pivot qualifies keep their column unchanged.
+__device__ __forceinline__ void pivot_cut(const Col& c, int& cnt, float& thr, int k, int aim, int tmax, bool on) {
+  const int cmax = warp_max(cnt);
   float s[8];
 #pragma unroll
   for (int u = 0; u < 8; ++u) s[u] = c.s(((2 * u + 1) * cnt) >> 4);
-  // Batcher odd-even merge sort of 8, descending
-  auto cx = [&](int a, int b) {
-    const float x = fmaxf(s[a], s[b]), y = fminf(s[a], s[b]);
-    s[a] = x;
-    s[b] = y;
-  };
-  cx(0, 1); cx(2, 3); cx(4, 5); cx(6, 7);
-  cx(0, 2); cx(1, 3); cx(4, 6); cx(5, 7);
-  cx(1, 2); cx(5, 6);
-  cx(0, 4); cx(1, 5); cx(2, 6); cx(3, 7);
-  cx(2, 4); cx(3, 5);
-  cx(1, 2); cx(3, 4); cx(5, 6);
+  sort_desc<8>(s);
   // sample q (0-based, descending) sits near entry rank (q + 0.5) cnt / 8
-  int q = (16 * aim / cnt - 1) >> 1;
+  int q = cnt > 0 ? (16 * aim / cnt - 1) >> 1 : 0;
   q = q < 0 ? 0 : (q > 7 ? 7 : q);
+  bool pending = on && cnt > k;
   for (int attempt = 0; attempt < 3; ++attempt) {
-    float p = s[0];
-#pragma unroll
-    for (int u = 1; u < 8; ++u)
-      if (u == q) p = s[u];
-    const int n = count_ge(c, cnt, p);
-    if (n >= k && n <= tmax) {
-      cnt = compact_ge(c, cnt, p);
+    if (!__any_sync(0xffffffffu, pending)) break;
+    const float p = pick<8>(s, q);
+    const int n = count_ge(c, cnt, cmax, p);
+    const bool ok = pending && n >= k && n <= tmax;
+    if (__any_sync(0xffffffffu, ok)) cnt = compact_ge(c, cnt, cmax, p, ok);
+    if (ok) {
       thr = fmaxf(thr, p);
-      return true;
+      pending = false;
+    } else if (pending) {
+      if (n < k) {
+        if (q == 7) pending = false;
+        ++q;
+      } else {
+        if (q == 0) pending = false;
+        --q;
+      }
     }
-    if (n < k) {
-      if (q == 7) return false;
-      ++q;
-    } else {
-      if (q == 0) return false;
-      --q;
-    }
-  }
-  return false;
-}
-
-// Warp-wide room making, run at a convergent point whenever any lane of the warp
-// has more than tmax candidates: every lane holding more than lo = (k + tmax)/2
-// shrinks at the same time (one pivot round for the whole warp instead of one per
-// lane, and the lanes' fill levels stay in step).  Lanes above tmax are brought
-// to at most tmax in every case; the row's top k is never dropped.
-__device__ __forceinline__ void shrink_warp(const Col& c, int& cnt, float& thr, int k, int tmax) {
-  const int lo = (k + tmax) >> 1;
-  if (cnt > lo) {
-    if (!pivot_round(c, cnt, thr, k, k + ((tmax - k) >> 3), lo) && cnt > tmax)
-      while (cnt > tmax) remove_worst(c, cnt, thr);
   }
 }
 
-// Exactly the k best (or all, if fewer).
-__device__ __forceinline__ void finalize(const Col& c, int& cnt, float& thr, int k) {
-  for (int guard = 0; cnt - k > 12 && guard < 4; ++guard)
-    if (!pivot_round(c, cnt, thr, k, k + 4, cnt - 1)) break;
-  while (cnt > k) remove_worst(c, cnt, thr);
-}
-
-// 16 scores of one row (register offset OFF of a 32-score load): mask the keys
-// the row cannot see and append the ones above thr (lanes diverge here).
-template <int OFF>
-__device__ __forceinline__ void append16(const uint32_t (&r)[32], int j0, int vis, const Col& c, int& cnt,
-                                         float thr) {
-  float v[16];
+// Exact cut of the lanes with `on` to their k best entries (slots [0, k)); thr
+// rises to the k-th best score (a later key, with a higher index, must score
+// above it to matter).  Quickselect by counting: a bracket [lo, hi] around the
+// k-th entry (na entries score above hi, at most k; nb score at or above lo, at
+// least k) narrows with pivots taken from 16 sampled scores of the bracket until
+// at most 16 entries remain in it; the entries above hi are kept, and the
+// boundary entries, ranked as 64-bit (score, index) keys in registers, fill the
+// remaining places.  Lanes whose bracket cannot narrow (many equal scores) fall
+// back to pivot cuts and single removals.
+__device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int k, float* scr, bool on) {
+  bool pending = on && cnt > k;
+  if (!__any_sync(0xffffffffu, pending)) return;
+  const int cmax = warp_max(cnt);
+  float s[16];
 #pragma unroll
-  for (int u = 0; u < 16; ++u) v[u] = __uint_as_float(r[OFF + u]);
-  if (j0 + 16 > vis) {
+  for (int u = 0; u < 16; ++u) s[u] = c.s(((2 * u + 1) * cnt) >> 5);
+  sort_desc<16>(s);
+  float hi = INFINITY, lo = -INFINITY;
+  int na = 0, nb = cnt;
+  bool ready = false;
+  for (int round = 0; round < 6; ++round) {
+    const bool act = pending && !ready;
+    if (!__any_sync(0xffffffffu, act)) break;
+    // sample q sits near rank (q + 0.5) pop / 16 of the bracket's population
+    const int pop = nb - na > 0 ? nb - na : 1;
+    int qc = (32 * (k - na) / pop - 1) >> 1;
+    qc = qc < 0 ? 0 : (qc > 15 ? 15 : qc);
+    const float hi2 = qc - 2 < 0 ? hi : pick<16>(s, qc - 2);
+    const float lo2 = qc + 2 > 15 ? lo : pick<16>(s, qc + 2);
+    int a2 = 0, b2 = 0;
+    for (int i = 0; i < cmax; i += 8) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = c.s(i + u);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const bool in = i + u < cnt;
+        a2 += (in && v[u] > hi2) ? 1 : 0;
+        b2 += (in && v[u] >= lo2) ? 1 : 0;
+      }
+    }
+    if (act) {
+      if (a2 <= k) { hi = hi2; na = a2; }
+      if (b2 >= k) { lo = lo2; nb = b2; }
+      ready = nb - na <= 16;
+    }
+    const bool resample = act && !ready;
+    if (__any_sync(0xffffffffu, resample)) {
+      // new samples: every stride-th score inside the bracket (pop > 16 there)
+      const int stride = (nb - na) >> 4;
+      int ns = 0, seen = 0;
+      for (int i = 0; i < cmax; i += 8) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = c.s(i + u);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const bool in = resample && i + u < cnt && v[u] >= lo && v[u] <= hi;
+          const bool take = in && seen == 0 && ns < 16;
+          if (take) scr[ns] = v[u];
+          ns += take ? 1 : 0;
+          seen = in ? (seen + 1 == stride ? 0 : seen + 1) : seen;
+        }
+      }
+      if (resample) {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) s[u] = u < ns ? scr[u] : -INFINITY;
+      }
+      sort_desc<16>(s);
+    }
+  }
+  const bool fin = pending && ready;
+  if (__any_sync(0xffffffffu, fin)) {
+    // entries above hi compacted in place, boundary entries to the scratch
+    int w = 0, nbd = 0;
+    for (int i = 0; i < cmax; i += 8) {
+      float v[8];
+      int j[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        v[u] = c.s(i + u);
+        j[u] = c.j(i + u);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const bool in = fin && i + u < cnt;
+        const bool sure = in && v[u] > hi;
+        const bool bnd = in && !sure && v[u] >= lo;
+        if (sure) c.put(w, v[u], j[u]);
+        if (bnd) {
+          scr[2 * nbd] = v[u];
+          scr[2 * nbd + 1] = __int_as_float(j[u]);
+        }
+        w += sure ? 1 : 0;
+        nbd += bnd ? 1 : 0;
+      }
+    }
+    uint64_t key[16];
 #pragma unroll
     for (int u = 0; u < 16; ++u)
-      if (j0 + u >= vis) v[u] = -INFINITY;
-  }
-  const float m = fmaxf(fmax3(fmax3(v[0], v[1], v[2]), fmax3(v[3], v[4], v[5]), fmax3(v[6], v[7], v[8])),
-                        fmax3(fmax3(v[9], v[10], v[11]), fmax3(v[12], v[13], v[14]), v[15]));
-  if (m > thr) {
-    // branch-free: write every key at the next free slot, advance only past
-    // the ones above thr (the slot stays in bounds: cnt <= CAP - 16 on entry)
+      key[u] = (fin && u < nbd) ? make_key(scr[2 * u], (uint32_t)__float_as_int(scr[2 * u + 1])) : 0ull;
+#pragma unroll
+    for (int size = 2; size <= 16; size <<= 1)
+#pragma unroll
+      for (int jj = size >> 1; jj > 0; jj >>= 1)
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int l = i ^ jj;
+          if (l > i) {
+            const uint64_t x = key[i], y = key[l];
+            const bool desc = (i & size) == 0;
+            const bool sw = desc ? (x < y) : (x > y);
+            key[i] = sw ? y : x;
+            key[l] = sw ? x : y;
+          }
+        }
+    float kth = hi;
 #pragma unroll
     for (int u = 0; u < 16; ++u) {
-      c.put(cnt, v[u], j0 + u);
-      cnt += v[u] > thr ? 1 : 0;
+      const bool use = fin && w + u < k && u < nbd;
+      if (use) c.put(w + u, key_score(key[u]), key_index(key[u]));
+      if (use) kth = key_score(key[u]);
     }
+    if (fin) {
+      cnt = k;
+      thr = fmaxf(thr, kth);
+      pending = false;
+    }
+  }
+  if (__any_sync(0xffffffffu, pending)) {
+    for (int g = 0; g < 3 && __any_sync(0xffffffffu, pending && cnt - k > 8); ++g)
+      pivot_cut(c, cnt, thr, k, k + 3, cnt - 1, pending && cnt - k > 8);
+    while (__any_sync(0xffffffffu, pending && cnt > k)) remove_worst(c, cnt, warp_max(cnt), thr, pending && cnt > k);
   }
 }
 
-// 32 scores of one row; the capacity check runs with the whole warp converged.
+// Pass 1: fold 32 scores of a row (keys j0 .. j0+31, key groups gb .. gb+31)
+// into the two highest scores of each group (g1 >= g2); keys the row cannot see
+// count as -inf.  Called from fully unrolled loops, so gb is a constant and the
+// maxima stay in registers.
+__device__ __forceinline__ void fold32(const uint32_t (&r)[32], float (&g1)[kGroups], float (&g2)[kGroups], int gb,
+                                       int j0, int vis) {
+  float v[32];
+#pragma unroll
+  for (int u = 0; u < 32; ++u) v[u] = __uint_as_float(r[u]);
+  if (j0 + 32 > vis) {
+#pragma unroll
+    for (int u = 0; u < 32; ++u)
+      if (j0 + u >= vis) v[u] = -INFINITY;
+  }
+#pragma unroll
+  for (int u = 0; u < 32; ++u) {
+    const float hi = fmaxf(g1[gb + u], v[u]);
+    g2[gb + u] = fmaxf(g2[gb + u], fminf(g1[gb + u], v[u]));
+    g1[gb + u] = hi;
+  }
+}
+
+// The certified bound of pass 1: a value tau with at least k of the 128 kept
+// values >= tau, taken from a sorted sample of 16 of them (the highest sample
+// that qualifies), or -inf if none does (then every visible key is a candidate).
+__device__ __forceinline__ float select_tau(const float (&g1)[kGroups], const float (&g2)[kGroups], int k) {
+  float s[16];
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    s[u] = g1[8 * u + 3];
+    s[8 + u] = g2[8 * u + 5];
+  }
+  sort_desc<16>(s);
+  // sample q (0-based) has about (q + 1) * 128 / 17 values at or above it
+  int q = (17 * k) / (2 * kGroups);
+  q = q > 15 ? 15 : q;
+  float tau = -INFINITY;
+  bool pending = true;
+  for (int attempt = 0; attempt < 4; ++attempt) {
+    const float p = pick<16>(s, q);
+    int n0 = 0, n1 = 0;
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) {
+      n0 += g1[g] >= p ? 1 : 0;
+      n1 += g2[g] >= p ? 1 : 0;
+    }
+    if (pending && n0 + n1 >= k) {
+      tau = p;
+      pending = false;
+    }
+    if (q == 15) pending = false;
+    q = q < 15 ? q + 1 : 15;
+    if (!__any_sync(0xffffffffu, pending)) break;
+  }
+  return tau;
+}
+
+__device__ __forceinline__ uint32_t above_mask(const uint32_t (&r)[32], int j0, int vis, float thr) {
+  uint32_t m4[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+  for (int u = 0; u < 32; ++u) m4[u & 3] |= (__uint_as_float(r[u]) > thr ? 1u : 0u) << u;
+  uint32_t mask = (m4[0] | m4[1]) | (m4[2] | m4[3]);
+  const int nv = vis - j0;
+  if (nv < 32) mask &= nv > 0 ? (0xffffffffu >> (32 - nv)) : 0u;
+  return mask;
+}
+
+// Pass 2: append the keys of 32 scores of a row (keys j0 .. j0+31) that score
+// above thr and are visible; a column that would overflow is first cut to its
+// k best (which raises thr; CAP >= k + 32 leaves room for the chunk).
 template <int CAP>
-__device__ __forceinline__ void take32(const uint32_t (&r)[32], int j0, int vis, const Col& c, int& cnt, float& thr,
-                                       int k) {
-  append16<0>(r, j0, vis, c, cnt, thr);
-  if (__any_sync(0xffffffffu, cnt > CAP - 16)) shrink_warp(c, cnt, thr, k, CAP - 16);
-  append16<16>(r, j0 + 16, vis, c, cnt, thr);
-  if (__any_sync(0xffffffffu, cnt > CAP - 16)) shrink_warp(c, cnt, thr, k, CAP - 16);
+__device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vis, float& thr, float* scr,
+                                         const Col& c, int& cnt, int k) {
+  uint32_t mask = above_mask(r, j0, vis, thr);
+  const bool over = cnt + __popc(mask) > CAP;
+  if (__any_sync(0xffffffffu, over)) {
+    cut_to_k(c, cnt, thr, k, scr, over);
+    mask = above_mask(r, j0, vis, thr);
+  }
+  if (!__any_sync(0xffffffffu, mask != 0)) return;
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+    *reinterpret_cast<uint4*>(scr + 4 * q) = make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]);
+  while (__any_sync(0xffffffffu, mask != 0)) {
+    if (mask) {
+      const int u = __ffs(mask) - 1;
+      mask &= mask - 1;
+      c.put(cnt, scr[u], j0 + u);
+      ++cnt;
+    }
+  }
 }
 
 template <int P>
@@ -322,6 +526,7 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* sStage = smem + C::OFF_STAGE;
   float* bs = reinterpret_cast<float*>(smem + C::OFF_CAND);
   uint16_t* bi = reinterpret_cast<uint16_t*>(smem + C::OFF_CAND + C::CAP * kLdc * 4);
+  float* scr_all = reinterpret_cast<float*>(smem + C::OFF_SCR);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* empty = full + C::STAGES;
   uint64_t* accf = empty + C::STAGES;
@@ -389,7 +594,8 @@ __global__ void __launch_bounds__(192, 1)
         if (!ok) break;
         const int ntiles = (t.vis_max + C::NT - 1) / C::NT;
         const int64_t xrow = (int64_t)(a.exact ? h / a.G : h) * a.N + t.key_base;
-        for (int i = 0; i < ntiles; ++i) {
+        for (int i2 = 0; i2 < 2 * ntiles; ++i2) {   // the two selection passes
+          const int i = i2 < ntiles ? i2 : i2 - ntiles;
           const int st = sc % C::STAGES;
           if (!(ok = tc::mbar_wait(empty + st, ((sc / C::STAGES) & 1) ^ 1, abort_f))) break;
           tc::mbar_arrive_expect_tx(full + st, C::STAGE_BYTES);
@@ -445,7 +651,7 @@ __global__ void __launch_bounds__(192, 1)
         if (!tc::mbar_wait(aready, it & 1, abort_f)) break;
         tc::fence_after_sync();
         const int ntiles = (t.vis_max + C::NT - 1) / C::NT;
-        for (int i = 0; i < ntiles; ++i) {
+        for (int i = 0; i < 2 * ntiles; ++i) {
           buf = ac & 1;
           if (!(ok = tc::mbar_wait(acce + buf, ((ac >> 1) & 1) ^ 1, abort_f))) break;
           const int st = sc % C::STAGES;
@@ -481,6 +687,7 @@ __global__ void __launch_bounds__(192, 1)
     const int m = quarter * 32 + lane;
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
     const Col col{bs, bi, m};
+    float* scr = scr_all + m * kScr;
     uint32_t ac = 0;
     int it = 0;
     bool ok = true;
@@ -500,9 +707,37 @@ __global__ void __launch_bounds__(192, 1)
         tc::mbar_arrive(aready);
       }
       const int vis = m < t.nrows ? a.vis[t.q0 + m] : 0;
-      int cnt = 0;
-      float thr = -INFINITY;
       const int ntiles = (t.vis_max + C::NT - 1) / C::NT;
+      // pass 1: the two highest scores per key group, then the certified bound
+      float g1[kGroups], g2[kGroups];
+#pragma unroll
+      for (int g = 0; g < kGroups; ++g) {
+        g1[g] = -INFINITY;
+        g2[g] = -INFINITY;
+      }
+      for (int i = 0; i < ntiles; ++i) {
+        const uint32_t buf = ac & 1;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac >> 1) & 1, abort_f));
+        if (!ok) break;
+        tc::fence_after_sync();
+#pragma unroll
+        for (int c = 0; c < C::NT / 32; ++c) {
+          uint32_t r[32];
+          __syncwarp();
+          tc::tmem_ld32(tl + buf * C::NT + c * 32, r);
+          tc::tmem_ld_wait();
+          if (c == C::NT / 32 - 1) {
+            tc::fence_before_sync();
+            tc::mbar_arrive(acce + buf);
+          }
+          fold32(r, g1, g2, (c % 2) * 32, i * C::NT + c * 32, vis);
+        }
+        ++ac;
+      }
+      if (!ok) break;
+      int cnt = 0;
+      float thr = below(select_tau(g1, g2, a.k));
+      // pass 2: candidates scoring >= tau
       for (int i = 0; i < ntiles; ++i) {
         const uint32_t buf = ac & 1;
         ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac >> 1) & 1, abort_f));
@@ -518,8 +753,7 @@ __global__ void __launch_bounds__(192, 1)
             tc::fence_before_sync();
             tc::mbar_arrive(acce + buf);
           }
-          const int j0 = i * C::NT + c * 32;
-          take32<C::CAP>(r, j0, vis, col, cnt, thr, a.k);
+          append32<C::CAP>(r, i * C::NT + c * 32, vis, thr, scr, col, cnt, a.k);
         }
         ++ac;
       }
@@ -538,7 +772,7 @@ __global__ void __launch_bounds__(192, 1)
         tc::fence_proxy_async_smem();
         tc::mbar_arrive(aready);
       }
-      finalize(col, cnt, thr, a.k);
+      cut_to_k(col, cnt, thr, a.k, scr, true);
       // coalesced output: the warp writes its 32 rows one after another
       __syncwarp();
       for (int rr = 0; rr < 32; ++rr) {
