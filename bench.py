@@ -375,8 +375,17 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--heads", type=int, default=0,
+                    help="query heads (KV heads follow the workload's group size): a smaller case of the same "
+                         "shapes, for profiler captures")
     args = ap.parse_args()
     w = synth.WORKLOADS[args.workload]
+    if args.heads:
+        import dataclasses
+        if args.heads % w.group:
+            ap.error(f"--heads must be a multiple of the group size {w.group}")
+        w = dataclasses.replace(w, name=f"{w.name}_h{args.heads}", num_q_heads=args.heads,
+                                num_kv_heads=args.heads // w.group)
     if args.impl == "reference":
         run_reference(args, w)
     else:

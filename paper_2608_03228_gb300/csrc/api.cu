@@ -342,7 +342,8 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
   if ((st = cuda_status(cudaMemsetAsync(status, 0, nm * sizeof(int), s))) != SAKI_OK) return st;
   if (!cfg->center && mu && (st = cuda_status(cudaMemsetAsync(mu, 0, (size_t)Hk * kD * sizeof(float), s))) != SAKI_OK)
     return st;
-  if ((st = cuda_status(launch_gram(q_calib, k_calib, n_calib, Hq, Hk, cfg->center, cfg->dtype, S, muw, s))) != SAKI_OK)
+  if ((st = cuda_status(launch_gram(q_calib, k_calib, n_calib, Hq, Hk, cfg->center, cfg->dtype, S, muw, status, s))) !=
+      SAKI_OK)
     return st;
   if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK) return st;
   if ((st = cuda_status(launch_fit(A, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
@@ -354,6 +355,7 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
   if ((st = cuda_status(cudaStreamSynchronize(s))) != SAKI_OK) return st;
   int acc = 0;
   for (int v : hst) acc |= v;
+  if (acc & kStTimeout) return SAKI_ERR_TIMEOUT;
   if (acc & kStNonFinite) return SAKI_ERR_NUMERIC;
   if (acc & kStNotConverged) return SAKI_ERR_NOT_CONVERGED;
   return SAKI_OK;

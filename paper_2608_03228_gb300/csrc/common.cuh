@@ -13,7 +13,7 @@ constexpr int kD = 128;          // head dimension supported by this build
 constexpr int kLdS = kD + 1;     // padded leading dimension of d x d tiles in shared memory
 
 // Device status bits (one int per fitted matrix / head).
-enum : int { kStNonFinite = 1, kStNotConverged = 2 };
+enum : int { kStNonFinite = 1, kStNotConverged = 2, kStTimeout = 4 };
 
 // ---------------------------------------------------------------- dtype helpers
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }

@@ -41,35 +41,55 @@ __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_count
     __syncthreads();
     int rot = 0;
     for (int round = 0; round < kD - 1; ++round) {
-#pragma unroll 1
+      // the warp's four pairs of this round side by side: their loads, products
+      // and butterfly reductions interleave instead of forming one long chain
+      float* xa[4];
+      float* xb[4];
+      float a[4][4], b[4][4], al[4], be[4], ga[4];
+#pragma unroll
       for (int q = 0; q < 4; ++q) {
         int pa, pb;
         rr_pair(round, warp * 4 + q, pa, pb);
-        float* xa = X + pa * kLdS;
-        float* xb = X + pb * kLdS;
-        float a[4], b[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) { a[u] = xa[lane + 32 * u]; b[u] = xb[lane + 32 * u]; }
-        float al = 0.f, be = 0.f, ga = 0.f;
+        xa[q] = X + pa * kLdS;
+        xb[q] = X + pb * kLdS;
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          al = fmaf(a[u], a[u], al);
-          be = fmaf(b[u], b[u], be);
-          ga = fmaf(a[u], b[u], ga);
+          a[q][u] = xa[q][lane + 32 * u];
+          b[q][u] = xb[q][lane + 32 * u];
         }
-        al = warp_sum(al);  // xor butterflies leave identical values in every lane
-        be = warp_sum(be);
-        ga = warp_sum(ga);
-        if (ga != 0.f && fabsf(ga) > tol * sqrtf(al) * sqrtf(be)) {
-          const float zeta = (be - al) / (2.f * ga);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        al[q] = 0.f;
+        be[q] = 0.f;
+        ga[q] = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          al[q] = fmaf(a[q][u], a[q][u], al[q]);
+          be[q] = fmaf(b[q][u], b[q][u], be[q]);
+          ga[q] = fmaf(a[q][u], b[q][u], ga[q]);
+        }
+      }
+#pragma unroll
+      for (int m = 16; m > 0; m >>= 1)  // xor butterflies leave identical values in every lane
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          al[q] += __shfl_xor_sync(0xffffffffu, al[q], m);
+          be[q] += __shfl_xor_sync(0xffffffffu, be[q], m);
+          ga[q] += __shfl_xor_sync(0xffffffffu, ga[q], m);
+        }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (ga[q] != 0.f && fabsf(ga[q]) > tol * sqrtf(al[q]) * sqrtf(be[q])) {
+          const float zeta = (be[q] - al[q]) / (2.f * ga[q]);
           const float t = fabsf(zeta) > 1e18f ? 0.5f / zeta
                                               : copysignf(1.f, zeta) / (fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
           const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
-          const float s = c * t;
+          const float sn = c * t;
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            xa[lane + 32 * u] = c * a[u] - s * b[u];
-            xb[lane + 32 * u] = s * a[u] + c * b[u];
+            xa[q][lane + 32 * u] = c * a[q][u] - sn * b[q][u];
+            xb[q][lane + 32 * u] = sn * a[q][u] + c * b[q][u];
           }
           ++rot;
         }

@@ -50,9 +50,10 @@ cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, 
 cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s);
 size_t score_generic_smem(int P, int kp, int nq);
 
-// calibration moments: S [(Hq+Hk)][d][d] (queries first), mu [Hk][d]
+// calibration moments: S [(Hq+Hk)][d][d] (queries first), mu [Hk][d]; err: set to 1
+// if a bounded wait of the tensor-core path gave up
 cudaError_t launch_gram(const void* q_calib, const void* k_calib, int64_t n, int Hq, int Hk,
-                        int center, int dtype, float* S, float* mu, cudaStream_t s);
+                        int center, int dtype, float* S, float* mu, int* err, cudaStream_t s);
 
 // factor F (F F^T = S, floor applied) and G = pseudo-inverse transpose of F, per matrix
 cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps,

@@ -39,9 +39,10 @@ constexpr int kScr = 36;      // per-row scratch stride (words): 32 scores + pad
 
 template <int P>
 struct TcCfg {
-  static constexpr int NT = P == 128 ? 128 : 256;            // keys per tile (MMA N)
-  static constexpr int STAGES = P <= 32 ? 4 : 2;
-  static constexpr int CAP = P == 128 ? 104 : 128;            // candidate slots per row (multiple of 8)
+  static constexpr int NT = 128;                              // keys per tile (MMA N)
+  static constexpr int NB = 4;                                // TMEM accumulator ring (lets the warps drift)
+  static constexpr int STAGES = P == 128 ? 2 : 4;
+  static constexpr int CAP = P == 128 ? 104 : (P == 64 ? 136 : 176);   // candidate slots per row (multiple of 8)
   static constexpr int KB = P == 128 ? 2 : 1;                 // 64-wide K blocks
   static constexpr int KW = P == 128 ? 64 : P;                // K width of one block
   static constexpr int KK = KW / 16;                          // MMA K steps per block
@@ -52,7 +53,7 @@ struct TcCfg {
   static constexpr int STAGE_BYTES = NT * P * 2;
   static constexpr int CAND_BYTES = CAP * kLdc * 4 + ((CAP * kLdc * 2 + 15) & ~15);
   static constexpr int SCR_BYTES = 128 * kScr * 4;
-  static constexpr int TMEM_COLS = 2 * NT;
+  static constexpr int TMEM_COLS = NB * NT;
   static constexpr int OFF_STAGE = A_BYTES;
   static constexpr int OFF_CAND = OFF_STAGE + STAGES * STAGE_BYTES;
   static constexpr int OFF_SCR = OFF_CAND + CAND_BYTES;
@@ -389,23 +390,23 @@ __device__ __forceinline__ void fold32(const uint32_t (&r)[32], float (&g1)[kGro
 }
 
 // The certified bound of pass 1: a value tau with at least k of the 128 kept
-// values >= tau, taken from a sorted sample of 16 of them (the highest sample
+// values >= tau, taken from a sorted sample of 32 of them (the highest sample
 // that qualifies), or -inf if none does (then every visible key is a candidate).
 __device__ __forceinline__ float select_tau(const float (&g1)[kGroups], const float (&g2)[kGroups], int k) {
-  float s[16];
+  float s[32];
 #pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    s[u] = g1[8 * u + 3];
-    s[8 + u] = g2[8 * u + 5];
+  for (int u = 0; u < 16; ++u) {
+    s[u] = g1[4 * u + 1];
+    s[16 + u] = g2[4 * u + 3];
   }
-  sort_desc<16>(s);
-  // sample q (0-based) has about (q + 1) * 128 / 17 values at or above it
-  int q = (17 * k) / (2 * kGroups);
-  q = q > 15 ? 15 : q;
+  sort_desc<32>(s);
+  // sample q (0-based) has about (q + 1) * 128 / 33 values at or above it
+  int q = (33 * k) / (2 * kGroups);
+  q = q > 31 ? 31 : q;
   float tau = -INFINITY;
   bool pending = true;
-  for (int attempt = 0; attempt < 4; ++attempt) {
-    const float p = pick<16>(s, q);
+  for (int attempt = 0; attempt < 6; ++attempt) {
+    const float p = pick<32>(s, q);
     int n0 = 0, n1 = 0;
 #pragma unroll
     for (int g = 0; g < kGroups; ++g) {
@@ -416,47 +417,51 @@ __device__ __forceinline__ float select_tau(const float (&g1)[kGroups], const fl
       tau = p;
       pending = false;
     }
-    if (q == 15) pending = false;
-    q = q < 15 ? q + 1 : 15;
+    if (q == 31) pending = false;
+    q = q < 31 ? q + 1 : 31;
     if (!__any_sync(0xffffffffu, pending)) break;
   }
   return tau;
 }
 
-__device__ __forceinline__ uint32_t above_mask(const uint32_t (&r)[32], int j0, int vis, float thr) {
-  uint32_t m4[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-  for (int u = 0; u < 32; ++u) m4[u & 3] |= (__uint_as_float(r[u]) > thr ? 1u : 0u) << u;
-  uint32_t mask = (m4[0] | m4[1]) | (m4[2] | m4[3]);
-  const int nv = vis - j0;
-  if (nv < 32) mask &= nv > 0 ? (0xffffffffu >> (32 - nv)) : 0u;
-  return mask;
-}
-
 // Pass 2: append the keys of 32 scores of a row (keys j0 .. j0+31) that score
-// above thr and are visible; a column that would overflow is first cut to its
-// k best (which raises thr; CAP >= k + 32 leaves room for the chunk).
+// above thr and are visible.  A column that could overflow is first cut to its
+// k best if the chunk's appends would not fit (which raises thr; CAP >= k + 32
+// leaves room for the chunk).  The appends are predicated stores at a running
+// slot pointer: no mask, no scratch, no data-dependent loop.
 template <int CAP>
 __device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vis, float& thr, float* scr,
                                          const Col& c, int& cnt, int k) {
-  uint32_t mask = above_mask(r, j0, vis, thr);
-  const bool over = cnt + __popc(mask) > CAP;
-  if (__any_sync(0xffffffffu, over)) {
-    cut_to_k(c, cnt, thr, k, scr, over);
-    mask = above_mask(r, j0, vis, thr);
-  }
-  if (!__any_sync(0xffffffffu, mask != 0)) return;
+  float v[32];
 #pragma unroll
-  for (int q = 0; q < 8; ++q)
-    *reinterpret_cast<uint4*>(scr + 4 * q) = make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]);
-  while (__any_sync(0xffffffffu, mask != 0)) {
-    if (mask) {
-      const int u = __ffs(mask) - 1;
-      mask &= mask - 1;
-      c.put(cnt, scr[u], j0 + u);
-      ++cnt;
-    }
+  for (int u = 0; u < 32; ++u) v[u] = __uint_as_float(r[u]);
+  if (j0 + 32 > vis) {
+#pragma unroll
+    for (int u = 0; u < 32; ++u)
+      if (j0 + u >= vis) v[u] = -INFINITY;
   }
+  if (__any_sync(0xffffffffu, cnt > CAP - 32)) {
+    int n = 0;
+#pragma unroll
+    for (int u = 0; u < 32; ++u) n += v[u] > thr ? 1 : 0;
+    const bool over = cnt + n > CAP;
+    if (__any_sync(0xffffffffu, over)) cut_to_k(c, cnt, thr, k, scr, over);
+  }
+  float* ps = c.bs + cnt * kLdc + c.row;
+  uint16_t* pi = c.bi + cnt * kLdc + c.row;
+  int added = 0;
+#pragma unroll
+  for (int u = 0; u < 32; ++u) {
+    const bool t = v[u] > thr;
+    if (t) {
+      *ps = v[u];
+      *pi = (uint16_t)(j0 + u);
+    }
+    ps += t ? kLdc : 0;
+    pi += t ? kLdc : 0;
+    added += t ? 1 : 0;
+  }
+  cnt += added;
 }
 
 template <int P>
@@ -530,8 +535,8 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* empty = full + C::STAGES;
   uint64_t* accf = empty + C::STAGES;
-  uint64_t* acce = accf + 2;
-  uint64_t* qfull = acce + 2;
+  uint64_t* acce = accf + C::NB;
+  uint64_t* qfull = acce + C::NB;
   uint64_t* afree = qfull + 1;
   uint64_t* aready = afree + 1;
   uint64_t* drain = aready + 1;
@@ -544,7 +549,7 @@ __global__ void __launch_bounds__(192, 1)
       tc::mbar_init(full + s, 1);
       tc::mbar_init(empty + s, 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < C::NB; ++b) {
       tc::mbar_init(accf + b, 1);
       tc::mbar_init(acce + b, 128);
     }
@@ -626,8 +631,8 @@ __global__ void __launch_bounds__(192, 1)
       for (int item = blockIdx.x; item < a.n_items; item += gridDim.x, ++it) {
         const TcTile t = a.tiles[item / Hq];
         if (!tc::mbar_wait(qfull, it & 1, abort_f)) break;
-        uint32_t buf = ac & 1;
-        if (!tc::mbar_wait(acce + buf, ((ac >> 1) & 1) ^ 1, abort_f)) break;
+        uint32_t buf = ac % C::NB;
+        if (!tc::mbar_wait(acce + buf, ((ac / C::NB) & 1) ^ 1, abort_f)) break;
         tc::fence_after_sync();
         bool ok = true;
         uint32_t acc = 0;
@@ -652,8 +657,8 @@ __global__ void __launch_bounds__(192, 1)
         tc::fence_after_sync();
         const int ntiles = (t.vis_max + C::NT - 1) / C::NT;
         for (int i = 0; i < 2 * ntiles; ++i) {
-          buf = ac & 1;
-          if (!(ok = tc::mbar_wait(acce + buf, ((ac >> 1) & 1) ^ 1, abort_f))) break;
+          buf = ac % C::NB;
+          if (!(ok = tc::mbar_wait(acce + buf, ((ac / C::NB) & 1) ^ 1, abort_f))) break;
           const int st = sc % C::STAGES;
           if (!(ok = tc::mbar_wait(full + st, (sc / C::STAGES) & 1, abort_f))) break;
           tc::fence_after_sync();
@@ -695,8 +700,8 @@ __global__ void __launch_bounds__(192, 1)
       const TcTile t = a.tiles[item / Hq];
       const int h = item % Hq;
       if (it == 0) {  // this item's projection (later items convert theirs ahead of time)
-        const uint32_t buf = ac & 1;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac >> 1) & 1, abort_f));
+        const uint32_t buf = ac % C::NB;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
         convert_projection<P>(tl + buf * C::NT, sA, m);
@@ -716,22 +721,25 @@ __global__ void __launch_bounds__(192, 1)
         g2[g] = -INFINITY;
       }
       for (int i = 0; i < ntiles; ++i) {
-        const uint32_t buf = ac & 1;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac >> 1) & 1, abort_f));
+        const uint32_t buf = ac % C::NB;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
+        // chunk c + 1 is read from TMEM while chunk c is folded
+        uint32_t ra[32], rb[32];
+        __syncwarp();
+        tc::tmem_ld32(tl + buf * C::NT, ra);
+        tc::tmem_ld_wait(ra);
 #pragma unroll
         for (int c = 0; c < C::NT / 32; ++c) {
-          uint32_t r[32];
-          __syncwarp();
-          tc::tmem_ld32(tl + buf * C::NT + c * 32, r);
-          tc::tmem_ld_wait();
-          if (c == C::NT / 32 - 1) {
-            tc::fence_before_sync();
-            tc::mbar_arrive(acce + buf);
-          }
-          fold32(r, g1, g2, (c % 2) * 32, i * C::NT + c * 32, vis);
+          uint32_t(&cur)[32] = (c & 1) ? rb : ra;
+          uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
+          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::NT + (c + 1) * 32, nxt);
+          fold32(cur, g1, g2, (c % 2) * 32, i * C::NT + c * 32, vis);
+          if (c + 1 < C::NT / 32) tc::tmem_ld_wait(nxt);
         }
+        tc::fence_before_sync();
+        tc::mbar_arrive(acce + buf);
         ++ac;
       }
       if (!ok) break;
@@ -739,30 +747,34 @@ __global__ void __launch_bounds__(192, 1)
       float thr = below(select_tau(g1, g2, a.k));
       // pass 2: candidates scoring >= tau
       for (int i = 0; i < ntiles; ++i) {
-        const uint32_t buf = ac & 1;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac >> 1) & 1, abort_f));
+        const uint32_t buf = ac % C::NB;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
-#pragma unroll 1
+        uint32_t ra[32], rb[32];
+        __syncwarp();
+        tc::tmem_ld32(tl + buf * C::NT, ra);
+        tc::tmem_ld_wait(ra);
+#pragma unroll
         for (int c = 0; c < C::NT / 32; ++c) {
-          uint32_t r[32];
+          uint32_t(&cur)[32] = (c & 1) ? rb : ra;
+          uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
           __syncwarp();
-          tc::tmem_ld32(tl + buf * C::NT + c * 32, r);
-          tc::tmem_ld_wait();
-          if (c == C::NT / 32 - 1) {
-            tc::fence_before_sync();
-            tc::mbar_arrive(acce + buf);
-          }
-          append32<C::CAP>(r, i * C::NT + c * 32, vis, thr, scr, col, cnt, a.k);
+          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::NT + (c + 1) * 32, nxt);
+          append32<C::CAP>(cur, i * C::NT + c * 32, vis, thr, scr, col, cnt, a.k);
+          __syncwarp();
+          if (c + 1 < C::NT / 32) tc::tmem_ld_wait(nxt);
         }
+        tc::fence_before_sync();
+        tc::mbar_arrive(acce + buf);
         ++ac;
       }
       if (!ok) break;
       // convert the next item's projection now, so the tensor core can move on
       const int nxt = item + gridDim.x;
       if (nxt < a.n_items) {
-        const uint32_t buf = ac & 1;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac >> 1) & 1, abort_f));
+        const uint32_t buf = ac % C::NB;
+        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
         convert_projection<P>(tl + buf * C::NT, sA, m);
