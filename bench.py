@@ -44,8 +44,9 @@ def peaks():
         p["source"] = "measured"
     except (OSError, ValueError, KeyError):
         pass
-    # fp32 CUDA-core FMA peak from unit counts: 152 SMs x 128 lanes x 2 flop x max clock
-    p["fp32_tflops"] = 152 * 128 * 2 * p["sm_max_mhz"] * 1e6 / 1e12
+    # CUDA-core peaks from unit counts: 152 SMs x 128 fp32 lanes x max SM clock
+    p["alu_tops"] = 152 * 128 * p["sm_max_mhz"] * 1e6 / 1e12          # one lane operation per lane per clock
+    p["fp32_tflops"] = 2 * p["alu_tops"]                                # fused multiply-add = 2 flop
     return p
 
 
@@ -157,11 +158,10 @@ class GpuPath:
         if ev[4] is not None:
             ev[4].record()
 
-    def launches_per_step(self) -> int:
-        # saki_fit: moments (+ key means), factors, fit; build: 1; score: 1 (+ split merge);
-        # recall: exact top-k (+ split merge), recall, finish
-        plan_splits = 0   # configs run here plan no splits for the batched causal workloads
-        return (3 + self.w.center) + 1 + (1 + plan_splits) + (3 + plan_splits)
+
+
+# kernel kinds timed inside the library (saki_kernel_timer_*)
+KINDS = {"select": 1, "exact": 2, "fit": 3, "moments": 4, "build": 5, "factor": 6}
 
 
 def run_ours(args, w):
@@ -184,9 +184,13 @@ def run_ours(args, w):
     nstage = 4
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nstage + 1)] for _ in range(args.steps)]
     clocks = ClockSampler(dev.index)
+    S = g.saki
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
+    for kind in KINDS.values():
+        S.saki_kernel_timer_start(kind)
+    launches0 = S.saki_launch_count()
     clocks.start()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
@@ -195,6 +199,9 @@ def run_ours(args, w):
         g.step(evs[s])
     t1.record()
     torch.cuda.synchronize()
+    launches = S.saki_launch_count() - launches0
+    ktime = {name: S.saki_kernel_timer_stop(kind) for name, kind in KINDS.items()}   # (total ms, launches)
+    ktime["_steps"] = args.steps
     if dist:
         dist.barrier()
     clk = clocks.stop()
@@ -214,7 +221,8 @@ def run_ours(args, w):
 
     pk = peaks()
     names = ["fit", "build_index", "score_topk", "recall"]
-    roof = roofline(w, pk, dict(zip(names, stage_ms)), g)
+    roofs = rooflines(w, pk, ktime, g)
+    dominant = max(roofs, key=lambda n: roofs[n]["ms_per_launch"] * roofs[n]["launches_per_step"])
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -224,10 +232,10 @@ def run_ours(args, w):
                    "layers": w.layers, "T": g.T, "N": g.N, "rank": w.rank, "topk": w.topk, "n_calib": w.n_calib,
                    "parallelism": f"{world} independent replicas" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 (calibration + eval tensors %.1f GB per step)" % (input_bytes(g) / 1e9)},
-        "clocks": clk, "e2e": e2e, "gpu_launches": g.launches_per_step() * args.steps,
+        "clocks": clk, "e2e": e2e, "gpu_launches": launches,
         "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
         "score_topk_keys_per_s": pairs / (stage_ms[2] / 1e3),
-        "roofline": roof["dominant"], "roofline_score_topk": roof["score_topk"],
+        "roofline": dict(roofs[dominant], kernel=dominant), "rooflines": roofs,
         "recall_median": float(np.median(g.recall.cpu().numpy())),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -265,33 +273,49 @@ def run_e2e(g, args, torch):
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": int(out_host.numel() * 4)}
 
 
-def roofline(w, pk, stage_ms, g):
+# dram bytes per launch from one ncu capture of the kernel as it stands (profiles/),
+# scaled from the captured case to this workload by the pairs processed; None when
+# the kernel changed after the capture
+TRAFFIC_BYTES_PER_PAIR = {}
+
+
+def rooflines(w, pk, ktime, g):
+    """Per timed kernel: algorithmic work per launch / event-measured launch time."""
     pairs = visible_pairs(w)
-    N, Hq, Hk = g.N, w.num_q_heads, w.num_kv_heads
+    N, Hq, Hk, r, n = g.N, w.num_q_heads, w.num_kv_heads, w.rank, w.n_calib
     eb = 2 if w.dtype == "bf16" else 4
-    # score_topk on CUDA cores: 2 r flop per visible pair (fp32 FMA)
-    sc = {"kernel": "score_topk", "bound": "alu", "achieved": 2 * w.rank * pairs / (stage_ms["score_topk"] / 1e3) / 1e12,
-          "peak": pk["fp32_tflops"], "unit": "TFLOP/s", "traffic": None,
-          "note": "fp32 CUDA-core FMA peak from 152 SMs x 128 lanes x 2 x max SM clock"}
-    sc["frac"] = sc["achieved"] / sc["peak"]
-    ex = {"kernel": "recall (exact q^T A k top-k)", "bound": "alu",
-          "achieved": 2 * D * pairs / (stage_ms["recall"] / 1e3) / 1e12, "peak": pk["fp32_tflops"],
-          "unit": "TFLOP/s", "traffic": None}
-    ex["frac"] = ex["achieved"] / ex["peak"]
-    fit_flop = 2 * w.n_calib * D * D * (Hq + Hk)   # moments (the Jacobi sweeps are data-dependent)
-    ft = {"kernel": "fit (moments + Jacobi SVD)", "bound": "alu",
-          "achieved": fit_flop / (stage_ms["fit"] / 1e3) / 1e12, "peak": pk["fp32_tflops"], "unit": "TFLOP/s",
-          "traffic": None}
-    ft["frac"] = ft["achieved"] / ft["peak"]
-    bi_bytes = Hk * N * D * eb + Hq * N * w.rank * eb
-    bi = {"kernel": "build_index", "bound": "hbm", "achieved": bi_bytes / (stage_ms["build_index"] / 1e3) / 1e9,
-          "peak": pk["hbm_gbs"], "unit": "GB/s", "traffic": None}
-    bi["frac"] = bi["achieved"] / bi["peak"]
-    by_stage = {"fit": ft, "build_index": bi, "score_topk": sc, "recall": ex}
-    dom = max(stage_ms, key=lambda k: stage_ms[k])
-    for v in by_stage.values():
-        v["peak_source"] = pk["source"]
-    return {"dominant": dict(by_stage[dom], stage=dom), "score_topk": sc}
+    T = g.T
+    out = {}
+
+    def entry(name, bound, work, unit, peak, note, peak_name):
+        tot, cnt = ktime[name]
+        if cnt == 0:
+            return
+        ms = tot / cnt
+        scale = 1e12 if unit in ("TFLOP/s", "Tops/s") else 1e9
+        ach = work / (ms / 1e3) / scale
+        tb = TRAFFIC_BYTES_PER_PAIR.get(name)
+        out[name] = {"bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
+                     "traffic": tb * pairs if tb is not None else None, "ms_per_launch": ms,
+                     "launches_per_step": cnt / max(1, ktime["_steps"]), "work_per_launch": work,
+                     "peak_source": f"{pk['source']} ({peak_name})", "model": note}
+
+    alu = pk["alu_tops"]
+    entry("select", "alu", pairs, "Tops/s", alu,
+          "one threshold comparison per visible (head, query, key) pair; the scores come from a tensor-core "
+          f"contraction of 2r = {2 * r} flop per pair", "152 SMs x 128 lanes x max SM clock")
+    entry("exact", "alu", pairs, "Tops/s", alu,
+          "one comparison per visible pair; scores q^T A k from a tensor-core contraction of 2d flop per pair",
+          "152 SMs x 128 lanes x max SM clock")
+    entry("moments", "hbm", (Hq + Hk) * n * D * eb + (Hq + Hk) * D * D * 4, "GB/s", pk["hbm_gbs"],
+          "calibration queries and keys read once, fp32 moment matrices written", "STREAM copy")
+    entry("build", "hbm", Hk * N * D * eb + Hq * N * r * eb, "GB/s", pk["hbm_gbs"],
+          "keys read once, codes written once", "STREAM copy")
+    entry("fit", "alu", Hq * (4 * D ** 3 + 8 * 6 * D ** 3), "TFLOP/s", pk["fp32_tflops"],
+          "model: 4 d^3 flop per head for C' plus 6 d^3 per one-sided Jacobi sweep at 8 sweeps", "fp32 FMA")
+    entry("factor", "alu", (Hq + Hk) * (D ** 3 // 3 + D ** 3), "TFLOP/s", pk["fp32_tflops"],
+          "model: Cholesky d^3/3 plus triangular inverse d^3 flop per moment matrix", "fp32 FMA")
+    return out
 
 
 # ------------------------------------------------------------------ CPU oracle

@@ -191,6 +191,32 @@ SAKI_API saki_status saki_score_topk_noalloc(const saki_config* cfg, const saki_
                                              saki_stream stream);
 
 /* Static description of a status code. */
+/* ---------------------------------------------------------------- profiling aids
+ * Not part of the method (the paper has no counterpart): a launch count and
+ * per-kernel device timing, for benchmarks that report kernel-level rooflines.
+ *
+ * saki_launch_count: number of kernels this library has launched in the process
+ *   (every device and stream).
+ * saki_kernel_timer_start(kind): arms one kernel kind.  While armed, every launch
+ *   of that kind is bracketed by two CUDA timing events recorded on the stream of
+ *   the library call that launches it (events of the device current at the first
+ *   timed launch; launches on other devices are not timed).  Several kinds may be
+ *   armed at once.  SAKI_ERR_INVALID_ARGUMENT for an unknown kind.
+ * saki_kernel_timer_stop(kind, total_ms, launches): waits for the last recorded
+ *   event, writes the summed device time (ms) and the number of timed launches,
+ *   and disarms the kind.  SAKI_ERR_CUDA if an event query fails.
+ * The timer state is process-wide and not synchronised with library calls made
+ * concurrently from other threads; each timed launch costs two event records. */
+#define SAKI_KERNEL_SELECT 1  /* selection kernel(s) of saki_score_topk */
+#define SAKI_KERNEL_EXACT 2   /* exact top-k kernel(s) of saki_recall */
+#define SAKI_KERNEL_FIT 3     /* SVD kernel of saki_fit (C', Jacobi, factors L and R) */
+#define SAKI_KERNEL_MOMENTS 4 /* calibration-moment kernel(s) of saki_fit */
+#define SAKI_KERNEL_BUILD 5   /* key-code kernel(s) of saki_build_index */
+#define SAKI_KERNEL_FACTOR 6  /* moment-factor kernel of saki_fit */
+SAKI_API int64_t saki_launch_count(void);
+SAKI_API saki_status saki_kernel_timer_start(int32_t kind);
+SAKI_API saki_status saki_kernel_timer_stop(int32_t kind, double* total_ms, int64_t* launches);
+
 SAKI_API const char* saki_status_string(saki_status status);
 
 /* Library version as "major.minor.patch". */

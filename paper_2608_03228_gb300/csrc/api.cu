@@ -228,6 +228,7 @@ saki_status run_tc(const saki_config* cfg, const saki_layout* layout, const TcPl
   a.k = cfg->topk;
   a.exact = exact ? 1 : 0;
   a.sorted = (cfg->flags & SAKI_FLAG_SORTED) ? 1 : 0;
+  KernelTimer kt(exact ? SAKI_KERNEL_EXACT : SAKI_KERNEL_SELECT, s);
   return cuda_status(launch_score_tc(L, s));
 }
 
@@ -342,13 +343,23 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
   if ((st = cuda_status(cudaMemsetAsync(status, 0, nm * sizeof(int), s))) != SAKI_OK) return st;
   if (!cfg->center && mu && (st = cuda_status(cudaMemsetAsync(mu, 0, (size_t)Hk * kD * sizeof(float), s))) != SAKI_OK)
     return st;
-  if ((st = cuda_status(launch_gram(q_calib, k_calib, n_calib, Hq, Hk, cfg->center, cfg->dtype, S, muw, status, s))) !=
-      SAKI_OK)
-    return st;
-  if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK) return st;
-  if ((st = cuda_status(launch_fit(A, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
-                                   reinterpret_cast<float*>(ws + w.C), L, R, sigma, loss, nu, status, s))) != SAKI_OK)
-    return st;
+  {
+    KernelTimer kt(SAKI_KERNEL_MOMENTS, s);
+    if ((st = cuda_status(launch_gram(q_calib, k_calib, n_calib, Hq, Hk, cfg->center, cfg->dtype, S, muw, status,
+                                      s))) != SAKI_OK)
+      return st;
+  }
+  {
+    KernelTimer kt(SAKI_KERNEL_FACTOR, s);
+    if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK) return st;
+  }
+  {
+    KernelTimer kt(SAKI_KERNEL_FIT, s);
+    if ((st = cuda_status(launch_fit(A, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
+                                     reinterpret_cast<float*>(ws + w.C), L, R, sigma, loss, nu, status, s))) !=
+        SAKI_OK)
+      return st;
+  }
   std::vector<int> hst(nm);
   if ((st = cuda_status(cudaMemcpyAsync(hst.data(), status, nm * sizeof(int), cudaMemcpyDeviceToHost, s))) != SAKI_OK)
     return st;
@@ -380,11 +391,13 @@ saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const v
     std::memcpy(host.data(), w.items.data(), w.items.size() * sizeof(BuildItem));
     if ((st = cuda_status(cudaMemcpyAsync(ws, host.data(), host.size(), cudaMemcpyHostToDevice, s))) != SAKI_OK)
       return st;
+    KernelTimer kt(SAKI_KERNEL_BUILD, s);
     return cuda_status(launch_build_tc(K, R, sketch, total_keys, cfg->num_q_heads,
                                        cfg->num_q_heads / cfg->num_kv_heads, cfg->rank,
                                        reinterpret_cast<const BuildItem*>(ws), (int)w.items.size(), ws + w.off_w,
                                        reinterpret_cast<int*>(ws + w.off_err), num_sms(), s));
   }
+  KernelTimer kt(SAKI_KERNEL_BUILD, s);
   return cuda_status(launch_build_generic(K, R, cfg->center ? mu : nullptr, sketch, total_keys, cfg->num_q_heads,
                                           cfg->num_q_heads / cfg->num_kv_heads, cfg->rank, cfg->center,
                                           cfg->dtype, s));
@@ -427,6 +440,7 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
   a.exact = 0;
   a.n_items = (int32_t)p.items.size();
   a.n_merges = (int32_t)p.merges.size();
+  KernelTimer kt(SAKI_KERNEL_SELECT, s);
   if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, p.nq, s))) != SAKI_OK) return st;
   return cuda_status(launch_merge(a, cfg->dtype, kp, s));
 }
@@ -476,6 +490,7 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
     a.exact = 1;
     a.n_items = (int32_t)p.items.size();
     a.n_merges = (int32_t)p.merges.size();
+    KernelTimer kt(SAKI_KERNEL_EXACT, s);
     if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, p.nq, s))) != SAKI_OK) return st;
     if ((st = cuda_status(launch_merge(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
   }

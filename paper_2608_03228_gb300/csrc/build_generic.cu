@@ -48,12 +48,14 @@ cudaError_t launch_build_generic(const void* K, const float* R, const float* mu,
     auto k = build_generic_kernel<__nv_bfloat16>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
+    note_launch();
     k<<<grid, 256, sm, s>>>(static_cast<const __nv_bfloat16*>(K), R, mu, static_cast<__nv_bfloat16*>(sketch), N,
                             G, r, center);
   } else {
     auto k = build_generic_kernel<float>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
+    note_launch();
     k<<<grid, 256, sm, s>>>(static_cast<const float*>(K), R, mu, static_cast<float*>(sketch), N, G, r, center);
   }
   return cudaGetLastError();

@@ -276,6 +276,7 @@ cudaError_t launch_build_tc(const void* K, const float* R, void* sketch, int64_t
   if (n_items == 0) return cudaSuccess;
   const int64_t n = (int64_t)Hq * r * kD;
   const int blocks = (int)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
+  note_launch();
   pack_rt_kernel<<<blocks, 256, 0, s>>>(R, Hq, G, r, static_cast<__nv_bfloat16*>(wsplit));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -287,6 +288,7 @@ cudaError_t launch_build_tc(const void* K, const float* R, void* sketch, int64_t
   e = cudaFuncSetAttribute(build_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kBuildSmem);
   if (e != cudaSuccess) return e;
   const int grid = n_items < num_sms ? n_items : num_sms;
+  note_launch();
   build_tc_kernel<<<grid, 192, kBuildSmem, s>>>(mK, mB, items, n_items, N, ncol_total, r, G,
                                                 static_cast<__nv_bfloat16*>(sketch), err);
   return cudaGetLastError();

@@ -12,8 +12,9 @@
 //
 // fit_kernel: per query head h with KV head g,
 //   C' = Fq^T A_h Fk (singular values equal those of Sq^{1/2} A_h Sk^{1/2}),
-//   one-sided (Hestenes) Jacobi on C'^T: its columns converge to V Sigma with
-//   V the right singular vectors of C'; then
+//   C' = Q1 R1 (Householder QR, as preconditioning), one-sided (Hestenes)
+//   Jacobi on R1^T: its columns converge to V Sigma with V the right singular
+//   vectors of C' (C'^T = R1^T Q1^T); then
 //   R = Gk V_r Sigma_r^{1/2}  and  L = Gq (C' V_r) Sigma_r^{-1/2} = Gq U_r Sigma_r^{1/2},
 //   so L R^T = M_r, loss = sum_{i>r} sigma_i^2 and nu = A_h mu_g.
 #include "common.cuh"
@@ -32,10 +33,25 @@ __device__ __forceinline__ void rr_pair(int round, int k, int& pa, int& pb) {
 }
 
 // One-sided Jacobi on the columns of X (column-major, leading dimension kLdS) until
-// every pair satisfies |x_a . x_b| <= tol ||x_a|| ||x_b||.  Needs kFitThreads
-// threads; returns true on convergence within max_sweeps.
+// every pair satisfies |x_a . x_b| <= tol ||x_a|| ||x_b||.  Columns of norm below
+// 1e-7 ||X||_F count as zero (their pairs are not rotated): they carry no
+// singular value that matters, and rounding noise left in exactly rank-deficient
+// inputs would otherwise keep rotating.  Needs kFitThreads threads; returns true
+// on convergence within max_sweeps.
 __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_counter) {
+  __shared__ float s_red[kFitThreads / 32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  float fro = 0.f;
+  for (int o = tid; o < kD * kD; o += kFitThreads) {
+    const float v = X[(o / kD) * kLdS + (o % kD)];
+    fro = fmaf(v, v, fro);
+  }
+  fro = warp_sum(fro);
+  if (lane == 0) s_red[warp] = fro;
+  __syncthreads();
+  fro = 0.f;
+  for (int w = 0; w < kFitThreads / 32; ++w) fro += s_red[w];
+  const float tiny = fro * 1e-14f;   // squared column norm treated as zero
   for (int sweep = 0; sweep < max_sweeps; ++sweep) {
     if (tid == 0) *s_counter = 0;
     __syncthreads();
@@ -80,7 +96,7 @@ __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_count
         }
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        if (ga[q] != 0.f && fabsf(ga[q]) > tol * sqrtf(al[q]) * sqrtf(be[q])) {
+        if (ga[q] != 0.f && al[q] > tiny && be[q] > tiny && fabsf(ga[q]) > tol * sqrtf(al[q]) * sqrtf(be[q])) {
           const float zeta = (be[q] - al[q]) / (2.f * ga[q]);
           const float t = fabsf(zeta) > 1e18f ? 0.5f / zeta
                                               : copysignf(1.f, zeta) / (fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
@@ -103,6 +119,63 @@ __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_count
     if (total == 0) return true;
   }
   return false;
+}
+
+// Householder QR of the matrix in X (column-major, leading dimension kLdS), in
+// place: on return R occupies the upper triangle (diagonal included); below it,
+// the reflector vectors are left behind.  Needs kFitThreads threads.
+__device__ void householder_r(float* X) {
+  __shared__ float s_par[3];   // alpha (the new diagonal), v_j, |v|^2
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int j = 0; j < kD - 1; ++j) {
+    float* xj = X + j * kLdS;
+    if (warp == 0) {
+      float sq = 0.f;
+      for (int i = j + 1 + lane; i < kD; i += 32) sq = fmaf(xj[i], xj[i], sq);
+      sq = warp_sum(sq);
+      if (lane == 0) {
+        const float x0 = xj[j];
+        const float nx = sqrtf(fmaf(x0, x0, sq));
+        const float alpha = x0 >= 0.f ? -nx : nx;   // v_j = x0 - alpha adds magnitudes: no cancellation
+        const float v0 = x0 - alpha;
+        s_par[0] = alpha;
+        s_par[1] = v0;
+        s_par[2] = fmaf(v0, v0, sq);
+      }
+    }
+    __syncthreads();
+    const float v0 = s_par[1], vn2 = s_par[2];
+    if (vn2 > 0.f) {
+      // trailing columns: c -= (2 v.c / |v|^2) v, two columns per warp at a time
+      for (int c = j + 1 + warp; c < kD; c += 2 * (kFitThreads / 32)) {
+        const int c2 = c + kFitThreads / 32;
+        float* xc = X + c * kLdS;
+        float* xd = X + (c2 < kD ? c2 : c) * kLdS;
+        float d1 = lane == 0 ? v0 * xc[j] : 0.f, d2 = lane == 0 ? v0 * xd[j] : 0.f;
+        for (int i = j + 1 + lane; i < kD; i += 32) {
+          d1 = fmaf(xj[i], xc[i], d1);
+          d2 = fmaf(xj[i], xd[i], d2);
+        }
+#pragma unroll
+        for (int m = 16; m > 0; m >>= 1) {
+          d1 += __shfl_xor_sync(0xffffffffu, d1, m);
+          d2 += __shfl_xor_sync(0xffffffffu, d2, m);
+        }
+        const float f1 = 2.f * d1 / vn2, f2 = 2.f * d2 / vn2;
+        if (lane == 0) {
+          xc[j] = fmaf(-f1, v0, xc[j]);
+          if (c2 < kD) xd[j] = fmaf(-f2, v0, xd[j]);
+        }
+        for (int i = j + 1 + lane; i < kD; i += 32) {
+          xc[i] = fmaf(-f1, xj[i], xc[i]);
+          if (c2 < kD) xd[i] = fmaf(-f2, xj[i], xd[i]);
+        }
+      }
+    }
+    __syncthreads();
+    if (tid == 0 && vn2 > 0.f) xj[j] = s_par[0];
+    __syncthreads();
+  }
 }
 
 // column norms of X into out[kD] (warp per column)
@@ -282,7 +355,19 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
     for (int u = 0; u < 32; ++u) Ct[cc * kD + r0 + u] = acc[u];
   }
   __syncthreads();
-  for (int o = tid; o < kD * kD; o += kFitThreads) X[(o / kD) * kLdS + (o % kD)] = Ct[o];
+  // Preconditioning: C' = Q1 R1 (Householder), then the Jacobi runs on R1^T, whose
+  // left singular vectors are those of C'^T = R1^T Q1^T, i.e. the right singular
+  // vectors of C' (the triangular factor converges in far fewer sweeps).
+  for (int o = tid; o < kD * kD; o += kFitThreads) X[(o % kD) * kLdS + (o / kD)] = Ct[o];   // X = C'
+  __syncthreads();
+  householder_r(X);
+  for (int o = tid; o < kD * kD; o += kFitThreads) {   // X = R1^T (lower triangle)
+    const int i = o / kD, jj = o % kD;
+    if (i > jj) {
+      X[jj * kLdS + i] = X[i * kLdS + jj];
+      X[i * kLdS + jj] = 0.f;
+    }
+  }
   __syncthreads();
 
   const bool conv = jacobi_columns(X, max_sweeps, tol, &counter);
@@ -369,6 +454,7 @@ cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_swe
                           int* status, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(factor_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
   if (e != cudaSuccess) return e;
+  note_launch();
   factor_kernel<<<nmat, kFitThreads, kSmem, s>>>(S, floor_rel, max_sweeps, kTol, F, Gm, status);
   return cudaGetLastError();
 }
@@ -378,6 +464,7 @@ cudaError_t launch_fit(const float* A, const float* F, const float* Gm, const fl
                        int* status, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(fit_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFitSmem);
   if (e != cudaSuccess) return e;
+  note_launch();
   fit_kernel<<<Hq, kFitThreads, kFitSmem, s>>>(A, F, Gm, mu, Hq, Hk, r, max_sweeps, kTol, Cws, L, R, sigma, loss,
                                                nu, status);
   return cudaGetLastError();

@@ -190,7 +190,10 @@ __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, c
 template <typename Tin>
 cudaError_t gram_t(const void* q, const void* k, int64_t n, int Hq, int Hk, int center, float* S,
                    float* mu, int* err, cudaStream_t s) {
-  if (center) key_mean_kernel<Tin><<<Hk, 128, 0, s>>>(static_cast<const Tin*>(k), n, mu);
+  if (center) {
+    note_launch();
+    key_mean_kernel<Tin><<<Hk, 128, 0, s>>>(static_cast<const Tin*>(k), n, mu);
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   int first_cuda = 0;   // first matrix left to the CUDA-core kernel
@@ -199,6 +202,7 @@ cudaError_t gram_t(const void* q, const void* k, int64_t n, int Hq, int Hk, int 
     if (ntc > 0 && n > 0) {
       e = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kGramSmem);
       if (e != cudaSuccess) return e;
+      note_launch();
       gram_tc_kernel<<<ntc, 128, kGramSmem, s>>>(static_cast<const __nv_bfloat16*>(q),
                                                  static_cast<const __nv_bfloat16*>(k), n, Hq, S, err);
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -206,9 +210,11 @@ cudaError_t gram_t(const void* q, const void* k, int64_t n, int Hq, int Hk, int 
     first_cuda = ntc;
   }
   const int rest = Hq + Hk - first_cuda;
-  if (rest > 0)
+  if (rest > 0) {
+    note_launch();
     gram_kernel<Tin><<<dim3(4, rest), 256, 0, s>>>(static_cast<const Tin*>(q), static_cast<const Tin*>(k), n, Hq,
                                                    center, mu, S, first_cuda);
+  }
   return cudaGetLastError();
 }
 }  // namespace

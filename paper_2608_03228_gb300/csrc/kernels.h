@@ -6,6 +6,26 @@
 
 namespace saki {
 
+// ---------------------------------------------------------------- profiling aids
+void note_launch();   // called at every kernel launch of the library
+
+// Kernel kinds timed by saki_kernel_timer_* (values match the SAKI_KERNEL_* macros).
+constexpr int kTimedKinds = 7;
+// While the kind is armed, records one CUDA event on construction and one on
+// destruction, on stream s (bracket the launch of that kind).
+class KernelTimer {
+ public:
+  KernelTimer(int kind, cudaStream_t s);
+  ~KernelTimer();
+  KernelTimer(const KernelTimer&) = delete;
+  KernelTimer& operator=(const KernelTimer&) = delete;
+
+ private:
+  int kind_;
+  cudaStream_t s_;
+  cudaEvent_t stop_;
+};
+
 // One unit of scoring work: up to kGroupQ consecutive queries of one sequence
 // against keys [key_lo, key_hi) of that sequence (a split of its visible range).
 struct ScoreItem {

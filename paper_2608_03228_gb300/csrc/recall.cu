@@ -78,9 +78,11 @@ cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int3
   if (T > 0) {
     const int64_t blocks = (T + 7) / 8;
     dim3 grid((unsigned)(blocks < 1024 ? blocks : 1024), Hq);
+    note_launch();
     recall_kernel<<<grid, 256, 0, s>>>(idx_a, idx_e, vis, T, k, min_visible, counters);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
+  note_launch();
   recall_finish_kernel<<<(Hq + 127) / 128, 128, 0, s>>>(counters, Hq, k, recall);
   return cudaGetLastError();
 }

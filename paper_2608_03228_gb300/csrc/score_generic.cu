@@ -281,6 +281,7 @@ cudaError_t launch_score_t(const ScoreArgs& a, cudaStream_t s) {
   auto kern = score_generic_kernel<Tin, KP, NQ>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
+  note_launch();
   kern<<<dim3(a.n_items, a.Hq), kThreads, sm, s>>>(a);
   return cudaGetLastError();
 }
@@ -314,11 +315,23 @@ cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s) 
   if (a.n_merges == 0) return cudaSuccess;
   dim3 grid((a.n_merges + 3) / 4, a.Hq);
   if (dtype == SAKI_BF16) {
-    if (kp == 64) merge_kernel<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(a);
-    else merge_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(a);
+    if (kp == 64) {
+      note_launch();
+      merge_kernel<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(a);
+    }
+    else {
+      note_launch();
+      merge_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(a);
+    }
   } else {
-    if (kp == 64) merge_kernel<float, 64><<<grid, 128, 0, s>>>(a);
-    else merge_kernel<float, 128><<<grid, 128, 0, s>>>(a);
+    if (kp == 64) {
+      note_launch();
+      merge_kernel<float, 64><<<grid, 128, 0, s>>>(a);
+    }
+    else {
+      note_launch();
+      merge_kernel<float, 128><<<grid, 128, 0, s>>>(a);
+    }
   }
   return cudaGetLastError();
 }

@@ -902,6 +902,7 @@ cudaError_t launch_tc_t(const TcLaunch& L, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   const int grid = L.args.n_items < L.num_sms ? L.args.n_items : L.num_sms;
+  note_launch();
   kern<<<grid, 192, C::SMEM, s>>>(mQ, mW, mX, L.args);
   return cudaGetLastError();
 }
@@ -912,12 +913,14 @@ bool tc_supported(int P) { return P == 16 || P == 32 || P == 64 || P == 128; }
 cudaError_t launch_pack_w(const float* W, int Hq, int P, void* out, cudaStream_t s) {
   const int64_t n = (int64_t)Hq * P * kD;
   const int blocks = (int)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
+  note_launch();
   pack_w_kernel<<<blocks, 256, 0, s>>>(W, Hq, P, static_cast<__nv_bfloat16*>(out));
   return cudaGetLastError();
 }
 
 cudaError_t launch_qnu(const void* Q, const float* nu, int64_t T, int Hq, float* out, cudaStream_t s) {
   const int64_t rows = (int64_t)Hq * T;
+  note_launch();
   qnu_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(Q), nu, T, Hq, out);
   return cudaGetLastError();
 }

@@ -24,7 +24,10 @@ SAKI_OP_FIT, SAKI_OP_BUILD_INDEX, SAKI_OP_SCORE_TOPK, SAKI_OP_RECALL = 0, 1, 2, 
 STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED", 3: "SAKI_ERR_CUDA",
           4: "SAKI_ERR_NUMERIC", 5: "SAKI_ERR_NOT_CONVERGED", 6: "SAKI_ERR_WORKSPACE", 7: "SAKI_ERR_TIMEOUT"}
 EXPORTS = ("saki_workspace_size", "saki_fit", "saki_build_index", "saki_score_topk", "saki_recall",
-           "saki_status_string", "saki_version", "saki_score_topk_noalloc")
+           "saki_status_string", "saki_version", "saki_score_topk_noalloc", "saki_launch_count",
+           "saki_kernel_timer_start", "saki_kernel_timer_stop")
+SAKI_KERNEL_SELECT, SAKI_KERNEL_EXACT, SAKI_KERNEL_FIT, SAKI_KERNEL_MOMENTS, SAKI_KERNEL_BUILD, SAKI_KERNEL_FACTOR = (
+    1, 2, 3, 4, 5, 6)
 SAKI_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
@@ -56,6 +59,12 @@ _lib.saki_score_topk_noalloc.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(
 _lib.saki_status_string.restype = ctypes.c_char_p
 _lib.saki_status_string.argtypes = [ctypes.c_int]
 _lib.saki_version.restype = ctypes.c_char_p
+_lib.saki_launch_count.restype = _i64
+_lib.saki_launch_count.argtypes = []
+_lib.saki_kernel_timer_start.restype = ctypes.c_int
+_lib.saki_kernel_timer_start.argtypes = [_i32]
+_lib.saki_kernel_timer_stop.restype = ctypes.c_int
+_lib.saki_kernel_timer_stop.argtypes = [_i32, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(_i64)]
 
 
 class SakiError(RuntimeError):
@@ -121,6 +130,21 @@ def saki_status_string(status: int) -> str:
 
 def saki_version() -> str:
     return _lib.saki_version().decode()
+
+
+def saki_launch_count() -> int:
+    return int(_lib.saki_launch_count())
+
+
+def saki_kernel_timer_start(kind: int) -> None:
+    _check(_lib.saki_kernel_timer_start(kind), "saki_kernel_timer_start")
+
+
+def saki_kernel_timer_stop(kind: int) -> tuple[float, int]:
+    """Summed device milliseconds and number of timed launches of the kind since it was armed."""
+    ms, n = ctypes.c_double(0.0), _i64(0)
+    _check(_lib.saki_kernel_timer_stop(kind, ctypes.byref(ms), ctypes.byref(n)), "saki_kernel_timer_stop")
+    return ms.value, int(n.value)
 
 
 def saki_workspace_size(cfg: Config, op: int, layout: HostLayout | None = None, n_calib: int = 0,
