@@ -57,62 +57,55 @@ __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_count
     __syncthreads();
     int rot = 0;
     for (int round = 0; round < kD - 1; ++round) {
-      // the warp's four pairs of this round side by side: their loads, products
-      // and butterfly reductions interleave instead of forming one long chain
-      float* xa[4];
-      float* xb[4];
-      float a[4][4], b[4][4], al[4], be[4], ga[4];
+      // eight lanes per pair: lane group q = lane / 8 of the warp holds rows
+      // sub + 8u (u < 16) of the pair's two columns, so a dot product needs only
+      // three butterfly steps inside the group, and the four pairs run side by side
+      // pair index (warp % 8) + 8 q + 32 (warp / 8): the four groups' columns sit 8
+      // apart, so their 8-bank windows of shared memory do not overlap
+      const int q = lane >> 3, sub = lane & 7;
+      int pa, pb;
+      rr_pair(round, (warp & 7) + 8 * q + 32 * (warp >> 3), pa, pb);
+      float* xa = X + pa * kLdS + sub;
+      float* xb = X + pb * kLdS + sub;
+      float a[16], b[16];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        int pa, pb;
-        rr_pair(round, warp * 4 + q, pa, pb);
-        xa[q] = X + pa * kLdS;
-        xb[q] = X + pb * kLdS;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          a[q][u] = xa[q][lane + 32 * u];
-          b[q][u] = xb[q][lane + 32 * u];
-        }
+      for (int u = 0; u < 16; ++u) {
+        a[u] = xa[8 * u];
+        b[u] = xb[8 * u];
       }
+      float al0 = 0.f, al1 = 0.f, be0 = 0.f, be1 = 0.f, ga0 = 0.f, ga1 = 0.f;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        al[q] = 0.f;
-        be[q] = 0.f;
-        ga[q] = 0.f;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          al[q] = fmaf(a[q][u], a[q][u], al[q]);
-          be[q] = fmaf(b[q][u], b[q][u], be[q]);
-          ga[q] = fmaf(a[q][u], b[q][u], ga[q]);
-        }
+      for (int u = 0; u < 16; u += 2) {
+        al0 = fmaf(a[u], a[u], al0);
+        al1 = fmaf(a[u + 1], a[u + 1], al1);
+        be0 = fmaf(b[u], b[u], be0);
+        be1 = fmaf(b[u + 1], b[u + 1], be1);
+        ga0 = fmaf(a[u], b[u], ga0);
+        ga1 = fmaf(a[u + 1], b[u + 1], ga1);
       }
+      float al = al0 + al1, be = be0 + be1, ga = ga0 + ga1;
 #pragma unroll
-      for (int m = 16; m > 0; m >>= 1)  // xor butterflies leave identical values in every lane
+      for (int m = 4; m > 0; m >>= 1) {  // butterflies leave the group's sums in all eight lanes
+        al += __shfl_xor_sync(0xffffffffu, al, m);
+        be += __shfl_xor_sync(0xffffffffu, be, m);
+        ga += __shfl_xor_sync(0xffffffffu, ga, m);
+      }
+      if (ga != 0.f && al > tiny && be > tiny && fabsf(ga) > tol * sqrtf(al) * sqrtf(be)) {
+        const float zeta = (be - al) / (2.f * ga);
+        const float t = fabsf(zeta) > 1e18f ? 0.5f / zeta
+                                            : copysignf(1.f, zeta) / (fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
+        const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
+        const float sn = c * t;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          al[q] += __shfl_xor_sync(0xffffffffu, al[q], m);
-          be[q] += __shfl_xor_sync(0xffffffffu, be[q], m);
-          ga[q] += __shfl_xor_sync(0xffffffffu, ga[q], m);
+        for (int u = 0; u < 16; ++u) {
+          xa[8 * u] = c * a[u] - sn * b[u];
+          xb[8 * u] = sn * a[u] + c * b[u];
         }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        if (ga[q] != 0.f && al[q] > tiny && be[q] > tiny && fabsf(ga[q]) > tol * sqrtf(al[q]) * sqrtf(be[q])) {
-          const float zeta = (be[q] - al[q]) / (2.f * ga[q]);
-          const float t = fabsf(zeta) > 1e18f ? 0.5f / zeta
-                                              : copysignf(1.f, zeta) / (fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
-          const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
-          const float sn = c * t;
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            xa[q][lane + 32 * u] = c * a[q][u] - sn * b[q][u];
-            xb[q][lane + 32 * u] = sn * a[q][u] + c * b[q][u];
-          }
-          ++rot;
-        }
+        if (sub == 0) ++rot;
       }
       __syncthreads();
     }
-    if (lane == 0 && rot) atomicAdd(s_counter, rot);
+    if ((lane & 7) == 0 && rot) atomicAdd(s_counter, rot);   // one counter per pair group
     __syncthreads();
     const int total = *s_counter;
     __syncthreads();
