@@ -266,30 +266,53 @@ def input_bytes(g) -> int:
 
 
 def run_e2e(g, args, torch):
+    """The step through the public API with the inputs in pinned host memory: every
+    step copies its inputs host-to-device and reads its recall vector back, inside
+    the timed region.  Inputs are double-buffered on the device and copied on a
+    second stream, so step i+1's copies overlap step i's kernels (as a pipeline
+    over successive batches would run)."""
     keys = ("q_calib", "k_calib", "A", "Q", "K")
     host = {k: g.data[k].cpu().pin_memory() for k in keys}
-    dev = {k: torch.empty_like(g.data[k]) for k in keys}
+    bufs = [{k: torch.empty_like(g.data[k]) for k in keys} for _ in range(2)]
     out_host = torch.empty((g.w.num_q_heads,), dtype=torch.float32).pin_memory()
     steps = max(2, min(args.steps, 5))
+    comp = torch.cuda.current_stream()
+    copy = torch.cuda.Stream()
     for k in keys:   # one untimed round trip: first use of the pinned buffers and of the copy engines
-        dev[k].copy_(host[k], non_blocking=True)
-    g.step(inputs=dev)
+        bufs[0][k].copy_(host[k], non_blocking=True)
+    g.step(inputs=bufs[0])
     out_host.copy_(g.recall, non_blocking=True)
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
-    t0.record()
-    for _ in range(steps):
-        for k in keys:
-            dev[k].copy_(host[k], non_blocking=True)
-        g.step(inputs=dev)
+    copied = [torch.cuda.Event() for _ in range(steps)]
+    used = [torch.cuda.Event() for _ in range(steps)]
+
+    def issue_copy(i):
+        with torch.cuda.stream(copy):
+            copy.wait_event(t0)
+            if i >= 2:
+                copy.wait_event(used[i - 2])      # the kernels of step i-2 read this buffer
+            for k in keys:
+                bufs[i % 2][k].copy_(host[k], non_blocking=True)
+            copied[i].record(copy)
+
+    t0.record(comp)
+    issue_copy(0)
+    for i in range(steps):
+        if i + 1 < steps:
+            issue_copy(i + 1)
+        comp.wait_event(copied[i])
+        g.step(inputs=bufs[i % 2])
+        used[i].record(comp)
         out_host.copy_(g.recall, non_blocking=True)
-    t1.record()
+    t1.record(comp)
     torch.cuda.synchronize()
     ms = t0.elapsed_time(t1) / steps
     h2d = sum(int(host[k].numel() * host[k].element_size()) for k in keys)
     return {"value": visible_pairs(g.w) / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "steps": steps,
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": int(out_host.numel() * 4)}
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": int(out_host.numel() * 4),
+            "overlap": "step i+1's host-to-device copies run on a second stream during step i"}
 
 
 # DRAM bytes (read + write) per visible pair, from one ncu capture of each kernel

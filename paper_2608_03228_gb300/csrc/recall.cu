@@ -1,65 +1,113 @@
 // Recall of the Sec. 3 protocol: per (head, query) with at least min_visible
-// visible keys, |approx set & exact set| / k, averaged per head.  A warp per
-// row inserts the approximate indices into a small open-addressing table in
-// shared memory and probes it with the exact ones; integer counts per head are
-// accumulated with atomics, so the per-head value is exact and order-free.
+// visible keys, |approx set & exact set| / k, averaged per head.  A warp walks a
+// contiguous range of (head, query) rows; per row it inserts the approximate
+// indices into a small open-addressing table in shared memory, probes it with
+// the exact ones and clears only the slots it used.  Integer counts per head
+// are flushed with atomics when the head changes, so the per-head value is
+// exact and order-free.
 #include "common.cuh"
 #include "kernels.h"
 
 namespace saki {
 namespace {
-constexpr int kSlots = 256;   // >= 2 k for k <= 128
+constexpr int kSlots = 256;       // >= 2 k for k <= 128
+constexpr int kPerLane = 4;       // k <= 128 indices per list: at most 4 per lane
 
 __device__ __forceinline__ uint32_t slot_of(int32_t v) { return ((uint32_t)v * 2654435761u) >> 24; }
 
 __global__ void __launch_bounds__(256) recall_kernel(const int32_t* ia, const int32_t* ie, const int32_t* vis,
-                                                     int64_t T, int k, int64_t min_visible,
+                                                     int64_t T, int Hq, int k, int64_t min_visible,
                                                      unsigned long long* counters) {
   __shared__ int32_t tab[8][kSlots];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int h = blockIdx.y;
   int32_t* tb = tab[warp];
-  unsigned long long matches = 0, rows = 0;
   for (int o = lane; o < kSlots; o += 32) tb[o] = -1;
   __syncwarp();
-  for (int64_t t = (int64_t)blockIdx.x * 8 + warp; t < T; t += (int64_t)gridDim.x * 8) {
-    if (vis[t] < min_visible) continue;   // warp-uniform
-    const int32_t* a = ia + ((int64_t)h * T + t) * k;
-    const int32_t* e = ie + ((int64_t)h * T + t) * k;
-    for (int i = lane; i < k; i += 32) {
-      const int32_t v = a[i];
-      if (v < 0) continue;
-      uint32_t s = slot_of(v);
+  const int64_t total = (int64_t)Hq * T;
+  const int64_t nwarps = (int64_t)gridDim.x * 8;
+  const int64_t per = (total + nwarps - 1) / nwarps;
+  const int64_t r0 = ((int64_t)blockIdx.x * 8 + warp) * per;
+  const int64_t r1 = r0 + per < total ? r0 + per : total;
+  int cur_h = -1;
+  unsigned long long matches = 0, rows = 0;
+  // the next row's two index lists are loaded while this row is matched
+  int32_t na[kPerLane], ne[kPerLane];
+  int64_t nt = r0 % T;   // query of the next row; its head follows from the row index
+  int nh = (int)(r0 / T);
+  int32_t nvis = r0 < r1 ? __ldg(vis + nt) : 0;
+  auto load_row = [&](int64_t r, int32_t (&va)[kPerLane], int32_t (&ve)[kPerLane]) {
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      const int i = lane + 32 * u;
+      const bool in = r < r1 && i < k;
+      va[u] = in ? __ldg(ia + r * k + i) : -1;
+      ve[u] = in ? __ldg(ie + r * k + i) : -1;
+    }
+  };
+  load_row(r0, na, ne);
+  for (int64_t r = r0; r < r1; ++r) {
+    int32_t av[kPerLane], ev[kPerLane];
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      av[u] = na[u];
+      ev[u] = ne[u];
+    }
+    const int h = nh;
+    const int32_t row_vis = nvis;
+    if (++nt == T) {
+      nt = 0;
+      ++nh;
+    }
+    nvis = r + 1 < r1 ? __ldg(vis + nt) : 0;
+    load_row(r + 1, na, ne);
+    if (h != cur_h) {
+      if (lane == 0 && rows) {
+        atomicAdd(counters + 2 * cur_h, matches);
+        atomicAdd(counters + 2 * cur_h + 1, rows);
+      }
+      cur_h = h;
+      matches = rows = 0;
+    }
+    if (row_vis < min_visible) continue;   // warp-uniform
+    uint32_t used[kPerLane];
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) used[u] = kSlots;
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      if (av[u] < 0) continue;
+      uint32_t sl = slot_of(av[u]);
       while (true) {
-        const int32_t prev = atomicCAS(&tb[s], -1, v);
-        if (prev == -1 || prev == v) break;
-        s = (s + 1) & (kSlots - 1);
+        const int32_t prev = atomicCAS(&tb[sl], -1, av[u]);
+        if (prev == -1) { used[u] = sl; break; }
+        if (prev == av[u]) break;
+        sl = (sl + 1) & (kSlots - 1);
       }
     }
     __syncwarp();
     int m = 0;
-    for (int i = lane; i < k; i += 32) {
-      const int32_t v = e[i];
-      if (v < 0) continue;
-      uint32_t s = slot_of(v);
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      if (ev[u] < 0) continue;
+      uint32_t sl = slot_of(ev[u]);
       while (true) {
-        const int32_t cur = tb[s];
-        if (cur == v) { ++m; break; }
+        const int32_t cur = tb[sl];
+        if (cur == ev[u]) { ++m; break; }
         if (cur == -1) break;
-        s = (s + 1) & (kSlots - 1);
+        sl = (sl + 1) & (kSlots - 1);
       }
     }
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) m += __shfl_xor_sync(0xffffffffu, m, d);
-    matches += m;
+    m = (int)warp_sum((float)m);
+    matches += (unsigned long long)m;
     rows += 1;
     __syncwarp();
-    for (int o = lane; o < kSlots; o += 32) tb[o] = -1;
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u)
+      if (used[u] < kSlots) tb[used[u]] = -1;
     __syncwarp();
   }
   if (lane == 0 && rows) {
-    atomicAdd(counters + 2 * h, matches);
-    atomicAdd(counters + 2 * h + 1, rows);
+    atomicAdd(counters + 2 * cur_h, matches);
+    atomicAdd(counters + 2 * cur_h + 1, rows);
   }
 }
 
@@ -76,10 +124,13 @@ cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int3
   cudaError_t e = cudaMemsetAsync(counters, 0, sizeof(unsigned long long) * 2 * Hq, s);
   if (e != cudaSuccess) return e;
   if (T > 0) {
-    const int64_t blocks = (T + 7) / 8;
-    dim3 grid((unsigned)(blocks < 1024 ? blocks : 1024), Hq);
+    int dev = 0, sms = 152;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t rows = (int64_t)Hq * T;
+    const int64_t want = (rows + 7) / 8;   // at least one row per warp
+    const int64_t blocks = want < (int64_t)sms * 4 ? want : (int64_t)sms * 4;
     note_launch();
-    recall_kernel<<<grid, 256, 0, s>>>(idx_a, idx_e, vis, T, k, min_visible, counters);
+    recall_kernel<<<(unsigned)blocks, 256, 0, s>>>(idx_a, idx_e, vis, T, Hq, k, min_visible, counters);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   note_launch();
