@@ -427,7 +427,8 @@ __device__ __forceinline__ float select_tau(const float (&g1)[kGroups], const fl
 // Pass 2: append the keys of 32 scores of a row (keys j0 .. j0+31) that score
 // above thr and are visible.  A column that could overflow is first cut to its
 // k best if the chunk's appends would not fit (which raises thr; CAP >= k + 32
-// leaves room for the chunk).  The appends are predicated stores at a running
+// leaves room for the chunk), together with every column of the warp that is
+// close to the capacity.  The appends are predicated stores at a running
 // slot pointer: no mask, no scratch, no data-dependent loop.
 template <int CAP>
 __device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vis, float& thr, float* scr,
@@ -445,7 +446,10 @@ __device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vi
 #pragma unroll
     for (int u = 0; u < 32; ++u) n += v[u] > thr ? 1 : 0;
     const bool over = cnt + n > CAP;
-    if (__any_sync(0xffffffffu, over)) cut_to_k(c, cnt, thr, k, scr, over);
+    // a cut costs the warp about the same for one row as for all 32: when one
+    // row must be cut, every row close to the capacity is cut in the same call
+    const int near = (k + 8 > CAP - 40) ? k + 8 : CAP - 40;
+    if (__any_sync(0xffffffffu, over)) cut_to_k(c, cnt, thr, k, scr, over || cnt > near);
   }
   float* ps = c.bs + cnt * kLdc + c.row;
   uint16_t* pi = c.bi + cnt * kLdc + c.row;
