@@ -2,8 +2,11 @@
 // host-side work plan of the selection kernels, and launches.  No device
 // memory is allocated here; every buffer belongs to the caller.
 #include <algorithm>
+#include <array>
 #include <climits>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <vector>
 
 #include "common.cuh"
@@ -12,6 +15,90 @@
 using namespace saki;
 
 namespace {
+
+thread_local bool t_pageable_only = false;
+
+// Pinned host staging for the library's own small transfers (per-call plans up,
+// the fit's status words down).  A pageable copy is staged by the driver through
+// its bounce buffers, which can stall behind large copies the caller runs on
+// other streams; these go through a ring of pinned slots per device instead.  A
+// slot is reused only after the event recorded behind its last copy completed.
+class Staging {
+ public:
+  // host -> device: n bytes of src to dst, ordered on s
+  cudaError_t upload(void* dst, const void* src, size_t n, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    if (t_pageable_only) return cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s);
+    std::lock_guard<std::mutex> lock(mu_);
+    Slot* sl = nullptr;
+    cudaError_t e = take(n, &sl);
+    if (e != cudaSuccess) return e;
+    std::memcpy(sl->p, src, n);
+    if ((e = cudaMemcpyAsync(dst, sl->p, n, cudaMemcpyHostToDevice, s)) != cudaSuccess) return e;
+    return cudaEventRecord(sl->ev, s);
+  }
+  // device -> host: n bytes of src to dst; waits for the stream
+  cudaError_t download_sync(void* dst, const void* src, size_t n, cudaStream_t s) {
+    if (t_pageable_only) {
+      const cudaError_t e = cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, s);
+      return e != cudaSuccess ? e : cudaStreamSynchronize(s);
+    }
+    std::lock_guard<std::mutex> lock(mu_);
+    Slot* sl = nullptr;
+    cudaError_t e = take(n, &sl);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaMemcpyAsync(sl->p, src, n, cudaMemcpyDeviceToHost, s)) != cudaSuccess) return e;
+    if ((e = cudaEventRecord(sl->ev, s)) != cudaSuccess) return e;
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return e;
+    std::memcpy(dst, sl->p, n);
+    return cudaSuccess;
+  }
+
+ private:
+  struct Slot {
+    void* p = nullptr;
+    size_t cap = 0;
+    cudaEvent_t ev = nullptr;
+  };
+  struct Ring {
+    std::array<Slot, 4> slot;
+    int next = 0;
+  };
+  cudaError_t take(size_t n, Slot** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    Ring& ring = rings_[dev];
+    Slot& sl = ring.slot[ring.next];
+    ring.next = (ring.next + 1) % (int)ring.slot.size();
+    if (sl.ev && (e = cudaEventSynchronize(sl.ev)) != cudaSuccess) return e;
+    if (!sl.ev && (e = cudaEventCreateWithFlags(&sl.ev, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if (sl.cap < n) {
+      if (sl.p) cudaFreeHost(sl.p);
+      sl.p = nullptr;
+      sl.cap = 0;
+      const size_t cap = std::max<size_t>(n, 64 << 10);
+      if ((e = cudaHostAlloc(&sl.p, cap, cudaHostAllocDefault)) != cudaSuccess) return e;
+      sl.cap = cap;
+    }
+    *out = &sl;
+    return cudaSuccess;
+  }
+  std::mutex mu_;
+  std::map<int, Ring> rings_;
+};
+
+}  // namespace
+
+PageableUploads::PageableUploads() : prev_(t_pageable_only) { t_pageable_only = true; }
+PageableUploads::~PageableUploads() { t_pageable_only = prev_; }
+
+namespace {
+
+Staging& staging() {
+  static Staging* st = new Staging();   // process lifetime: the pinned slots outlive every call
+  return *st;
+}
 
 constexpr size_t kAlign = 256;
 constexpr int kNumSMs = 152;
@@ -123,8 +210,7 @@ saki_status upload_plan(const Plan& p, char* ws, cudaStream_t s) {
   if (!p.merges.empty())
     std::memcpy(host.data() + p.off_merges, p.merges.data(), p.merges.size() * sizeof(MergeItem));
   if (!p.vis.empty()) std::memcpy(host.data() + p.off_vis, p.vis.data(), p.vis.size() * sizeof(int32_t));
-  return cudaMemcpyAsync(ws, host.data(), p.staged, cudaMemcpyHostToDevice, s) == cudaSuccess ? SAKI_OK
-                                                                                              : SAKI_ERR_CUDA;
+  return staging().upload(ws, host.data(), p.staged, s) == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA;
 }
 
 // Tensor-core plan: tiles of up to 128 consecutive queries of one sequence,
@@ -183,8 +269,7 @@ saki_status upload_tc_plan(const TcPlan& p, char* ws, cudaStream_t s) {
   std::vector<char> host(p.staged, 0);
   if (!p.tiles.empty()) std::memcpy(host.data(), p.tiles.data(), p.tiles.size() * sizeof(TcTile));
   if (!p.vis.empty()) std::memcpy(host.data() + p.off_vis, p.vis.data(), p.vis.size() * sizeof(int32_t));
-  return cudaMemcpyAsync(ws, host.data(), p.staged, cudaMemcpyHostToDevice, s) == cudaSuccess ? SAKI_OK
-                                                                                              : SAKI_ERR_CUDA;
+  return staging().upload(ws, host.data(), p.staged, s) == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA;
 }
 
 int num_sms() {
@@ -361,9 +446,7 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
       return st;
   }
   std::vector<int> hst(nm);
-  if ((st = cuda_status(cudaMemcpyAsync(hst.data(), status, nm * sizeof(int), cudaMemcpyDeviceToHost, s))) != SAKI_OK)
-    return st;
-  if ((st = cuda_status(cudaStreamSynchronize(s))) != SAKI_OK) return st;
+  if ((st = cuda_status(staging().download_sync(hst.data(), status, nm * sizeof(int), s))) != SAKI_OK) return st;
   int acc = 0;
   for (int v : hst) acc |= v;
   if (acc & kStTimeout) return SAKI_ERR_TIMEOUT;
@@ -389,8 +472,7 @@ saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const v
     char* ws = static_cast<char*>(workspace);
     std::vector<char> host(w.off_w, 0);
     std::memcpy(host.data(), w.items.data(), w.items.size() * sizeof(BuildItem));
-    if ((st = cuda_status(cudaMemcpyAsync(ws, host.data(), host.size(), cudaMemcpyHostToDevice, s))) != SAKI_OK)
-      return st;
+    if ((st = cuda_status(staging().upload(ws, host.data(), host.size(), s))) != SAKI_OK) return st;
     KernelTimer kt(SAKI_KERNEL_BUILD, s);
     return cuda_status(launch_build_tc(K, R, sketch, total_keys, cfg->num_q_heads,
                                        cfg->num_q_heads / cfg->num_kv_heads, cfg->rank,

@@ -9,6 +9,20 @@ namespace saki {
 // ---------------------------------------------------------------- profiling aids
 void note_launch();   // called at every kernel launch of the library
 
+// While alive on this thread, the library's plan uploads use plain pageable
+// copies instead of its pinned staging ring (whose first use allocates pinned
+// host memory): for the entry points that promise to allocate nothing.
+class PageableUploads {
+ public:
+  PageableUploads();
+  ~PageableUploads();
+  PageableUploads(const PageableUploads&) = delete;
+  PageableUploads& operator=(const PageableUploads&) = delete;
+
+ private:
+  bool prev_;
+};
+
 // Kernel kinds timed by saki_kernel_timer_* (values match the SAKI_KERNEL_* macros).
 constexpr int kTimedKinds = 7;
 // While the kind is armed, records one CUDA event on construction and one on

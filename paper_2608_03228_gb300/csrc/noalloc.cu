@@ -4,6 +4,7 @@
 #include <atomic>
 
 #include "common.cuh"
+#include "kernels.h"
 
 // The scratch.  On the host this name is only a stand-in for the device array
 // (passing it to a kernel would fault, or read host memory where the GPU can
@@ -26,5 +27,6 @@ extern "C" saki_status saki_score_topk_noalloc(const saki_config* cfg, const sak
     if (cudaGetSymbolAddress(&addr, g_noalloc_scratch) != cudaSuccess) return SAKI_ERR_CUDA;
     g_scratch_addr[dev].store(addr, std::memory_order_release);
   }
+  saki::PageableUploads pageable;   // no pinned staging either: its first use allocates
   return saki_score_topk(cfg, layout, Q, L, sketch, nu, idx, score, addr, SAKI_NOALLOC_SCRATCH_BYTES, stream);
 }
