@@ -225,27 +225,27 @@ __global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, flo
     for (int i = j + 1 + tid; i < kD; i += kFitThreads) Sb[i * kLdS + j] /= ljj;
     __syncthreads();
     if (tid == 0) Sb[j * kLdS + j] = ljj;
-    const int mm = kD - j - 1;
-    for (int o = tid; o < mm * mm; o += kFitThreads) {
-      const int i = j + 1 + o / mm, c = j + 1 + o % mm;
-      if (c <= i) Sb[i * kLdS + c] -= Sb[i * kLdS + j] * Sb[c * kLdS + j];
+    // trailing update of the lower triangle: a warp per row, lanes over columns
+    for (int i = j + 1 + warp; i < kD; i += kFitThreads / 32) {
+      const float lij = Sb[i * kLdS + j];
+      for (int c = j + 1 + lane; c <= i; c += 32) Sb[i * kLdS + c] = fmaf(-lij, Sb[c * kLdS + j], Sb[i * kLdS + c]);
     }
     __syncthreads();
   }
 
   bool chol_ok = (flag == 0);
   if (chol_ok) {
-    // Linv = F^{-1}, row by row; thread c owns column c
+    // Linv = F^{-1} by right-looking substitution on the identity: row i is
+    // divided by F_ii, then subtracted (times F_ri) from every row below it
+    for (int o = tid; o < kD * kD; o += kFitThreads) Xb[(o / kD) * kLdS + (o % kD)] = (o / kD == o % kD) ? 1.f : 0.f;
+    __syncthreads();
     for (int i = 0; i < kD; ++i) {
-      if (tid < kD) {
-        const int c = tid;
-        float v = 0.f;
-        if (c <= i) {
-          float acc = (c == i) ? 1.f : 0.f;
-          for (int p = c; p < i; ++p) acc -= Sb[i * kLdS + p] * Xb[p * kLdS + c];
-          v = acc / Sb[i * kLdS + i];
-        }
-        Xb[i * kLdS + c] = v;
+      const float inv = 1.f / Sb[i * kLdS + i];
+      if (tid <= i) Xb[i * kLdS + tid] *= inv;   // columns > i of row i are zero
+      __syncthreads();
+      for (int r = i + 1 + warp; r < kD; r += kFitThreads / 32) {
+        const float lri = Sb[r * kLdS + i];
+        for (int c = lane; c <= i; c += 32) Xb[r * kLdS + c] = fmaf(-lri, Xb[i * kLdS + c], Xb[r * kLdS + c]);
       }
       __syncthreads();
     }

@@ -789,7 +789,32 @@ __global__ void __launch_bounds__(192, 1)
         tc::mbar_arrive(aready);
       }
       cut_to_k(col, cnt, thr, a.k, scr, true);
-      // coalesced output: the warp writes its 32 rows one after another
+      if (!a.sorted && (a.k & 3) == 0) {
+        // unsorted lists: each thread writes its own row, four entries per store
+        if (m < t.nrows) {
+          const int64_t o = ((int64_t)h * a.T + t.q0 + m) * a.k;
+          const float qn = a.qnu ? a.qnu[(int64_t)h * a.T + t.q0 + m] : 0.f;
+#pragma unroll 4
+          for (int i = 0; i < a.k; i += 4) {
+            int4 v;
+            v.x = i < cnt ? col.j(i) : -1;
+            v.y = i + 1 < cnt ? col.j(i + 1) : -1;
+            v.z = i + 2 < cnt ? col.j(i + 2) : -1;
+            v.w = i + 3 < cnt ? col.j(i + 3) : -1;
+            *reinterpret_cast<int4*>(a.idx + o + i) = v;
+            if (a.score) {
+              float4 f;
+              f.x = i < cnt ? col.s(i) + qn : -INFINITY;
+              f.y = i + 1 < cnt ? col.s(i + 1) + qn : -INFINITY;
+              f.z = i + 2 < cnt ? col.s(i + 2) + qn : -INFINITY;
+              f.w = i + 3 < cnt ? col.s(i + 3) + qn : -INFINITY;
+              *reinterpret_cast<float4*>(a.score + o + i) = f;
+            }
+          }
+        }
+        continue;
+      }
+      // sorted lists: the warp sorts and writes its 32 rows one after another
       __syncwarp();
       for (int rr = 0; rr < 32; ++rr) {
         const int row = quarter * 32 + rr;
