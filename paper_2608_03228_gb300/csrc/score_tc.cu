@@ -26,6 +26,8 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "tc.cuh"
@@ -41,8 +43,12 @@ template <int P>
 struct TcCfg {
   static constexpr int NT = 128;                              // keys per tile (MMA N)
   static constexpr int NB = 4;                                // TMEM accumulator ring (lets the warps drift)
-  static constexpr int STAGES = P == 128 ? 2 : 4;
-  static constexpr int CAP = P == 128 ? 104 : (P == 64 ? 136 : 176);   // candidate slots per row (multiple of 8)
+  // ranks up to 64 store 32-bit key indices at a fixed distance from the
+  // scores (one slot pointer serves both stores of an append); rank 128 needs
+  // the room for its operands and keeps 16-bit indices in their own array
+  static constexpr bool WIDE = P <= 64;
+  static constexpr int STAGES = P >= 64 ? 2 : 4;
+  static constexpr int CAP = P == 128 ? 104 : 136;               // candidate slots per row (multiple of 8)
   static constexpr int KB = P == 128 ? 2 : 1;                 // 64-wide K blocks
   static constexpr int KW = P == 128 ? 64 : P;                // K width of one block
   static constexpr int KK = KW / 16;                          // MMA K steps per block
@@ -51,7 +57,8 @@ struct TcCfg {
   static constexpr int A_PART = 128 * P * 2;                  // u_hi (or u_lo) bytes
   static constexpr int A_BYTES = 2 * A_PART > 32768 ? 2 * A_PART : 32768;  // also holds the 128x128 query tile
   static constexpr int STAGE_BYTES = NT * P * 2;
-  static constexpr int CAND_BYTES = CAP * kLdc * 4 + ((CAP * kLdc * 2 + 15) & ~15);
+  static constexpr int IDX_BYTES = WIDE ? CAP * kLdc * 4 : ((CAP * kLdc * 2 + 15) & ~15);
+  static constexpr int CAND_BYTES = CAP * kLdc * 4 + IDX_BYTES;
   static constexpr int SCR_BYTES = 128 * kScr * 4;
   static constexpr int TMEM_COLS = NB * NT;
   static constexpr int OFF_STAGE = A_BYTES;
@@ -63,6 +70,8 @@ struct TcCfg {
   static_assert(CAP % 8 == 0 && CAP >= 64 + 32, "candidate capacity: k + one chunk of appends");
   static_assert(NT % 64 == 0, "a key tile covers whole key groups");
   static_assert(SMEM <= 232448, "shared memory budget");
+  static_assert(OFF_STAGE % 1024 == 0 && STAGE_BYTES % 1024 == 0, "swizzled TMA tiles sit on 1024-byte boundaries");
+  static_assert(OFF_SCR % 16 == 0 && OFF_BAR % 16 == 0, "16-byte scratch stores and 8-byte mbarriers stay aligned");
 };
 
 // ---------------------------------------------------------------- selection
@@ -78,9 +87,12 @@ struct TcCfg {
 // the warp's largest count with per-lane predicates, so the 32 rows of a warp
 // never split into separately executed paths.
 
-// A row's candidate column: scores (fp32) and key indices (16-bit; the host only
-// sends sequences of at most 65535 keys here).
-struct Col {
+// A row's candidate column: slot i holds a score (fp32) and its key index.
+// ColSplit keeps 16-bit indices in their own array (the host only sends
+// sequences of at most 65535 keys here); ColWide keeps 32-bit indices IOFF
+// words after their scores, so one slot pointer addresses both.
+struct ColSplit {
+  static constexpr bool kWide = false;
   float* bs;
   uint16_t* bi;
   int row;
@@ -90,7 +102,27 @@ struct Col {
     bs[i * kLdc + row] = v;
     bi[i * kLdc + row] = (uint16_t)k;
   }
+  __device__ __forceinline__ ColSplit at(int r) const { return ColSplit{bs, bi, r}; }
 };
+template <int IOFF>
+struct ColWide {
+  static constexpr bool kWide = true;
+  static constexpr int kIOff = IOFF;
+  float* bs;
+  int row;
+  __device__ __forceinline__ float s(int i) const { return bs[i * kLdc + row]; }
+  __device__ __forceinline__ int j(int i) const { return __float_as_int(bs[IOFF + i * kLdc + row]); }
+  __device__ __forceinline__ void put(int i, float v, int k) const {
+    bs[i * kLdc + row] = v;
+    bs[IOFF + i * kLdc + row] = __int_as_float(k);
+  }
+  __device__ __forceinline__ ColWide at(int r) const { return ColWide{bs, r}; }
+};
+template <class Col>
+__device__ __forceinline__ Col make_col(float* bs, uint16_t* bi, int row) {
+  if constexpr (Col::kWide) return Col{bs, row};
+  else return Col{bs, bi, row};
+}
 
 __device__ __forceinline__ int warp_max(int v) { return __reduce_max_sync(0xffffffffu, v); }
 
@@ -130,6 +162,7 @@ __device__ __forceinline__ float pick(const float (&s)[N], int q) {
 }
 
 // Entries scoring >= p among the lane's first cnt (slots read up to the warp's cmax).
+template <class Col>
 __device__ __forceinline__ int count_ge(const Col& c, int cnt, int cmax, float p) {
   int n0 = 0, n1 = 0;
   for (int i = 0; i < cmax; i += 8) {
@@ -146,6 +179,7 @@ __device__ __forceinline__ int count_ge(const Col& c, int cnt, int cmax, float p
 }
 
 // Lanes with `on` keep their entries scoring >= p (in place, order preserved).
+template <class Col>
 __device__ __forceinline__ int compact_ge(const Col& c, int cnt, int cmax, float p, bool on) {
   int w = 0;
   for (int i = 0; i < cmax; i += 8) {
@@ -171,6 +205,7 @@ __device__ __forceinline__ bool worse(float a, int ja, float b, int jb) { return
 
 // Lanes with `on` drop their worst entry (lowest score, then highest index) and
 // raise thr to its score.
+template <class Col>
 __device__ __forceinline__ void remove_worst(const Col& c, int& cnt, int cmax, float& thr, bool on) {
   float ws[4];
   int wj[4], wp[4];
@@ -200,6 +235,7 @@ __device__ __forceinline__ void remove_worst(const Col& c, int& cnt, int cmax, f
 // for a pivot leaving between k and tmax entries; thr becomes p (every later key
 // has a higher index, so a later key scoring exactly p loses to all kept ones).
 // Lanes for which no tried pivot qualifies keep their column unchanged.
+template <class Col>
 __device__ __forceinline__ void pivot_cut(const Col& c, int& cnt, float& thr, int k, int aim, int tmax, bool on) {
   const int cmax = warp_max(cnt);
   float s[8];
@@ -232,14 +268,17 @@ __device__ __forceinline__ void pivot_cut(const Col& c, int& cnt, float& thr, in
 }
 
 // Exact cut of the lanes with `on` to their k best entries (slots [0, k)); thr
-// rises to the k-th best score (a later key, with a higher index, must score
-// above it to matter).  Quickselect by counting: a bracket [lo, hi] around the
-// k-th entry (na entries score above hi, at most k; nb score at or above lo, at
-// least k) narrows with pivots taken from 16 sampled scores of the bracket until
-// at most 16 entries remain in it; the entries above hi are kept, and the
-// boundary entries, ranked as 64-bit (score, index) keys in registers, fill the
-// remaining places.  Lanes whose bracket cannot narrow (many equal scores) fall
-// back to pivot cuts and single removals.
+// rises to a lower bound of the k-th best score (a later key, with a higher
+// index, must score above it to matter).  Quickselect by counting over a
+// half-open bracket [lo, hi): na entries score >= hi (na <= k, all of them
+// kept) and nb score >= lo (nb >= k, so the k best all score >= lo).  A round
+// counts the entries at or above five pivots taken from 16 sorted samples of
+// the bracket around the k-th entry's expected rank and keeps the tightest
+// bracket; once at most 16 entries lie in [lo, hi), they are ranked as 64-bit
+// (score, index) keys in registers and fill the remaining places.  Lanes whose
+// bracket cannot narrow (many equal scores) fall back to pivot cuts and single
+// removals.
+template <class Col>
 __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int k, float* scr, bool on) {
   bool pending = on && cnt > k;
   if (!__any_sync(0xffffffffu, pending)) return;
@@ -251,30 +290,33 @@ __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int
   float hi = INFINITY, lo = -INFINITY;
   int na = 0, nb = cnt;
   bool ready = false;
-  for (int round = 0; round < 6; ++round) {
+  const float kNaN = __int_as_float(0x7fffffff);   // compares false: slots past the lane's count
+  for (int round = 0; round < 4; ++round) {
     const bool act = pending && !ready;
     if (!__any_sync(0xffffffffu, act)) break;
     // sample q sits near rank (q + 0.5) pop / 16 of the bracket's population
     const int pop = nb - na > 0 ? nb - na : 1;
     int qc = (32 * (k - na) / pop - 1) >> 1;
-    qc = qc < 0 ? 0 : (qc > 15 ? 15 : qc);
-    const float hi2 = qc - 2 < 0 ? hi : pick<16>(s, qc - 2);
-    const float lo2 = qc + 2 > 15 ? lo : pick<16>(s, qc + 2);
-    int a2 = 0, b2 = 0;
+    qc = qc < 2 ? 2 : (qc > 13 ? 13 : qc);
+    float p[5];
+#pragma unroll
+    for (int j = 0; j < 5; ++j) p[j] = pick<16>(s, qc - 2 + j);
+    int n[5] = {0, 0, 0, 0, 0};
     for (int i = 0; i < cmax; i += 8) {
       float v[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) v[u] = c.s(i + u);
+      for (int u = 0; u < 8; ++u) v[u] = i + u < cnt ? c.s(i + u) : kNaN;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const bool in = i + u < cnt;
-        a2 += (in && v[u] > hi2) ? 1 : 0;
-        b2 += (in && v[u] >= lo2) ? 1 : 0;
-      }
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int j = 0; j < 5; ++j) n[j] += v[u] >= p[j] ? 1 : 0;
     }
     if (act) {
-      if (a2 <= k) { hi = hi2; na = a2; }
-      if (b2 >= k) { lo = lo2; nb = b2; }
+#pragma unroll
+      for (int j = 0; j < 5; ++j) {
+        if (n[j] <= k && p[j] < hi) { hi = p[j]; na = n[j]; }
+        if (n[j] >= k && p[j] > lo) { lo = p[j]; nb = n[j]; }
+      }
       ready = nb - na <= 16;
     }
     const bool resample = act && !ready;
@@ -288,7 +330,7 @@ __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int
         for (int u = 0; u < 8; ++u) v[u] = c.s(i + u);
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-          const bool in = resample && i + u < cnt && v[u] >= lo && v[u] <= hi;
+          const bool in = resample && i + u < cnt && v[u] >= lo && v[u] < hi;
           const bool take = in && seen == 0 && ns < 16;
           if (take) scr[ns] = v[u];
           ns += take ? 1 : 0;
@@ -304,7 +346,7 @@ __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int
   }
   const bool fin = pending && ready;
   if (__any_sync(0xffffffffu, fin)) {
-    // entries above hi compacted in place, boundary entries to the scratch
+    // entries at or above hi compacted in place, boundary entries to the scratch
     int w = 0, nbd = 0;
     for (int i = 0; i < cmax; i += 8) {
       float v[8];
@@ -317,7 +359,7 @@ __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         const bool in = fin && i + u < cnt;
-        const bool sure = in && v[u] > hi;
+        const bool sure = in && v[u] >= hi;
         const bool bnd = in && !sure && v[u] >= lo;
         if (sure) c.put(w, v[u], j[u]);
         if (bnd) {
@@ -425,12 +467,12 @@ __device__ __forceinline__ float select_tau(const float (&g1)[kGroups], const fl
 }
 
 // Pass 2: append the keys of 32 scores of a row (keys j0 .. j0+31) that score
-// above thr and are visible.  A column that could overflow is first cut to its
-// k best if the chunk's appends would not fit (which raises thr; CAP >= k + 32
-// leaves room for the chunk), together with every column of the warp that is
-// close to the capacity.  The appends are predicated stores at a running
-// slot pointer: no mask, no scratch, no data-dependent loop.
-template <int CAP>
+// above thr and are visible.  A column whose chunk of appends would not fit is
+// first cut to between k and CAP - 32 entries at a sampled pivot (which raises
+// thr to the pivot), together with every column of the warp that is close to
+// the capacity.  The appends are predicated stores at a running slot pointer:
+// no mask, no scratch, no data-dependent loop.
+template <int CAP, class Col>
 __device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vis, float& thr, float* scr,
                                          const Col& c, int& cnt, int k) {
   float v[32];
@@ -449,23 +491,45 @@ __device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vi
     // a cut costs the warp about the same for one row as for all 32: when one
     // row must be cut, every row close to the capacity is cut in the same call
     const int near = (k + 8 > CAP - 40) ? k + 8 : CAP - 40;
-    if (__any_sync(0xffffffffu, over)) cut_to_k(c, cnt, thr, k, scr, over || cnt > near);
+    if (__any_sync(0xffffffffu, over)) {
+      // a pivot cut (two passes) leaves between k and CAP - 32 entries; the
+      // exact cut only for lanes where no sampled pivot qualifies
+      pivot_cut(c, cnt, thr, k, k + 8, CAP - 32, over || cnt > near);
+      const bool still = over && cnt > CAP - 32;
+      if (__any_sync(0xffffffffu, still)) cut_to_k(c, cnt, thr, k, scr, still);
+    }
+    __syncwarp();
   }
   float* ps = c.bs + cnt * kLdc + c.row;
-  uint16_t* pi = c.bi + cnt * kLdc + c.row;
-  int added = 0;
+  if constexpr (Col::kWide) {
+    // score and index through one slot pointer; the count is the pointer's advance
+    float* const p0 = ps;
 #pragma unroll
-  for (int u = 0; u < 32; ++u) {
-    const bool t = v[u] > thr;
-    if (t) {
-      *ps = v[u];
-      *pi = (uint16_t)(j0 + u);
+    for (int u = 0; u < 32; ++u) {
+      const bool t = v[u] > thr;
+      if (t) {
+        ps[0] = v[u];
+        ps[Col::kIOff] = __int_as_float(j0 + u);
+      }
+      ps += t ? kLdc : 0;
     }
-    ps += t ? kLdc : 0;
-    pi += t ? kLdc : 0;
-    added += t ? 1 : 0;
+    cnt += (int)(ps - p0) / kLdc;
+  } else {
+    uint16_t* pi = c.bi + cnt * kLdc + c.row;
+    int added = 0;
+#pragma unroll
+    for (int u = 0; u < 32; ++u) {
+      const bool t = v[u] > thr;
+      if (t) {
+        *ps = v[u];
+        *pi = (uint16_t)(j0 + u);
+      }
+      ps += t ? kLdc : 0;
+      pi += t ? kLdc : 0;
+      added += t ? 1 : 0;
+    }
+    cnt += added;
   }
-  cnt += added;
 }
 
 template <int P>
@@ -695,7 +759,8 @@ __global__ void __launch_bounds__(192, 1)
     const int quarter = warp & 3;
     const int m = quarter * 32 + lane;
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
-    const Col col{bs, bi, m};
+    using Col = typename std::conditional<C::WIDE, ColWide<C::CAP * kLdc>, ColSplit>::type;
+    const Col col = make_col<Col>(bs, bi, m);
     float* scr = scr_all + m * kScr;
     uint32_t ac = 0;
     int it = 0;
@@ -763,10 +828,8 @@ __global__ void __launch_bounds__(192, 1)
         for (int c = 0; c < C::NT / 32; ++c) {
           uint32_t(&cur)[32] = (c & 1) ? rb : ra;
           uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
-          __syncwarp();
           if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::NT + (c + 1) * 32, nxt);
           append32<C::CAP>(cur, i * C::NT + c * 32, vis, thr, scr, col, cnt, a.k);
-          __syncwarp();
           if (c + 1 < C::NT / 32) tc::tmem_ld_wait(nxt);
         }
         tc::fence_before_sync();
@@ -827,7 +890,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int e = 0; e < 2; ++e) {
             const int i = e * 32 + lane;
-            v[e] = i < n ? make_key(bs[i * kLdc + row], (uint32_t)bi[i * kLdc + row]) : 0ull;
+            v[e] = i < n ? make_key(col.at(row).s(i), (uint32_t)col.at(row).j(i)) : 0ull;
           }
           warp_sort_desc<2>(v);
 #pragma unroll
@@ -840,8 +903,8 @@ __global__ void __launch_bounds__(192, 1)
           }
         } else {
           for (int i = lane; i < a.k; i += 32) {
-            a.idx[o + i] = i < n ? bi[i * kLdc + row] : -1;
-            if (a.score) a.score[o + i] = i < n ? bs[i * kLdc + row] + qn : -INFINITY;
+            a.idx[o + i] = i < n ? col.at(row).j(i) : -1;
+            if (a.score) a.score[o + i] = i < n ? col.at(row).s(i) + qn : -INFINITY;
           }
         }
       }
