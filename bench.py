@@ -322,10 +322,10 @@ def run_e2e(g, args, torch):
 # the heads, as the pairs do, so bench.py scales these to the workload; a kernel
 # changed after its capture is left out (traffic null).
 TRAFFIC_BYTES_PER_PAIR = {
-    "select": (604097536 + 233009408) / 2148007936,
-    "exact": (976500992 + 259099648) / 2148007936,
-    "moments": (335572224 + 3011584) / 2148007936,
-    "build": (73441792 + 13733632) / 2148007936,
+    "select": (571618304 + 227735808) / 2148007936,
+    "exact": (925922816 + 254329600) / 2148007936,
+    "moments": (335570944 + 2971136) / 2148007936,
+    "build": (73441792 + 13647872) / 2148007936,
 }
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only
 
