@@ -234,37 +234,44 @@ __device__ __forceinline__ void remove_worst(const Col& c, int& cnt, int cmax, f
 // Lanes with `on` cut their column to the entries scoring >= a sampled pivot p,
 // for a pivot leaving between k and tmax entries; thr becomes p (every later key
 // has a higher index, so a later key scoring exactly p loses to all kept ones).
-// Lanes for which no tried pivot qualifies keep their column unchanged.
+// One counting pass tries four adjacent pivots of 16 sorted samples around
+// rank aim and takes the one leaving the fewest entries that still number at
+// least k.  Lanes for which no tried pivot qualifies keep their column unchanged.
 template <class Col>
 __device__ __forceinline__ void pivot_cut(const Col& c, int& cnt, float& thr, int k, int aim, int tmax, bool on) {
+  const bool pending = on && cnt > k;
+  if (!__any_sync(0xffffffffu, pending)) return;
   const int cmax = warp_max(cnt);
-  float s[8];
+  float s[16];
 #pragma unroll
-  for (int u = 0; u < 8; ++u) s[u] = c.s(((2 * u + 1) * cnt) >> 4);
-  sort_desc<8>(s);
-  // sample q (0-based, descending) sits near entry rank (q + 0.5) cnt / 8
-  int q = cnt > 0 ? (16 * aim / cnt - 1) >> 1 : 0;
-  q = q < 0 ? 0 : (q > 7 ? 7 : q);
-  bool pending = on && cnt > k;
-  for (int attempt = 0; attempt < 3; ++attempt) {
-    if (!__any_sync(0xffffffffu, pending)) break;
-    const float p = pick<8>(s, q);
-    const int n = count_ge(c, cnt, cmax, p);
-    const bool ok = pending && n >= k && n <= tmax;
-    if (__any_sync(0xffffffffu, ok)) cnt = compact_ge(c, cnt, cmax, p, ok);
-    if (ok) {
-      thr = fmaxf(thr, p);
-      pending = false;
-    } else if (pending) {
-      if (n < k) {
-        if (q == 7) pending = false;
-        ++q;
-      } else {
-        if (q == 0) pending = false;
-        --q;
-      }
-    }
+  for (int u = 0; u < 16; ++u) s[u] = c.s(((2 * u + 1) * cnt) >> 5);
+  sort_desc<16>(s);
+  // sample q (0-based, descending) sits near entry rank (q + 0.5) cnt / 16
+  int q = cnt > 0 ? (32 * aim / cnt - 1) >> 1 : 0;
+  q = q < 1 ? 1 : (q > 13 ? 13 : q);
+  float p[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) p[j] = pick<16>(s, q - 1 + j);
+  const float kNaN = __int_as_float(0x7fffffff);   // compares false: slots past the lane's count
+  int n[4] = {0, 0, 0, 0};
+  for (int i = 0; i < cmax; i += 8) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = i + u < cnt ? c.s(i + u) : kNaN;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) n[j] += v[u] >= p[j] ? 1 : 0;
   }
+  // descending pivots give ascending counts: the first count reaching k
+  float pc = p[3];
+  int nc = n[3];
+#pragma unroll
+  for (int j = 2; j >= 0; --j)
+    if (n[j] >= k) { pc = p[j]; nc = n[j]; }
+  const bool ok = pending && nc >= k && nc <= tmax;
+  if (__any_sync(0xffffffffu, ok)) cnt = compact_ge(c, cnt, cmax, pc, ok);
+  if (ok) thr = fmaxf(thr, pc);
 }
 
 // Exact cut of the lanes with `on` to their k best entries (slots [0, k)); thr
