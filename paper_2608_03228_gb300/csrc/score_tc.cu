@@ -41,14 +41,17 @@ constexpr int kScr = 36;      // per-row scratch stride (words): 32 scores + pad
 
 template <int P>
 struct TcCfg {
-  static constexpr int NT = 128;                              // keys per tile (MMA N)
+  // keys per tile (MMA N): rank 128 takes 64-key tiles, halving its stage
+  // buffers so that its candidate columns get 144 slots
+  static constexpr int NT = P == 128 ? 64 : 128;
   static constexpr int NB = 4;                                // TMEM accumulator ring (lets the warps drift)
+  static constexpr int BUFC = 128;                            // TMEM columns per ring buffer (a tile or a projection)
   // ranks up to 64 store 32-bit key indices at a fixed distance from the
   // scores (one slot pointer serves both stores of an append); rank 128 needs
   // the room for its operands and keeps 16-bit indices in their own array
   static constexpr bool WIDE = P <= 64;
   static constexpr int STAGES = P >= 64 ? 2 : 4;
-  static constexpr int CAP = P == 128 ? 104 : 136;               // candidate slots per row (multiple of 8)
+  static constexpr int CAP = P == 128 ? 144 : 136;               // candidate slots per row (multiple of 8)
   static constexpr int KB = P == 128 ? 2 : 1;                 // 64-wide K blocks
   static constexpr int KW = P == 128 ? 64 : P;                // K width of one block
   static constexpr int KK = KW / 16;                          // MMA K steps per block
@@ -60,7 +63,7 @@ struct TcCfg {
   static constexpr int IDX_BYTES = WIDE ? CAP * kLdc * 4 : ((CAP * kLdc * 2 + 15) & ~15);
   static constexpr int CAND_BYTES = CAP * kLdc * 4 + IDX_BYTES;
   static constexpr int SCR_BYTES = 128 * kScr * 4;
-  static constexpr int TMEM_COLS = NB * NT;
+  static constexpr int TMEM_COLS = NB * BUFC;
   static constexpr int OFF_STAGE = A_BYTES;
   static constexpr int OFF_CAND = OFF_STAGE + STAGES * STAGE_BYTES;
   static constexpr int OFF_SCR = OFF_CAND + CAND_BYTES;
@@ -69,6 +72,7 @@ struct TcCfg {
   static_assert(STAGE_BYTES >= P * 128, "a projection chunk must fit a stage");
   static_assert(CAP % 8 == 0 && CAP >= 64 + 32, "candidate capacity: k + one chunk of appends");
   static_assert(NT % 64 == 0, "a key tile covers whole key groups");
+  static_assert(NT <= BUFC && P <= BUFC && TMEM_COLS <= 512, "a ring buffer holds a tile's or a projection's columns");
   static_assert(SMEM <= 232448, "shared memory budget");
   static_assert(OFF_STAGE % 1024 == 0 && STAGE_BYTES % 1024 == 0, "swizzled TMA tiles sit on 1024-byte boundaries");
   static_assert(OFF_SCR % 16 == 0 && OFF_BAR % 16 == 0, "16-byte scratch stores and 8-byte mbarriers stay aligned");
@@ -718,7 +722,7 @@ __global__ void __launch_bounds__(192, 1)
             tc::fence_after_sync();
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
-              tc::mma_bf16(tmem + buf * C::NT, tc::sdesc(aBase + kh * 16384 + kk * 32, 1024, 2),
+              tc::mma_bf16(tmem + buf * C::BUFC, tc::sdesc(aBase + kh * 16384 + kk * 32, 1024, 2),
                            tc::sdesc(sBase + st * C::STAGE_BYTES + kk * 32, 1024, 2), idP, acc);
               acc = 1;
             }
@@ -746,7 +750,7 @@ __global__ void __launch_bounds__(192, 1)
               for (int kk = 0; kk < C::KK; ++kk) {
                 const uint32_t ad = aBase + part * C::A_PART + kb * 16384 + kk * 32;
                 const uint32_t bd = sBase + st * C::STAGE_BYTES + kb * (C::NT * 128) + kk * 32;
-                tc::mma_bf16(tmem + buf * C::NT, tc::sdesc(ad, C::SBO, C::SW), tc::sdesc(bd, C::SBO, C::SW), idN,
+                tc::mma_bf16(tmem + buf * C::BUFC, tc::sdesc(ad, C::SBO, C::SW), tc::sdesc(bd, C::SBO, C::SW), idN,
                              accum);
                 accum = 1;
               }
@@ -780,7 +784,7 @@ __global__ void __launch_bounds__(192, 1)
         ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
-        convert_projection<P>(tl + buf * C::NT, sA, m);
+        convert_projection<P>(tl + buf * C::BUFC, sA, m);
         tc::fence_before_sync();
         tc::mbar_arrive(acce + buf);
         ++ac;
@@ -804,13 +808,13 @@ __global__ void __launch_bounds__(192, 1)
         // chunk c + 1 is read from TMEM while chunk c is folded
         uint32_t ra[32], rb[32];
         __syncwarp();
-        tc::tmem_ld32(tl + buf * C::NT, ra);
+        tc::tmem_ld32(tl + buf * C::BUFC, ra);
         tc::tmem_ld_wait(ra);
 #pragma unroll
         for (int c = 0; c < C::NT / 32; ++c) {
           uint32_t(&cur)[32] = (c & 1) ? rb : ra;
           uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
-          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::NT + (c + 1) * 32, nxt);
+          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::BUFC + (c + 1) * 32, nxt);
           fold32(cur, g1, g2, (c % 2) * 32, i * C::NT + c * 32, vis);
           if (c + 1 < C::NT / 32) tc::tmem_ld_wait(nxt);
         }
@@ -829,13 +833,13 @@ __global__ void __launch_bounds__(192, 1)
         tc::fence_after_sync();
         uint32_t ra[32], rb[32];
         __syncwarp();
-        tc::tmem_ld32(tl + buf * C::NT, ra);
+        tc::tmem_ld32(tl + buf * C::BUFC, ra);
         tc::tmem_ld_wait(ra);
 #pragma unroll
         for (int c = 0; c < C::NT / 32; ++c) {
           uint32_t(&cur)[32] = (c & 1) ? rb : ra;
           uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
-          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::NT + (c + 1) * 32, nxt);
+          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::BUFC + (c + 1) * 32, nxt);
           append32<C::CAP>(cur, i * C::NT + c * 32, vis, thr, scr, col, cnt, a.k);
           if (c + 1 < C::NT / 32) tc::tmem_ld_wait(nxt);
         }
@@ -851,7 +855,7 @@ __global__ void __launch_bounds__(192, 1)
         ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
-        convert_projection<P>(tl + buf * C::NT, sA, m);
+        convert_projection<P>(tl + buf * C::BUFC, sA, m);
         tc::fence_before_sync();
         tc::mbar_arrive(acce + buf);
         ++ac;
