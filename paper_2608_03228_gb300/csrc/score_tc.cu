@@ -41,16 +41,17 @@ constexpr int kScr = 36;      // per-row scratch stride (words): 32 scores + pad
 
 template <int P>
 struct TcCfg {
-  // keys per tile (MMA N): rank 128 takes 64-key tiles, halving its stage
-  // buffers so that its candidate columns get 144 slots
-  static constexpr int NT = P == 128 ? 64 : 128;
+  // keys per tile (MMA N): 64-key tiles keep two chunks per tile in the
+  // unrolled selection loops (fewer inlined overflow-cut copies) and halve the
+  // stage buffers, so that rank-128 columns get 144 slots
+  static constexpr int NT = 64;
   static constexpr int NB = 4;                                // TMEM accumulator ring (lets the warps drift)
   static constexpr int BUFC = 128;                            // TMEM columns per ring buffer (a tile or a projection)
   // ranks up to 64 store 32-bit key indices at a fixed distance from the
   // scores (one slot pointer serves both stores of an append); rank 128 needs
   // the room for its operands and keeps 16-bit indices in their own array
   static constexpr bool WIDE = P <= 64;
-  static constexpr int STAGES = P >= 64 ? 2 : 4;
+  static constexpr int STAGES = P == 128 ? 2 : 4;
   static constexpr int CAP = P == 128 ? 144 : 136;               // candidate slots per row (multiple of 8)
   static constexpr int KB = P == 128 ? 2 : 1;                 // 64-wide K blocks
   static constexpr int KW = P == 128 ? 64 : P;                // K width of one block
