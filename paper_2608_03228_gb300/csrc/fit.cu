@@ -114,6 +114,93 @@ __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_count
   return false;
 }
 
+// Leading dimension of the fit kernel's Jacobi matrix: 16-byte aligned columns
+// whose starts step through the banks by four.
+constexpr int kLdJ = kD + 4;
+
+// jacobi_columns for a matrix with leading dimension kLdJ, with 16-byte shared
+// accesses and packed fp32 pairs (same rotations, same stopping rule): lane
+// group q = lane / 8 of a warp holds rows 32 w + 4 sub + j (w, j < 4, sub =
+// lane % 8) of its pair's two columns, so a column moves in four 16-byte
+// accesses per lane and the group's eight lanes cover all 32 banks; the dot
+// products and the rotation run on float2 pairs (two fp32 FMAs per instruction,
+// each rounded as the scalar one).
+__device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol, int* s_counter) {
+  __shared__ float s_red[kFitThreads / 32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  float fro = 0.f;
+  for (int o = tid; o < kD * kD; o += kFitThreads) {
+    const float v = X[(o / kD) * kLdJ + (o % kD)];
+    fro = fmaf(v, v, fro);
+  }
+  fro = warp_sum(fro);
+  if (lane == 0) s_red[warp] = fro;
+  __syncthreads();
+  fro = 0.f;
+  for (int w = 0; w < kFitThreads / 32; ++w) fro += s_red[w];
+  const float tiny = fro * 1e-14f;   // squared column norm treated as zero
+  const int q = lane >> 3, sub = lane & 7;
+  for (int sweep = 0; sweep < max_sweeps; ++sweep) {
+    if (tid == 0) *s_counter = 0;
+    __syncthreads();
+    int rot = 0;
+    for (int round = 0; round < kD - 1; ++round) {
+      int pa, pb;
+      rr_pair(round, (warp & 7) + 8 * q + 32 * (warp >> 3), pa, pb);
+      float4* xa = reinterpret_cast<float4*>(X + pa * kLdJ) + sub;
+      float4* xb = reinterpret_cast<float4*>(X + pb * kLdJ) + sub;
+      float2 a[8], b[8];
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float4 va = xa[8 * w], vb = xb[8 * w];
+        a[2 * w] = make_float2(va.x, va.y);
+        a[2 * w + 1] = make_float2(va.z, va.w);
+        b[2 * w] = make_float2(vb.x, vb.y);
+        b[2 * w + 1] = make_float2(vb.z, vb.w);
+      }
+      float2 al2 = make_float2(0.f, 0.f), be2 = al2, ga2 = al2;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        al2 = __ffma2_rn(a[e], a[e], al2);
+        be2 = __ffma2_rn(b[e], b[e], be2);
+        ga2 = __ffma2_rn(a[e], b[e], ga2);
+      }
+      float al = al2.x + al2.y, be = be2.x + be2.y, ga = ga2.x + ga2.y;
+#pragma unroll
+      for (int m = 4; m > 0; m >>= 1) {  // butterflies leave the group's sums in all eight lanes
+        al += __shfl_xor_sync(0xffffffffu, al, m);
+        be += __shfl_xor_sync(0xffffffffu, be, m);
+        ga += __shfl_xor_sync(0xffffffffu, ga, m);
+      }
+      if (ga != 0.f && al > tiny && be > tiny && fabsf(ga) > tol * sqrtf(al) * sqrtf(be)) {
+        const float zeta = (be - al) / (2.f * ga);
+        const float t = fabsf(zeta) > 1e18f ? 0.5f / zeta
+                                            : copysignf(1.f, zeta) / (fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
+        const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
+        const float sn = c * t;
+        const float2 c2 = make_float2(c, c), s2 = make_float2(sn, sn), ms2 = make_float2(-sn, -sn);
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const float2 na0 = __ffma2_rn(ms2, b[2 * w], __fmul2_rn(c2, a[2 * w]));
+          const float2 na1 = __ffma2_rn(ms2, b[2 * w + 1], __fmul2_rn(c2, a[2 * w + 1]));
+          const float2 nb0 = __ffma2_rn(s2, a[2 * w], __fmul2_rn(c2, b[2 * w]));
+          const float2 nb1 = __ffma2_rn(s2, a[2 * w + 1], __fmul2_rn(c2, b[2 * w + 1]));
+          xa[8 * w] = make_float4(na0.x, na0.y, na1.x, na1.y);
+          xb[8 * w] = make_float4(nb0.x, nb0.y, nb1.x, nb1.y);
+        }
+        if (sub == 0) ++rot;
+      }
+      __syncthreads();
+    }
+    if (sub == 0 && rot) atomicAdd(s_counter, rot);   // one counter per pair group
+    __syncthreads();
+    const int total = *s_counter;
+    __syncthreads();
+    if (total == 0) return true;
+  }
+  return false;
+}
+
 // Householder QR of the matrix in X (column-major, leading dimension kLdS), in
 // place: on return R occupies the upper triangle (diagonal included); below it,
 // the reflector vectors are left behind.  Needs kFitThreads threads.
@@ -171,12 +258,12 @@ __device__ void householder_r(float* X) {
   }
 }
 
-// column norms of X into out[kD] (warp per column)
-__device__ void column_norms(const float* X, float* out) {
+// column norms of X (leading dimension ld) into out[kD] (warp per column)
+__device__ void column_norms(const float* X, float* out, int ld = kLdS) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int c = warp; c < kD; c += kFitThreads / 32) {
     float v = 0.f;
-    for (int i = lane; i < kD; i += 32) v = fmaf(X[c * kLdS + i], X[c * kLdS + i], v);
+    for (int i = lane; i < kD; i += 32) v = fmaf(X[c * ld + i], X[c * ld + i], v);
     v = warp_sum(v);
     if (lane == 0) out[c] = sqrtf(v);
   }
@@ -298,7 +385,7 @@ __global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, flo
   }
 }
 
-// Shared memory holds only the Jacobi matrix (66 KB), so two CTAs share an SM;
+// Shared memory holds only the Jacobi matrix (68 KB), so two CTAs share an SM;
 // C'^T is kept in a global scratch slice (L2-resident) for the steps after the SVD.
 __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, const float* Fm, const float* Gm,
                                                              const float* mu, int Hq, int Hk, int r, int max_sweeps,
@@ -354,18 +441,25 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
   for (int o = tid; o < kD * kD; o += kFitThreads) X[(o % kD) * kLdS + (o / kD)] = Ct[o];   // X = C'
   __syncthreads();
   householder_r(X);
-  for (int o = tid; o < kD * kD; o += kFitThreads) {   // X = R1^T (lower triangle)
-    const int i = o / kD, jj = o % kD;
-    if (i > jj) {
-      X[jj * kLdS + i] = X[i * kLdS + jj];
-      X[i * kLdS + jj] = 0.f;
+  {  // X = R1^T (lower triangle), re-laid out with leading dimension kLdJ
+    float v[kD * kD / kFitThreads];
+#pragma unroll
+    for (int t = 0; t < kD * kD / kFitThreads; ++t) {
+      const int o = tid + t * kFitThreads, i = o / kD, jj = o % kD;
+      v[t] = i >= jj ? X[i * kLdS + jj] : 0.f;   // R1^T (i, jj) = R1 (jj, i)
+    }
+    __syncthreads();
+#pragma unroll
+    for (int t = 0; t < kD * kD / kFitThreads; ++t) {
+      const int o = tid + t * kFitThreads, i = o / kD, jj = o % kD;
+      X[jj * kLdJ + i] = v[t];
     }
   }
   __syncthreads();
 
-  const bool conv = jacobi_columns(X, max_sweeps, tol, &counter);
+  const bool conv = jacobi_columns_v4(X, max_sweeps, tol, &counter);
   if (!conv && tid == 0) status[h] |= kStNotConverged;
-  column_norms(X, sig);
+  column_norms(X, sig, kLdJ);
   __syncthreads();
   if (tid < kD) {  // rank = position in descending order, ties by index
     const float s = sig[tid];
@@ -386,7 +480,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
     float z = 0.f, q = 0.f;
     const float* ct = Ct + a * kD;   // column a of C'^T = row a of C'
     for (int b = 0; b < kD; ++b) {
-      const float x = X[i * kLdS + b];
+      const float x = X[i * kLdJ + b];
       z = fmaf(__ldg(ct + b), x, z);
       q = fmaf(__ldg(Gk + a * kD + b), x, q);
     }
@@ -440,7 +534,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
 
 constexpr float kTol = 1e-6f;
 constexpr size_t kSmem = 2 * sizeof(float) * kD * kLdS;     // factor kernel: S and its inverse factor
-constexpr size_t kFitSmem = sizeof(float) * kD * kLdS;      // fit kernel: the Jacobi matrix
+constexpr size_t kFitSmem = sizeof(float) * kD * kLdJ;      // fit kernel: the Jacobi matrix
 }  // namespace
 
 cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps, float* F, float* Gm,
