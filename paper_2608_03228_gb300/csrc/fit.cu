@@ -6,7 +6,9 @@
 //   floor * lambda_max(S) proves that the eigenvalue floor of App. A drops
 //   nothing.  Otherwise the floor is applied exactly: eigenpairs of S from a
 //   one-sided Jacobi run on S (S V = V Lambda for a PSD matrix), F = V_+
-//   Lambda_+^{1/2}, G = V_+ Lambda_+^{-1/2} over the kept eigenvalues.
+//   Lambda_+^{1/2}, G = V_+ Lambda_+^{-1/2} over the kept eigenvalues.  F is
+//   stored row-major, G column-major (the fit kernel reads G's columns with
+//   consecutive rows in consecutive lanes).
 //   Any factor with F F^T = S yields the same optimum, because
 //   ||F_q^T X F_k||_F^2 = tr(X^T Sq X Sk) for every X.
 //
@@ -356,7 +358,10 @@ __global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, flo
     for (int o = tid; o < kD * kD; o += kFitThreads) {
       const int i = o / kD, c = o % kD;
       F[o] = c <= i ? Sb[i * kLdS + c] : 0.f;
-      G[o] = i <= c ? Xb[c * kLdS + i] : 0.f;   // G = Linv^T
+    }
+    for (int o = tid; o < kD * kD; o += kFitThreads) {   // G = Linv^T, stored transposed
+      const int c = o / kD, i = o % kD;
+      G[o] = i <= c ? Xb[c * kLdS + i] : 0.f;
     }
     return;
   }
@@ -379,9 +384,13 @@ __global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, flo
     const int i = o / kD, c = o % kD;
     const float l = lam[c];
     const bool keep = l > 0.f && l >= floor_rel * lmax;
-    const float w = Xb[c * kLdS + i];
-    F[o] = keep ? w / sqrtf(l) : 0.f;          // v sqrt(l),  v = w / l
-    G[o] = keep ? w / (l * sqrtf(l)) : 0.f;    // v / sqrt(l)
+    F[o] = keep ? Xb[c * kLdS + i] / sqrtf(l) : 0.f;          // v sqrt(l),  v = w / l
+  }
+  for (int o = tid; o < kD * kD; o += kFitThreads) {   // G stored transposed
+    const int c = o / kD, i = o % kD;
+    const float l = lam[c];
+    const bool keep = l > 0.f && l >= floor_rel * lmax;
+    G[o] = keep ? Xb[c * kLdS + i] / (l * sqrtf(l)) : 0.f;    // v / sqrt(l)
   }
 }
 
@@ -404,7 +413,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
   const float* Gq = Gm + (int64_t)h * kD * kD;
   const float* Fk = Fm + (int64_t)(Hq + g) * kD * kD;
   const float* Gk = Gm + (int64_t)(Hq + g) * kD * kD;
-  float* Ct = Cws + (int64_t)h * kD * kD;   // C'^T, column-major: (row, col) at [col * d + row]
+  float* Ct = Cws + (int64_t)h * kD * kD;   // C', column-major: (row, col) at [col * d + row]
   float* Lh = L + (int64_t)h * kD * r;
   float* Rh = R + (int64_t)h * kD * r;
 
@@ -422,7 +431,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
     for (int u = 0; u < 32; ++u) X[cc * kLdS + r0 + u] = acc[u];
   }
   __syncthreads();
-  {  // C'^T = X^T Fq -> global scratch
+  {  // C'^T = X^T Fq, stored as C' column-major in the global scratch
     float acc[32];
 #pragma unroll
     for (int u = 0; u < 32; ++u) acc[u] = 0.f;
@@ -432,13 +441,13 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
       for (int u = 0; u < 32; ++u) acc[u] = fmaf(X[(r0 + u) * kLdS + p], f, acc[u]);
     }
 #pragma unroll
-    for (int u = 0; u < 32; ++u) Ct[cc * kD + r0 + u] = acc[u];
+    for (int u = 0; u < 32; ++u) Ct[(r0 + u) * kD + cc] = acc[u];   // C'(cc, r0 + u)
   }
   __syncthreads();
   // Preconditioning: C' = Q1 R1 (Householder), then the Jacobi runs on R1^T, whose
   // left singular vectors are those of C'^T = R1^T Q1^T, i.e. the right singular
   // vectors of C' (the triangular factor converges in far fewer sweeps).
-  for (int o = tid; o < kD * kD; o += kFitThreads) X[(o % kD) * kLdS + (o / kD)] = Ct[o];   // X = C'
+  for (int o = tid; o < kD * kD; o += kFitThreads) X[(o / kD) * kLdS + (o % kD)] = Ct[o];   // X = C'
   __syncthreads();
   householder_r(X);
   {  // X = R1^T (lower triangle), re-laid out with leading dimension kLdJ
@@ -478,11 +487,10 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
     const float s = sig[i];
     const bool live = s > 0.f && s > smax * 1e-20f;
     float z = 0.f, q = 0.f;
-    const float* ct = Ct + a * kD;   // column a of C'^T = row a of C'
-    for (int b = 0; b < kD; ++b) {
+    for (int b = 0; b < kD; ++b) {   // C'(a, b) and Gk(a, b): consecutive a in consecutive lanes
       const float x = X[i * kLdJ + b];
-      z = fmaf(__ldg(ct + b), x, z);
-      q = fmaf(__ldg(Gk + a * kD + b), x, q);
+      z = fmaf(__ldg(Ct + b * kD + a), x, z);
+      q = fmaf(__ldg(Gk + b * kD + a), x, q);
     }
     Lh[a * r + c] = live ? z / (s * s) : 0.f;    // C' x_i / s^2 = u_i (x_i = s v_i)
     Rh[a * r + c] = live ? q / sqrtf(s) : 0.f;   // Gk v_i sqrt(s) = Gk x_i / sqrt(s)
@@ -514,7 +522,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
   for (int c = tid / kD; c < r; c += kFitThreads / kD) {
     const float s = sig[perm[c]];
     float acc = 0.f;
-    for (int e = 0; e < kD; ++e) acc = fmaf(__ldg(Gq + a * kD + e), X[c * kLdS + e], acc);
+    for (int e = 0; e < kD; ++e) acc = fmaf(__ldg(Gq + e * kD + a), X[c * kLdS + e], acc);
     Lh[a * r + c] = sgn[c] * acc * sqrtf(fmaxf(s, 0.f));   // Gq u_i sqrt(s)
   }
   if (tid < kD && sigma) sigma[(int64_t)h * kD + tid] = sig[perm[tid]];

@@ -89,7 +89,8 @@ size_t score_generic_smem(int P, int kp, int nq);
 cudaError_t launch_gram(const void* q_calib, const void* k_calib, int64_t n, int Hq, int Hk,
                         int center, int dtype, float* S, float* mu, int* err, cudaStream_t s);
 
-// factor F (F F^T = S, floor applied) and G = pseudo-inverse transpose of F, per matrix
+// factor F (F F^T = S, floor applied, row-major) and G = pseudo-inverse transpose of F
+// (stored transposed, i.e. column-major), per matrix
 cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps,
                           float* F, float* Gm, int* status, cudaStream_t s);
 
