@@ -146,9 +146,12 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol, int* s_co
     if (tid == 0) *s_counter = 0;
     __syncthreads();
     int rot = 0;
-    for (int round = 0; round < kD - 1; ++round) {
-      int pa, pb;
-      rr_pair(round, (warp & 7) + 8 * q + 32 * (warp >> 3), pa, pb);
+    // round-robin (circle) schedule: the players at the pair's two positions in
+    // round 0, then every player but 0 moves on by one (mod kD - 1) per round
+    int pa, pb;
+    rr_pair(0, (warp & 7) + 8 * q + 32 * (warp >> 3), pa, pb);
+    for (int round = 0; round < kD - 1; ++round, pa = pa == 0 ? 0 : (pa == kD - 1 ? 1 : pa + 1),
+             pb = pb == kD - 1 ? 1 : pb + 1) {
       float4* xa = reinterpret_cast<float4*>(X + pa * kLdJ) + sub;
       float4* xb = reinterpret_cast<float4*>(X + pb * kLdJ) + sub;
       float2 a[8], b[8];
@@ -174,10 +177,12 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol, int* s_co
         be += __shfl_xor_sync(0xffffffffu, be, m);
         ga += __shfl_xor_sync(0xffffffffu, ga, m);
       }
-      if (ga != 0.f && al > tiny && be > tiny && fabsf(ga) > tol * sqrtf(al) * sqrtf(be)) {
-        const float zeta = (be - al) / (2.f * ga);
-        const float t = fabsf(zeta) > 1e18f ? 0.5f / zeta
-                                            : copysignf(1.f, zeta) / (fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
+      if (ga != 0.f && al > tiny && be > tiny && fabsf(ga) * rsqrtf(al) * rsqrtf(be) > tol) {
+        // the angle only needs to be close (fast divisions); c = 1 / sqrt(1 + t^2)
+        // is rounded correctly, so that the rotation stays orthogonal
+        const float zeta = __fdividef(be - al, 2.f * ga);
+        const float t = fabsf(zeta) > 1e18f ? __fdividef(0.5f, zeta)
+                                            : __fdividef(copysignf(1.f, zeta), fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
         const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
         const float sn = c * t;
         const float2 c2 = make_float2(c, c), s2 = make_float2(sn, sn), ms2 = make_float2(-sn, -sn);
