@@ -210,29 +210,41 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol, int* s_co
 
 // Householder QR of the matrix in X (column-major, leading dimension kLdS), in
 // place: on return R occupies the upper triangle (diagonal included); below it,
-// the reflector vectors are left behind.  Needs kFitThreads threads.
+// the reflector vectors are left behind.  Needs kFitThreads threads.  One
+// barrier per column: warp 0 updates column j + 1 first and then derives the
+// next reflector from it while the other warps finish step j (parameters
+// double-buffered by step parity); the new diagonal is written without a
+// barrier, as the trailing update never reads it.
+
+// Reflector parameters of column x below row j - 1 (warp-wide; lane 0 writes):
+// alpha (the new diagonal), v_j, and 2 / |v|^2 (0 when there is nothing to reflect).
+__device__ __forceinline__ void householder_par(const float* x, int j, float* par, int lane) {
+  float sq = 0.f;
+  for (int i = j + 1 + lane; i < kD; i += 32) sq = fmaf(x[i], x[i], sq);
+  sq = warp_sum(sq);
+  if (lane == 0) {
+    const float x0 = x[j];
+    const float nx = sqrtf(fmaf(x0, x0, sq));
+    const float alpha = x0 >= 0.f ? -nx : nx;   // v_j = x0 - alpha adds magnitudes: no cancellation
+    const float v0 = x0 - alpha;
+    const float vn2 = fmaf(v0, v0, sq);
+    par[0] = alpha;
+    par[1] = v0;
+    par[2] = vn2 > 0.f ? 2.f / vn2 : 0.f;
+  }
+}
+
 __device__ void householder_r(float* X) {
-  __shared__ float s_par[3];   // alpha (the new diagonal), v_j, |v|^2
+  __shared__ float s_par[2][3];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (warp == 0) householder_par(X, 0, s_par[0], lane);
+  __syncthreads();
   for (int j = 0; j < kD - 1; ++j) {
+    const float* par = s_par[j & 1];
+    float* nxt = s_par[(j + 1) & 1];
+    const float v0 = par[1], inv = par[2];
     float* xj = X + j * kLdS;
-    if (warp == 0) {
-      float sq = 0.f;
-      for (int i = j + 1 + lane; i < kD; i += 32) sq = fmaf(xj[i], xj[i], sq);
-      sq = warp_sum(sq);
-      if (lane == 0) {
-        const float x0 = xj[j];
-        const float nx = sqrtf(fmaf(x0, x0, sq));
-        const float alpha = x0 >= 0.f ? -nx : nx;   // v_j = x0 - alpha adds magnitudes: no cancellation
-        const float v0 = x0 - alpha;
-        s_par[0] = alpha;
-        s_par[1] = v0;
-        s_par[2] = fmaf(v0, v0, sq);
-      }
-    }
-    __syncthreads();
-    const float v0 = s_par[1], vn2 = s_par[2];
-    if (vn2 > 0.f) {
+    if (inv > 0.f) {
       // trailing columns: c -= (2 v.c / |v|^2) v, two columns per warp at a time
       for (int c = j + 1 + warp; c < kD; c += 2 * (kFitThreads / 32)) {
         const int c2 = c + kFitThreads / 32;
@@ -248,7 +260,7 @@ __device__ void householder_r(float* X) {
           d1 += __shfl_xor_sync(0xffffffffu, d1, m);
           d2 += __shfl_xor_sync(0xffffffffu, d2, m);
         }
-        const float f1 = 2.f * d1 / vn2, f2 = 2.f * d2 / vn2;
+        const float f1 = d1 * inv, f2 = d2 * inv;
         if (lane == 0) {
           xc[j] = fmaf(-f1, v0, xc[j]);
           if (c2 < kD) xd[j] = fmaf(-f2, v0, xd[j]);
@@ -257,10 +269,15 @@ __device__ void householder_r(float* X) {
           xc[i] = fmaf(-f1, xj[i], xc[i]);
           if (c2 < kD) xd[i] = fmaf(-f2, xj[i], xd[i]);
         }
+        if (c == j + 1) {   // warp 0: column j + 1 is final for step j + 1
+          __syncwarp();
+          householder_par(xc, j + 1, nxt, lane);
+        }
       }
+      if (tid == 0) xj[j] = par[0];
+    } else if (warp == 0) {
+      householder_par(X + (j + 1) * kLdS, j + 1, nxt, lane);   // nothing to reflect: column j + 1 unchanged
     }
-    __syncthreads();
-    if (tid == 0 && vn2 > 0.f) xj[j] = s_par[0];
     __syncthreads();
   }
 }
