@@ -23,6 +23,34 @@ thread_local bool t_pageable_only = false;
 // its bounce buffers, which can stall behind large copies the caller runs on
 // other streams; these go through a ring of pinned slots per device instead.  A
 // slot is reused only after the event recorded behind its last copy completed.
+// Byte copy on the SMs (16-byte words when both ends allow), for the staging
+// ring: one side is mapped pinned host memory read or written through its
+// device alias, so no copy engine is involved.
+__global__ void staged_copy_kernel(uint8_t* dst, const uint8_t* src, size_t n) {
+  const size_t stride = (size_t)gridDim.x * blockDim.x;
+  size_t i0 = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (((reinterpret_cast<uintptr_t>(dst) | reinterpret_cast<uintptr_t>(src)) & 15u) == 0) {
+    const size_t nv = n / 16;
+    for (size_t i = i0; i < nv; i += stride)
+      reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(src)[i];
+    for (size_t i = nv * 16 + i0; i < n; i += stride) dst[i] = src[i];
+  } else {
+    for (size_t i = i0; i < n; i += stride) dst[i] = src[i];
+  }
+}
+
+cudaError_t staged_copy(void* dst, const void* src, size_t n, cudaStream_t s) {
+  const size_t words = (n + 15) / 16;
+  const int blocks = (int)std::min<size_t>((words + 255) / 256, 64);
+  note_launch();
+  staged_copy_kernel<<<blocks, 256, 0, s>>>(static_cast<uint8_t*>(dst), static_cast<const uint8_t*>(src), n);
+  return cudaGetLastError();
+}
+
+// The library's own small transfers (plans up, status words down) go through a
+// ring of mapped pinned slots and are carried by staged_copy_kernel: a copy
+// engine would queue them behind the caller's large transfers on other
+// streams (an input copy of the next batch), stalling this stream for as long.
 class Staging {
  public:
   // host -> device: n bytes of src to dst, ordered on s
@@ -34,7 +62,7 @@ class Staging {
     cudaError_t e = take(n, &sl);
     if (e != cudaSuccess) return e;
     std::memcpy(sl->p, src, n);
-    if ((e = cudaMemcpyAsync(dst, sl->p, n, cudaMemcpyHostToDevice, s)) != cudaSuccess) return e;
+    if ((e = staged_copy(dst, sl->d, n, s)) != cudaSuccess) return e;
     return cudaEventRecord(sl->ev, s);
   }
   // device -> host: n bytes of src to dst; waits for the stream
@@ -47,7 +75,7 @@ class Staging {
     Slot* sl = nullptr;
     cudaError_t e = take(n, &sl);
     if (e != cudaSuccess) return e;
-    if ((e = cudaMemcpyAsync(sl->p, src, n, cudaMemcpyDeviceToHost, s)) != cudaSuccess) return e;
+    if ((e = staged_copy(sl->d, src, n, s)) != cudaSuccess) return e;
     if ((e = cudaEventRecord(sl->ev, s)) != cudaSuccess) return e;
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return e;
     std::memcpy(dst, sl->p, n);
@@ -56,7 +84,8 @@ class Staging {
 
  private:
   struct Slot {
-    void* p = nullptr;
+    void* p = nullptr;   // host address
+    void* d = nullptr;   // its device alias
     size_t cap = 0;
     cudaEvent_t ev = nullptr;
   };
@@ -78,7 +107,12 @@ class Staging {
       sl.p = nullptr;
       sl.cap = 0;
       const size_t cap = std::max<size_t>(n, 64 << 10);
-      if ((e = cudaHostAlloc(&sl.p, cap, cudaHostAllocDefault)) != cudaSuccess) return e;
+      if ((e = cudaHostAlloc(&sl.p, cap, cudaHostAllocMapped | cudaHostAllocPortable)) != cudaSuccess) return e;
+      if ((e = cudaHostGetDevicePointer(&sl.d, sl.p, 0)) != cudaSuccess) {
+        cudaFreeHost(sl.p);
+        sl.p = nullptr;
+        return e;
+      }
       sl.cap = cap;
     }
     *out = &sl;
