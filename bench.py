@@ -268,12 +268,15 @@ def input_bytes(g) -> int:
 def run_e2e(g, args, torch):
     """The step through the public API with the inputs in pinned host memory: every
     step copies its inputs host-to-device and reads its recall vector back, inside
-    the timed region.  Inputs are double-buffered on the device and copied on a
-    second stream, so step i+1's copies overlap step i's kernels (as a pipeline
-    over successive batches would run)."""
+    the timed region.  Inputs rotate through DEPTH device buffer sets and are copied
+    on a second stream up to DEPTH - 1 steps ahead (as a pipeline over successive
+    batches would stage them): host-to-device copies on the GB300 machine slow to a
+    fraction of their rate for tens of milliseconds about twice a second (seen with
+    no library call running), and one step of lead would expose each episode."""
+    DEPTH = 4
     keys = ("q_calib", "k_calib", "A", "Q", "K")
     host = {k: g.data[k].cpu().pin_memory() for k in keys}
-    bufs = [{k: torch.empty_like(g.data[k]) for k in keys} for _ in range(2)]
+    bufs = [{k: torch.empty_like(g.data[k]) for k in keys} for _ in range(DEPTH)]
     out_host = torch.empty((g.w.num_q_heads,), dtype=torch.float32).pin_memory()
     steps = max(2, min(args.steps, 10))
     comp = torch.cuda.current_stream()
@@ -294,7 +297,7 @@ def run_e2e(g, args, torch):
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
         for k in keys:
-            bufs[rep % 2][k].copy_(host[k], non_blocking=True)
+            bufs[rep % DEPTH][k].copy_(host[k], non_blocking=True)
         e1.record()
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1)
@@ -309,28 +312,31 @@ def run_e2e(g, args, torch):
     def issue_copy(i):
         with torch.cuda.stream(copy):
             copy.wait_event(t0)
-            if i >= 2:
-                copy.wait_event(used[i - 2])      # the kernels of step i-2 read this buffer
+            if i >= DEPTH:
+                copy.wait_event(used[i - DEPTH])      # the kernels of step i-DEPTH read this buffer
             for k in keys:
-                bufs[i % 2][k].copy_(host[k], non_blocking=True)
+                bufs[i % DEPTH][k].copy_(host[k], non_blocking=True)
             copied[i].record(copy)
 
     t0.record(comp)
     issue_copy(0)
+    issued = 1
     for i in range(steps):
-        if i + 1 < steps:
-            issue_copy(i + 1)
         comp.wait_event(copied[i])
-        g.step(inputs=bufs[i % 2])
+        g.step(inputs=bufs[i % DEPTH])
         used[i].record(comp)
         out_host.copy_(g.recall, non_blocking=True)
+        while issued < min(steps, i + DEPTH):   # after step i's calls, so that step i never waits on them
+            issue_copy(issued)
+            issued += 1
     t1.record(comp)
     torch.cuda.synchronize()
     ms = t0.elapsed_time(t1) / steps
     h2d = sum(int(host[k].numel() * host[k].element_size()) for k in keys)
     return {"value": visible_pairs(g.w) / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "steps": steps,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": int(out_host.numel() * 4),
-            "overlap": "step i+1's host-to-device copies run on a second stream during step i"}
+            "overlap": f"inputs copied on a second stream up to {DEPTH - 1} steps ahead of the step that reads "
+                       f"them, into {DEPTH} device buffer sets"}
 
 
 # DRAM bytes (read + write) per visible pair, from one ncu capture of each kernel
