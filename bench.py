@@ -345,10 +345,11 @@ def run_e2e(g, args, torch):
 # the heads, as the pairs do, so bench.py scales these to the workload; a kernel
 # changed after its capture is left out (traffic null).
 TRAFFIC_BYTES_PER_PAIR = {
-    "select": (571618304 + 227735808) / 2148007936,
-    "exact": (925922816 + 254329600) / 2148007936,
-    "moments": (335570944 + 2971136) / 2148007936,
-    "build": (73441792 + 13647872) / 2148007936,
+    "select": (554087936 + 225715712) / 2148007936,
+    "exact": (868380928 + 238369792) / 2148007936,
+    "moments": (335566848 + 3014400) / 2148007936,
+    "build": (73444608 + 13551872) / 2148007936,
+    "fit": (59018496 + 30720) / 2148007936,
 }
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only
 
