@@ -310,12 +310,16 @@ __device__ void column_norms(const float* X, float* out, int ld = kLdS) {
   }
 }
 
-__global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, float floor_rel, int max_sweeps,
-                                                             float tol, float* Fout, float* Gout, int* status) {
+// One d x d buffer in shared memory (two CTAs per SM): the Cholesky factor L
+// in its lower triangle, L^{-1} transposed in its strict upper triangle with
+// L^{-1}'s diagonal in dinv; or, on the fallback path, the Jacobi matrix.
+__global__ void __launch_bounds__(kFitThreads, 2) factor_kernel(const float* S, float floor_rel, int max_sweeps,
+                                                                float tol, float* Fout, float* Gout, int* status) {
   extern __shared__ __align__(16) float sm[];
-  float* Sb = sm;               // row-major, lower triangle becomes the Cholesky factor
-  float* Xb = sm + kD * kLdS;   // inverse factor, or the Jacobi matrix
+  float* Sb = sm;   // row-major
+  float* Xb = sm;   // the Jacobi matrix of the fallback path
   __shared__ float lam[kD];
+  __shared__ float dinv[kD];
   __shared__ float red[32];
   __shared__ int flag, counter;
   const int m = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -364,22 +368,31 @@ __global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, flo
   bool chol_ok = (flag == 0);
   if (chol_ok) {
     // Linv = F^{-1} by right-looking substitution on the identity: row i is
-    // divided by F_ii, then subtracted (times F_ri) from every row below it
-    for (int o = tid; o < kD * kD; o += kFitThreads) Xb[(o / kD) * kLdS + (o % kD)] = (o / kD == o % kD) ? 1.f : 0.f;
+    // divided by F_ii, then subtracted (times F_ri) from every row below it.
+    // Linv(r, c) for r > c lives at Sb[c][r] (the strict upper triangle, whose
+    // copy of S is no longer needed), Linv(i, i) in dinv[i].
+    for (int o = tid; o < kD * kD; o += kFitThreads) {
+      const int i = o / kD, c = o % kD;
+      if (c > i) Sb[i * kLdS + c] = 0.f;
+    }
+    if (tid < kD) dinv[tid] = 1.f;
     __syncthreads();
     for (int i = 0; i < kD; ++i) {
       const float inv = 1.f / Sb[i * kLdS + i];
-      if (tid <= i) Xb[i * kLdS + tid] *= inv;   // columns > i of row i are zero
+      if (tid < i) Sb[tid * kLdS + i] *= inv;   // Linv(i, c) for c < i; columns > i of row i are zero
+      if (tid == i) dinv[i] *= inv;
       __syncthreads();
       for (int r = i + 1 + warp; r < kD; r += kFitThreads / 32) {
         const float lri = Sb[r * kLdS + i];
-        for (int c = lane; c <= i; c += 32) Xb[r * kLdS + c] = fmaf(-lri, Xb[i * kLdS + c], Xb[r * kLdS + c]);
+        for (int c = lane; c < i; c += 32) Sb[c * kLdS + r] = fmaf(-lri, Sb[c * kLdS + i], Sb[c * kLdS + r]);
+        if (lane == 0) Sb[i * kLdS + r] = fmaf(-lri, dinv[i], Sb[i * kLdS + r]);
       }
       __syncthreads();
     }
     float ss = 0.f;
     for (int o = tid; o < kD * kD; o += kFitThreads) {
-      const float v = Xb[(o / kD) * kLdS + (o % kD)];
+      const int i = o / kD, c = o % kD;
+      const float v = c > i ? Sb[i * kLdS + c] : (c == i ? dinv[i] : 0.f);
       ss = fmaf(v, v, ss);
     }
     ss = warp_sum(ss);
@@ -398,9 +411,9 @@ __global__ void __launch_bounds__(kFitThreads) factor_kernel(const float* S, flo
       const int i = o / kD, c = o % kD;
       F[o] = c <= i ? Sb[i * kLdS + c] : 0.f;
     }
-    for (int o = tid; o < kD * kD; o += kFitThreads) {   // G = Linv^T, stored transposed
+    for (int o = tid; o < kD * kD; o += kFitThreads) {   // G = Linv^T, stored transposed: G[c][i] = Linv(c, i)
       const int c = o / kD, i = o % kD;
-      G[o] = i <= c ? Xb[c * kLdS + i] : 0.f;
+      G[o] = i < c ? Sb[i * kLdS + c] : (i == c ? dinv[i] : 0.f);
     }
     return;
   }
@@ -580,7 +593,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
 }
 
 constexpr float kTol = 1e-6f;
-constexpr size_t kSmem = 2 * sizeof(float) * kD * kLdS;     // factor kernel: S and its inverse factor
+constexpr size_t kSmem = sizeof(float) * kD * kLdS;         // factor kernel: L and L^{-1} share one buffer
 constexpr size_t kFitSmem = sizeof(float) * kD * kLdJ;      // fit kernel: the Jacobi matrix
 }  // namespace
 
