@@ -195,7 +195,7 @@ struct Plan {
   std::vector<int32_t> vis;
   int64_t cand_slots = 0;
   // workspace offsets (bytes)
-  size_t off_items = 0, off_merges = 0, off_vis = 0, off_cand = 0, bytes = 0, staged = 0;
+  size_t off_items = 0, off_merges = 0, off_vis = 0, off_err = 0, off_cand = 0, bytes = 0, staged = 0;
 };
 
 // Groups of up to kGroupQ consecutive queries of one sequence; a group's visible
@@ -240,7 +240,8 @@ Plan make_plan(const saki_layout* L, int Hq, int kp) {
   p.off_items = 0;
   p.off_merges = align_up(p.items.size() * sizeof(ScoreItem));
   p.off_vis = p.off_merges + align_up(p.merges.size() * sizeof(MergeItem));
-  p.staged = p.off_vis + p.vis.size() * sizeof(int32_t);
+  p.off_err = p.off_vis + align_up(p.vis.size() * sizeof(int32_t));   // zeroed by the upload
+  p.staged = p.off_err + sizeof(int);
   p.off_cand = align_up(p.staged);
   p.bytes = p.off_cand + align_up((size_t)p.cand_slots * Hq * kp * sizeof(uint64_t));
   return p;
@@ -560,6 +561,7 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
   a.idx = idx; a.score = score;
   a.cand = reinterpret_cast<uint64_t*>(ws + p.off_cand);
   a.cand_per_head = p.cand_slots;
+  a.err = reinterpret_cast<int*>(ws + p.off_err);
   a.T = T; a.N = N;
   a.Hq = cfg->num_q_heads; a.G = cfg->num_q_heads / cfg->num_kv_heads; a.P = cfg->rank; a.k = cfg->topk;
   a.exact = 0;
@@ -610,6 +612,7 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
     a.idx = ie; a.score = nullptr;
     a.cand = reinterpret_cast<uint64_t*>(ws + p.off_cand);
     a.cand_per_head = p.cand_slots;
+    a.err = reinterpret_cast<int*>(ws + p.off_err);
     a.T = T; a.N = N;
     a.Hq = cfg->num_q_heads; a.G = cfg->num_q_heads / cfg->num_kv_heads; a.P = kD; a.k = cfg->topk;
     a.exact = 1;

@@ -74,6 +74,7 @@ struct ScoreArgs {
   float* score;         // [Hq][T][k] or null
   uint64_t* cand;       // candidate lists, kp keys per slot, per head: cand_per_head slots
   int64_t cand_per_head;
+  int* err;             // zeroed workspace word; the tensor-core variant sets kStTimeout if a bounded wait gave up
   int64_t T, N;
   int32_t Hq, G, P, k, exact, n_items, n_merges;
 };

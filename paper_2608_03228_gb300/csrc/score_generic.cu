@@ -9,8 +9,13 @@
 // query, a shared-memory buffer of candidates above its running k-th best key
 // and re-selects (warp bitonic sort) when the buffer fills; warps are merged at
 // the end, and splits of a long sequence by a second small kernel.
+//
+// score_decode_tc_kernel runs the same work items with the scores from the
+// tensor core (bf16 keys or codes): see its comment.
 #include "common.cuh"
 #include "kernels.h"
+#include "tc.cuh"
+#include "tmap.cuh"
 
 namespace saki {
 
@@ -275,6 +280,327 @@ __global__ void __launch_bounds__(128) merge_kernel(const ScoreArgs a) {
   }
 }
 
+// ---------------------------------------------------------------- tensor-core variant
+// The work items of score_generic_kernel (up to kGroupQ queries of one sequence
+// against one split of its keys) with the scores on the tensor core: tiles of
+// 128 keys (codes, or keys for the exact scores) are the A operand (M = 128,
+// TMA), u = W^T q of the group's queries split into bf16 hi + lo the B operand
+// (N = 16, rows past the group zero), D[key][query] in a ring of TMEM
+// accumulators.  Each epilogue thread owns one key of a tile (its TMEM lane) and
+// reads that key's scores for all queries in one load; the selection is
+// score_generic_kernel's.  Roles: warp 0 TMA producer, warp 1 TMEM owner and MMA
+// issuer, warps 2-5 projection and selection.  Every mbarrier wait is bounded;
+// a CTA that gives up sets kStTimeout in the error word.
+template <int P>
+struct DcCfg {
+  static constexpr int KW = P == 128 ? 64 : P;   // K width of one swizzled block
+  static constexpr int KB = P / KW;
+  static constexpr int KK = KW / 16;
+  static constexpr uint32_t SW = KW == 64 ? 2u : (KW == 32 ? 4u : 6u);
+  static constexpr uint32_t SBO = 8 * KW * 2;
+  static constexpr int NT = 128;                 // keys per tile (MMA M)
+  static constexpr int NQ = 16;                  // queries per MMA (N), the group zero-padded
+  static constexpr int NB = 8;                   // TMEM ring of NQ-column accumulators
+  static constexpr int STAGES = P == 128 ? 3 : 4;
+  static constexpr int STAGE_BYTES = NT * P * 2;
+  static constexpr int U_PART = (NQ * P * 2 + 1023) & ~1023;   // u_hi or u_lo
+  static constexpr int OFF_U = STAGES * STAGE_BYTES;
+  static constexpr int OFF_BUF = OFF_U + 2 * U_PART;
+  static int smem(int kp) { return OFF_BUF + 4 * kGroupQ * 2 * kp * 8 + 1024; }
+  static_assert(kGroupQ <= NQ && NQ % 16 == 0, "the group fits the MMA's N");
+  static_assert(STAGE_BYTES % 1024 == 0 && OFF_U % 1024 == 0, "swizzled blocks on 1024-byte boundaries");
+};
+
+// 16 bytes (8 bf16 of K columns 8 c8 .. 8 c8 + 7) of row n of u's part `part`,
+// in the swizzled K-major layout the MMA's B descriptor reads.
+template <int P>
+__device__ __forceinline__ void store_u_chunk(uint8_t* sU, int part, int n, int c8, uint4 v) {
+  using C = DcCfg<P>;
+  uint32_t off;
+  if constexpr (P == 128) {
+    const int kb = c8 >> 3, ch = c8 & 7;
+    off = part * C::U_PART + kb * (C::NQ * 128) + n * 128 + ((ch ^ (n & 7)) << 4);
+  } else {
+    const int sw = P == 64 ? (n & 7) : (P == 32 ? ((n >> 1) & 3) : ((n >> 2) & 1));
+    off = part * C::U_PART + n * (2 * P) + ((c8 ^ sw) << 4);
+  }
+  *reinterpret_cast<uint4*>(sU + off) = v;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo_elem, float hi_elem) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo_elem, hi_elem);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+template <int P, int KP>
+__global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_constant__ CUtensorMap tmX,
+                                                              const ScoreArgs a) {
+  using C = DcCfg<P>;
+  constexpr int CAP = 2 * KP;
+  constexpr int EK = KP / 32;
+  constexpr int GQ = kGroupQ;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint8_t* sStage = smem;
+  uint8_t* sU = smem + C::OFF_U;
+  uint64_t* buf = reinterpret_cast<uint64_t*>(smem + C::OFF_BUF);   // [4 warps][GQ][CAP]
+  __shared__ float qs[GQ][kD];
+  __shared__ float us[GQ][P];
+  __shared__ float qnu[GQ];
+  __shared__ int visq[GQ];
+  __shared__ int cnt_s[4 * GQ];
+  __shared__ unsigned long long cta_thr[GQ];
+  __shared__ __align__(8) uint64_t bars[2 * C::STAGES + 2 * C::NB + 2];
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_s;
+  uint64_t* full = bars;
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* accf = empty + C::STAGES;
+  uint64_t* acce = accf + C::NB;
+  uint64_t* uready = acce + C::NB;
+  uint64_t* drain = uready + 1;
+  volatile int* abort_f = &abort_s;
+
+  const ScoreItem it = a.items[blockIdx.x];
+  const int h = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nq = it.q_count;
+  const int nkeys = it.key_hi - it.key_lo;
+  const int ntiles = (nkeys + C::NT - 1) / C::NT;
+
+  if (threadIdx.x == 0) {
+    for (int s2 = 0; s2 < C::STAGES; ++s2) {
+      tc::mbar_init(full + s2, 1);
+      tc::mbar_init(empty + s2, 1);
+    }
+    for (int b = 0; b < C::NB; ++b) {
+      tc::mbar_init(accf + b, 1);
+      tc::mbar_init(acce + b, 128);
+    }
+    tc::mbar_init(uready, 128);
+    tc::mbar_init(drain, 1);
+    *abort_f = 0;
+    tc::fence_barrier_init();
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(&tmem_slot, C::NB * C::NQ);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmX);
+      const int64_t xrow = (int64_t)(a.exact ? h / a.G : h) * a.N + it.key_base + it.key_lo;
+      int issued = 0;
+      for (int i = 0; i < ntiles; ++i) {
+        const int st = i % C::STAGES;
+        if (!tc::mbar_wait(empty + st, ((i / C::STAGES) & 1) ^ 1, abort_f)) break;
+        tc::mbar_arrive_expect_tx(full + st, C::STAGE_BYTES);
+#pragma unroll
+        for (int kb = 0; kb < C::KB; ++kb)
+          tc::tma_load_2d(sStage + st * C::STAGE_BYTES + kb * (C::NT * C::KW * 2), &tmX, full + st, kb * C::KW,
+                          (int)(xrow + (int64_t)i * C::NT));
+        ++issued;
+      }
+      // every issued load has landed before the CTA may exit
+      for (int s2 = 0; s2 < C::STAGES && s2 < issued; ++s2) {
+        const int last = s2 + C::STAGES * ((issued - 1 - s2) / C::STAGES);
+        if (!tc::mbar_wait_bounded(full + s2, (last / C::STAGES) & 1)) *abort_f = 1;
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16(C::NT, C::NQ);
+      const uint32_t sBase = tc::smem_u32(sStage), uBase = tc::smem_u32(sU);
+      bool ok = tc::mbar_wait(uready, 0, abort_f);
+      if (ok) tc::fence_after_sync();
+      for (int i = 0; ok && i < ntiles; ++i) {
+        const int st = i % C::STAGES, b = i % C::NB;
+        if (!(ok = tc::mbar_wait(acce + b, ((i / C::NB) & 1) ^ 1, abort_f))) break;
+        if (!(ok = tc::mbar_wait(full + st, (i / C::STAGES) & 1, abort_f))) break;
+        tc::fence_after_sync();
+        uint32_t accum = 0;
+#pragma unroll
+        for (int part = 0; part < 2; ++part)
+#pragma unroll
+          for (int kb = 0; kb < C::KB; ++kb)
+#pragma unroll
+            for (int kk = 0; kk < C::KK; ++kk) {
+              const uint32_t ad = sBase + st * C::STAGE_BYTES + kb * (C::NT * C::KW * 2) + kk * 32;
+              const uint32_t bd = uBase + part * C::U_PART + kb * (C::NQ * C::KW * 2) + kk * 32;
+              tc::mma_bf16(tmem + b * C::NQ, tc::sdesc(ad, C::SBO, C::SW), tc::sdesc(bd, C::SBO, C::SW), idesc,
+                           accum);
+              accum = 1;
+            }
+        tc::mma_commit(empty + st);
+        tc::mma_commit(accf + b);
+      }
+      tc::mma_commit(drain);
+      if (!tc::mbar_wait_bounded(drain, 0)) *abort_f = 1;
+    }
+  } else {
+    // ------------------------------------------------------------ projection and selection
+    const int e = warp - 2;                 // candidate buffers of this warp
+    const int quarter = warp & 3;           // the TMEM lanes (keys of a tile) this warp may read
+    const int et = threadIdx.x - 64;
+    const __nv_bfloat16* Q = static_cast<const __nv_bfloat16*>(a.Q);
+    for (int o = et; o < GQ * kD; o += 128) {
+      const int b = o / kD;
+      qs[b][o % kD] = b < nq ? __bfloat162float(Q[((int64_t)h * a.T + it.q_begin + b) * kD + (o % kD)]) : 0.f;
+    }
+    if (et < GQ) {
+      visq[et] = et < nq ? a.vis[it.q_begin + et] : 0;
+      cta_thr[et] = 0ull;
+    }
+    if (et < 4 * GQ) cnt_s[et] = 0;
+    for (int o = et; o < 4 * GQ * CAP; o += 128) buf[o] = 0ull;
+    epilogue_sync();
+    // u_b = W_h^T q_b (fp32) and the mean term q_b^T nu_h
+    const float* W = a.W + (int64_t)h * kD * P;
+    for (int o = et; o < GQ * P; o += 128) {
+      const int b = o / P, p = o % P;
+      float acc = 0.f;
+      for (int i = 0; i < kD; ++i) acc = fmaf(__ldg(W + i * P + p), qs[b][i], acc);
+      us[b][p] = acc;
+    }
+    for (int b = e; b < GQ; b += 4) {
+      float v = 0.f;
+      if (a.nu)
+        for (int i = lane; i < kD; i += 32) v = fmaf(qs[b][i], __ldg(a.nu + (int64_t)h * kD + i), v);
+      v = warp_sum(v);
+      if (lane == 0) qnu[b] = v;
+    }
+    epilogue_sync();
+    // u = u_hi + u_lo in bf16, the MMA's B operand; rows past the group are zero
+    for (int o = et; o < C::NQ * (P / 8); o += 128) {
+      const int n = o / (P / 8), c8 = o % (P / 8);
+      uint32_t hw[4], lw[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float u0 = n < nq ? us[n][8 * c8 + 2 * q] : 0.f, u1 = n < nq ? us[n][8 * c8 + 2 * q + 1] : 0.f;
+        const float h0 = __bfloat162float(__float2bfloat16_rn(u0)), h1 = __bfloat162float(__float2bfloat16_rn(u1));
+        hw[q] = pack_bf16x2(h0, h1);
+        lw[q] = pack_bf16x2(u0 - h0, u1 - h1);
+      }
+      store_u_chunk<P>(sU, 0, n, c8, make_uint4(hw[0], hw[1], hw[2], hw[3]));
+      store_u_chunk<P>(sU, 1, n, c8, make_uint4(lw[0], lw[1], lw[2], lw[3]));
+    }
+    tc::fence_proxy_async_smem();
+    tc::mbar_arrive(uready);
+
+    uint64_t thr[GQ];
+    float thr_f[GQ];   // score part of thr: a key can only pass if its score is >= thr_f
+#pragma unroll
+    for (int b = 0; b < GQ; ++b) {
+      thr[b] = 0ull;
+      thr_f[b] = -INFINITY;
+    }
+    uint64_t* wbuf = buf + e * GQ * CAP;
+    int* wcnt = cnt_s + e * GQ;
+    const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
+    for (int i = 0; i < ntiles; ++i) {
+      const int b = i % C::NB;
+      if (!__all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f))) break;
+      tc::fence_after_sync();
+      uint32_t r[16];
+      __syncwarp();
+      tc::tmem_ld16(tl + b * C::NQ, r);
+      tc::tmem_ld_wait(r);
+      tc::fence_before_sync();
+      tc::mbar_arrive(acce + b);
+      const int jl = i * C::NT + quarter * 32 + lane;
+      const int j = it.key_lo + jl;
+#pragma unroll
+      for (int q = 0; q < GQ; ++q) {
+        if (q < nq) {
+          const float sc = __uint_as_float(r[q]);
+          const bool ok = jl < nkeys && j < visq[q] && sc >= thr_f[q];
+          if (__ballot_sync(0xffffffffu, ok)) {
+            const uint64_t key = make_key(sc, (uint32_t)j);
+            const bool pass = ok && key > thr[q];
+            const unsigned mask = __ballot_sync(0xffffffffu, pass);
+            if (mask) {
+              thr[q] = append_keys<KP>(wbuf + q * CAP, wcnt + q, cta_thr + q, key, pass, mask, thr[q], a.k);
+              thr_f[q] = key_score(thr[q]);
+            }
+          }
+        }
+      }
+    }
+    for (int q = 0; q < nq; ++q) {
+      int c = wcnt[q];
+      reselect<KP>(wbuf + q * CAP, c, a.k);
+    }
+    epilogue_sync();
+    // merge the four warps' lists of each query
+    for (int q = e; q < nq; q += 4) {
+      uint64_t best[EK], other[EK];
+#pragma unroll
+      for (int x = 0; x < EK; ++x) best[x] = buf[(0 * GQ + q) * CAP + x * 32 + lane];
+      for (int w2 = 1; w2 < 4; ++w2) {
+#pragma unroll
+        for (int x = 0; x < EK; ++x) other[x] = buf[(w2 * GQ + q) * CAP + x * 32 + lane];
+        warp_merge_top<EK>(best, other);
+      }
+      if (it.cand < 0) {
+        const int64_t row = ((int64_t)h * a.T + it.q_begin + q) * a.k;
+#pragma unroll
+        for (int x = 0; x < EK; ++x) {
+          const int ii = x * 32 + lane;
+          if (ii < a.k) {
+            a.idx[row + ii] = key_index(best[x]);
+            if (a.score) a.score[row + ii] = best[x] ? key_score(best[x]) + qnu[q] : -INFINITY;
+          }
+        }
+      } else {
+        uint64_t* c = a.cand + ((int64_t)h * a.cand_per_head + it.cand + (int64_t)q * it.cand_stride) * KP;
+#pragma unroll
+        for (int x = 0; x < EK; ++x) c[x * 32 + lane] = best[x];
+      }
+    }
+  }
+
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (*abort_f && threadIdx.x == 0) atomicOr(a.err, kStTimeout);
+  if (warp == 1) tc::tmem_dealloc(tmem, C::NB * C::NQ);
+}
+
+template <int P, int KP>
+cudaError_t launch_decode_tc_t(const ScoreArgs& a, cudaStream_t s) {
+  using C = DcCfg<P>;
+  const int xheads = a.exact ? a.Hq / a.G : a.Hq;
+  CUtensorMap mX;
+  if (!make_tmap(&mX, a.X, (uint64_t)P, (uint64_t)xheads * a.N, C::KW, C::NT, swizzle_for(C::KW)))
+    return cudaErrorInvalidValue;
+  const int sm = C::smem(KP);
+  auto kern = score_decode_tc_kernel<P, KP>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  if (e != cudaSuccess) return e;
+  note_launch();
+  kern<<<dim3(a.n_items, a.Hq), 192, sm, s>>>(mX, a);
+  return cudaGetLastError();
+}
+
+template <int KP>
+cudaError_t launch_decode_tc(const ScoreArgs& a, cudaStream_t s) {
+  switch (a.P) {
+    case 16: return launch_decode_tc_t<16, KP>(a, s);
+    case 32: return launch_decode_tc_t<32, KP>(a, s);
+    case 64: return launch_decode_tc_t<64, KP>(a, s);
+    default: return launch_decode_tc_t<128, KP>(a, s);
+  }
+}
+
 template <typename Tin, int KP, int NQ>
 cudaError_t launch_score_t(const ScoreArgs& a, cudaStream_t s) {
   const size_t sm = score_generic_smem(a.P, KP, NQ);
@@ -306,6 +632,9 @@ cudaError_t launch_nq(const ScoreArgs& a, int nq, cudaStream_t s) {
 
 cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, cudaStream_t s) {
   if (a.n_items == 0) return cudaSuccess;
+  // bf16 keys or codes of a tensor-core width take the tensor-core variant
+  if (dtype == SAKI_BF16 && a.err && (a.P == 16 || a.P == 32 || a.P == 64 || a.P == 128))
+    return kp == 64 ? launch_decode_tc<64>(a, s) : launch_decode_tc<128>(a, s);
   if (dtype == SAKI_BF16)
     return kp == 64 ? launch_nq<__nv_bfloat16, 64>(a, nq, s) : launch_nq<__nv_bfloat16, 128>(a, nq, s);
   return kp == 64 ? launch_nq<float, 64>(a, nq, s) : launch_nq<float, 128>(a, nq, s);

@@ -31,6 +31,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "tc.cuh"
+#include "tmap.cuh"
 
 namespace saki {
 namespace {
@@ -962,45 +963,15 @@ __global__ void qnu_kernel(const __nv_bfloat16* Q, const float* nu, int64_t T, i
   if (lane == 0) out[rowi] = v;
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
-  return fn;
-}
-
-bool make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t rows, uint32_t box_inner, uint32_t box_rows,
-              CUtensorMapSwizzle sw) {
-  auto enc = encoder();
-  if (!enc) return false;
-  cuuint64_t dims[2] = {inner, rows};
-  cuuint64_t strides[1] = {inner * 2};
-  cuuint32_t box[2] = {box_inner, box_rows};
-  cuuint32_t es[2] = {1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-CUtensorMapSwizzle swz_of(int kw) {
-  return kw == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : (kw == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B);
-}
-
 template <int P>
 cudaError_t launch_tc_t(const TcLaunch& L, cudaStream_t s) {
   using C = TcCfg<P>;
   CUtensorMap mQ, mW, mX;
   const int xrows_heads = L.args.exact ? L.Hk : L.args.Hq;
   const int xcols = L.args.exact ? kD : P;
-  if (!make_map(&mQ, L.Q, kD, (uint64_t)L.args.Hq * L.args.T, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mW, L.Wsplit, kD, (uint64_t)L.args.Hq * 3 * P, 64, P, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !make_map(&mX, L.X, xcols, (uint64_t)xrows_heads * L.args.N, C::KW, C::NT, swz_of(C::KW)))
+  if (!make_tmap(&mQ, L.Q, kD, (uint64_t)L.args.Hq * L.args.T, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_tmap(&mW, L.Wsplit, kD, (uint64_t)L.args.Hq * 3 * P, 64, P, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_tmap(&mX, L.X, xcols, (uint64_t)xrows_heads * L.args.N, C::KW, C::NT, swizzle_for(C::KW)))
     return cudaErrorInvalidValue;
   auto kern = score_tc_kernel<P>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
