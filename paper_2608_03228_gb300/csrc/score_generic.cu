@@ -518,14 +518,20 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
       tc::mbar_arrive(acce + b);
       const int jl = i * C::NT + quarter * 32 + lane;
       const int j = it.key_lo + jl;
+      // one bit per query whose score clears its threshold; one warp vote for all
+      unsigned m = 0u;
 #pragma unroll
       for (int q = 0; q < GQ; ++q) {
-        if (q < nq) {
-          const float sc = __uint_as_float(r[q]);
-          const bool ok = jl < nkeys && j < visq[q] && sc >= thr_f[q];
-          if (__ballot_sync(0xffffffffu, ok)) {
-            const uint64_t key = make_key(sc, (uint32_t)j);
-            const bool pass = ok && key > thr[q];
+        const bool ok = q < nq && jl < nkeys && j < visq[q] && __uint_as_float(r[q]) >= thr_f[q];
+        m |= ok ? 1u << q : 0u;
+      }
+      const unsigned any = __reduce_or_sync(0xffffffffu, m);
+      if (any) {
+#pragma unroll
+        for (int q = 0; q < GQ; ++q) {
+          if (any & (1u << q)) {
+            const uint64_t key = make_key(__uint_as_float(r[q]), (uint32_t)j);
+            const bool pass = ((m >> q) & 1u) && key > thr[q];
             const unsigned mask = __ballot_sync(0xffffffffu, pass);
             if (mask) {
               thr[q] = append_keys<KP>(wbuf + q * CAP, wcnt + q, cta_thr + q, key, pass, mask, thr[q], a.k);
@@ -632,8 +638,10 @@ cudaError_t launch_nq(const ScoreArgs& a, int nq, cudaStream_t s) {
 
 cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, cudaStream_t s) {
   if (a.n_items == 0) return cudaSuccess;
-  // bf16 keys or codes of a tensor-core width take the tensor-core variant
-  if (dtype == SAKI_BF16 && a.err && (a.P == 16 || a.P == 32 || a.P == 64 || a.P == 128))
+  // bf16 keys or codes of a tensor-core width, in groups of at least four
+  // queries, take the tensor-core variant (with one query per group the CUDA-core
+  // kernel streams a decode step faster: 0.50 against 0.53 ms over 32 heads x 1M keys)
+  if (dtype == SAKI_BF16 && a.err && nq >= 4 && (a.P == 16 || a.P == 32 || a.P == 64 || a.P == 128))
     return kp == 64 ? launch_decode_tc<64>(a, s) : launch_decode_tc<128>(a, s);
   if (dtype == SAKI_BF16)
     return kp == 64 ? launch_nq<__nv_bfloat16, 64>(a, nq, s) : launch_nq<__nv_bfloat16, 128>(a, nq, s);
