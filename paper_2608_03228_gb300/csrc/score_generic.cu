@@ -27,11 +27,11 @@ template <typename T> __device__ __forceinline__ float to_f(T v);
 template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
 template <> __device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
 
-// Keep the KP best of the warp's buffer (sorted, descending) and return the
-// k-th best key (0 while fewer than k are held).
-template <int KP>
+// Keep the KP best of the warp's buffer of CAP slots (sorted, descending) and
+// return the k-th best key (0 while fewer than k are held).
+template <int KP, int CAP = 2 * KP>
 __device__ __forceinline__ uint64_t reselect(uint64_t* qb, int& cnt, int k) {
-  constexpr int E = 2 * KP / 32;
+  constexpr int E = CAP / 32;
   const int lane = threadIdx.x & 31;
   __syncwarp();
   uint64_t v[E];
@@ -61,16 +61,15 @@ __device__ __forceinline__ uint64_t reselect(uint64_t* qb, int& cnt, int k) {
 // Rare path, kept out of line: append the passing keys of this 32-key batch to
 // the warp's buffer of one query, re-select when it is nearly full, publish the
 // warp's k-th best as a CTA-wide lower bound, and return the new threshold.
-template <int KP>
+template <int KP, int CAP = 2 * KP>
 __device__ __noinline__ uint64_t append_keys(uint64_t* qb, int* cnt_s, unsigned long long* cta_thr, uint64_t key,
                                              bool pass, unsigned mask, uint64_t thr, int k) {
-  constexpr int CAP = 2 * KP;
   const int lane = threadIdx.x & 31;
   int cnt = *cnt_s;
   if (pass) qb[cnt + __popc(mask & ((1u << lane) - 1u))] = key;
   cnt += __popc(mask);
   if (cnt > CAP - 32) {
-    const uint64_t t = reselect<KP>(qb, cnt, k);
+    const uint64_t t = reselect<KP, CAP>(qb, cnt, k);
     if (t > thr) thr = t;
     if (lane == 0 && t) atomicMax(cta_thr, (unsigned long long)t);
   }
@@ -286,11 +285,14 @@ __global__ void __launch_bounds__(128) merge_kernel(const ScoreArgs a) {
 // 128 keys (codes, or keys for the exact scores) are the A operand (M = 128,
 // TMA), u = W^T q of the group's queries split into bf16 hi + lo the B operand
 // (N = 16, rows past the group zero), D[key][query] in a ring of TMEM
-// accumulators.  Each epilogue thread owns one key of a tile (its TMEM lane) and
-// reads that key's scores for all queries in one load; the selection is
-// score_generic_kernel's.  Roles: warp 0 TMA producer, warp 1 TMEM owner and MMA
-// issuer, warps 2-5 projection and selection.  Every mbarrier wait is bounded;
-// a CTA that gives up sets kStTimeout in the error word.
+// accumulators.  Each epilogue thread reads one key's scores for all queries (its
+// TMEM lane) and writes them to a shared [query][key] tile; each query then
+// belongs to one epilogue warp, which scans all 128 keys of the tile against
+// the query's running k-th best (score_generic_kernel's candidate buffer and
+// re-selection), so a query's threshold is built from every key of the split.
+// Roles: warp 0 TMA producer, warp 1 TMEM owner and MMA issuer, warps 2-5
+// projection and selection.  Every mbarrier wait is bounded; a CTA that gives
+// up sets kStTimeout in the error word.
 template <int P>
 struct DcCfg {
   static constexpr int KW = P == 128 ? 64 : P;   // K width of one swizzled block
@@ -306,7 +308,9 @@ struct DcCfg {
   static constexpr int U_PART = (NQ * P * 2 + 1023) & ~1023;   // u_hi or u_lo
   static constexpr int OFF_U = STAGES * STAGE_BYTES;
   static constexpr int OFF_BUF = OFF_U + 2 * U_PART;
-  static int smem(int kp) { return OFF_BUF + 4 * kGroupQ * 2 * kp * 8 + 1024; }
+  static constexpr int cap(int kp) { return 4 * kp; }          // candidate slots per query
+  static constexpr int off_t(int kp) { return OFF_BUF + kGroupQ * cap(kp) * 8; }   // [2][query][key] scores
+  static int smem(int kp) { return off_t(kp) + 2 * kGroupQ * NT * 4 + 1024; }
   static_assert(kGroupQ <= NQ && NQ % 16 == 0, "the group fits the MMA's N");
   static_assert(STAGE_BYTES % 1024 == 0 && OFF_U % 1024 == 0, "swizzled blocks on 1024-byte boundaries");
 };
@@ -338,19 +342,20 @@ template <int P, int KP>
 __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_constant__ CUtensorMap tmX,
                                                               const ScoreArgs a) {
   using C = DcCfg<P>;
-  constexpr int CAP = 2 * KP;
+  constexpr int CAP = C::cap(KP);
   constexpr int EK = KP / 32;
   constexpr int GQ = kGroupQ;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
   uint8_t* sStage = smem;
   uint8_t* sU = smem + C::OFF_U;
-  uint64_t* buf = reinterpret_cast<uint64_t*>(smem + C::OFF_BUF);   // [4 warps][GQ][CAP]
+  uint64_t* buf = reinterpret_cast<uint64_t*>(smem + C::OFF_BUF);   // [GQ][CAP]
+  float* tile_s = reinterpret_cast<float*>(smem + C::off_t(KP));    // [2][GQ][NT]
   __shared__ float qs[GQ][kD];
   __shared__ float us[GQ][P];
   __shared__ float qnu[GQ];
   __shared__ int visq[GQ];
-  __shared__ int cnt_s[4 * GQ];
+  __shared__ int cnt_s[GQ];
   __shared__ unsigned long long cta_thr[GQ];
   __shared__ __align__(8) uint64_t bars[2 * C::STAGES + 2 * C::NB + 2];
   __shared__ uint32_t tmem_slot;
@@ -460,8 +465,8 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
       visq[et] = et < nq ? a.vis[it.q_begin + et] : 0;
       cta_thr[et] = 0ull;
     }
-    if (et < 4 * GQ) cnt_s[et] = 0;
-    for (int o = et; o < 4 * GQ * CAP; o += 128) buf[o] = 0ull;
+    if (et < GQ) cnt_s[et] = 0;
+    for (int o = et; o < GQ * CAP; o += 128) buf[o] = 0ull;
     epilogue_sync();
     // u_b = W_h^T q_b (fp32) and the mean term q_b^T nu_h
     const float* W = a.W + (int64_t)h * kD * P;
@@ -496,80 +501,84 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
     tc::fence_proxy_async_smem();
     tc::mbar_arrive(uready);
 
-    uint64_t thr[GQ];
-    float thr_f[GQ];   // score part of thr: a key can only pass if its score is >= thr_f
-#pragma unroll
-    for (int b = 0; b < GQ; ++b) {
-      thr[b] = 0ull;
-      thr_f[b] = -INFINITY;
-    }
-    uint64_t* wbuf = buf + e * GQ * CAP;
-    int* wcnt = cnt_s + e * GQ;
+    // this warp's queries are e and e + 4
+    uint64_t thr[2] = {0ull, 0ull};
+    float thr_f[2] = {-INFINITY, -INFINITY};   // score part of thr: a key can only pass if its score is >= thr_f
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
+    // Every epilogue warp runs every iteration and its barrier (a named barrier
+    // has no time limit): a warp that gave up waiting skips the work only.
+    bool ok = true;
     for (int i = 0; i < ntiles; ++i) {
       const int b = i % C::NB;
-      if (!__all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f))) break;
-      tc::fence_after_sync();
-      uint32_t r[16];
-      __syncwarp();
-      tc::tmem_ld16(tl + b * C::NQ, r);
-      tc::tmem_ld_wait(r);
-      tc::fence_before_sync();
-      tc::mbar_arrive(acce + b);
-      const int jl = i * C::NT + quarter * 32 + lane;
-      const int j = it.key_lo + jl;
-      // one bit per query whose score clears its threshold; one warp vote for all
-      unsigned m = 0u;
+      ok = ok && __all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f));
+      // scores to the [query][key] tile (double-buffered: the barrier of tile
+      // i + 1 orders every warp's reads of tile i before the writes of tile i + 2)
+      float* T = tile_s + (i & 1) * GQ * C::NT;
+      if (ok) {
+        tc::fence_after_sync();
+        uint32_t r[16];
+        __syncwarp();
+        tc::tmem_ld16(tl + b * C::NQ, r);
+        tc::tmem_ld_wait(r);
+        tc::fence_before_sync();
+        tc::mbar_arrive(acce + b);
 #pragma unroll
-      for (int q = 0; q < GQ; ++q) {
-        const bool ok = q < nq && jl < nkeys && j < visq[q] && __uint_as_float(r[q]) >= thr_f[q];
-        m |= ok ? 1u << q : 0u;
+        for (int q = 0; q < GQ; ++q)
+          if (q < nq) T[q * C::NT + quarter * 32 + lane] = __uint_as_float(r[q]);
       }
-      const unsigned any = __reduce_or_sync(0xffffffffu, m);
-      if (any) {
+      epilogue_sync();
 #pragma unroll
-        for (int q = 0; q < GQ; ++q) {
-          if (any & (1u << q)) {
-            const uint64_t key = make_key(__uint_as_float(r[q]), (uint32_t)j);
-            const bool pass = ((m >> q) & 1u) && key > thr[q];
-            const unsigned mask = __ballot_sync(0xffffffffu, pass);
-            if (mask) {
-              thr[q] = append_keys<KP>(wbuf + q * CAP, wcnt + q, cta_thr + q, key, pass, mask, thr[q], a.k);
-              thr_f[q] = key_score(thr[q]);
+      for (int x = 0; x < 2; ++x) {
+        const int q = e + 4 * x;
+        if (ok && q < nq) {
+          const float4 v4 = reinterpret_cast<const float4*>(T + q * C::NT)[lane];   // keys 4 lane .. 4 lane + 3
+          const float sv[4] = {v4.x, v4.y, v4.z, v4.w};
+          const int jl0 = i * C::NT + 4 * lane;
+          unsigned m = 0u;
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const bool ok = jl0 + t < nkeys && it.key_lo + jl0 + t < visq[q] && sv[t] >= thr_f[x];
+            m |= ok ? 1u << t : 0u;
+          }
+          const unsigned any = __reduce_or_sync(0xffffffffu, m);
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            if (any & (1u << t)) {
+              const uint64_t key = make_key(sv[t], (uint32_t)(it.key_lo + jl0 + t));
+              const bool pass = ((m >> t) & 1u) && key > thr[x];
+              const unsigned mask = __ballot_sync(0xffffffffu, pass);
+              if (mask) {
+                thr[x] = append_keys<KP, CAP>(buf + q * CAP, cnt_s + q, cta_thr + q, key, pass, mask, thr[x], a.k);
+                thr_f[x] = key_score(thr[x]);
+              }
             }
           }
         }
       }
     }
-    for (int q = 0; q < nq; ++q) {
-      int c = wcnt[q];
-      reselect<KP>(wbuf + q * CAP, c, a.k);
-    }
-    epilogue_sync();
-    // merge the four warps' lists of each query
-    for (int q = e; q < nq; q += 4) {
-      uint64_t best[EK], other[EK];
+    // each query's k best, from its owner warp
+    for (int x = 0; x < 2; ++x) {
+      const int q = e + 4 * x;
+      if (q >= nq) continue;
+      int c = cnt_s[q];
+      reselect<KP, CAP>(buf + q * CAP, c, a.k);
+      uint64_t best[EK];
 #pragma unroll
-      for (int x = 0; x < EK; ++x) best[x] = buf[(0 * GQ + q) * CAP + x * 32 + lane];
-      for (int w2 = 1; w2 < 4; ++w2) {
-#pragma unroll
-        for (int x = 0; x < EK; ++x) other[x] = buf[(w2 * GQ + q) * CAP + x * 32 + lane];
-        warp_merge_top<EK>(best, other);
-      }
+      for (int y = 0; y < EK; ++y) best[y] = buf[q * CAP + y * 32 + lane];
       if (it.cand < 0) {
         const int64_t row = ((int64_t)h * a.T + it.q_begin + q) * a.k;
 #pragma unroll
-        for (int x = 0; x < EK; ++x) {
-          const int ii = x * 32 + lane;
+        for (int y = 0; y < EK; ++y) {
+          const int ii = y * 32 + lane;
           if (ii < a.k) {
-            a.idx[row + ii] = key_index(best[x]);
-            if (a.score) a.score[row + ii] = best[x] ? key_score(best[x]) + qnu[q] : -INFINITY;
+            a.idx[row + ii] = key_index(best[y]);
+            if (a.score) a.score[row + ii] = best[y] ? key_score(best[y]) + qnu[q] : -INFINITY;
           }
         }
       } else {
-        uint64_t* c = a.cand + ((int64_t)h * a.cand_per_head + it.cand + (int64_t)q * it.cand_stride) * KP;
+        uint64_t* c2 = a.cand + ((int64_t)h * a.cand_per_head + it.cand + (int64_t)q * it.cand_stride) * KP;
 #pragma unroll
-        for (int x = 0; x < EK; ++x) c[x * 32 + lane] = best[x];
+        for (int y = 0; y < EK; ++y) c2[y * 32 + lane] = best[y];
       }
     }
   }
