@@ -309,8 +309,9 @@ struct DcCfg {
   static constexpr int OFF_U = STAGES * STAGE_BYTES;
   static constexpr int OFF_BUF = OFF_U + 2 * U_PART;
   static constexpr int cap(int kp) { return 4 * kp; }          // candidate slots per query
-  static constexpr int off_t(int kp) { return OFF_BUF + kGroupQ * cap(kp) * 8; }   // [2][query][key] scores
-  static int smem(int kp) { return off_t(kp) + 2 * kGroupQ * NT * 4 + 1024; }
+  static constexpr int TS = 4;                                  // [query][key] score tiles in flight
+  static constexpr int off_t(int kp) { return OFF_BUF + kGroupQ * cap(kp) * 8; }   // [TS][query][key] scores
+  static int smem(int kp) { return off_t(kp) + TS * kGroupQ * NT * 4 + 1024; }
   static_assert(kGroupQ <= NQ && NQ % 16 == 0, "the group fits the MMA's N");
   static_assert(STAGE_BYTES % 1024 == 0 && OFF_U % 1024 == 0, "swizzled blocks on 1024-byte boundaries");
 };
@@ -350,14 +351,14 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
   uint8_t* sStage = smem;
   uint8_t* sU = smem + C::OFF_U;
   uint64_t* buf = reinterpret_cast<uint64_t*>(smem + C::OFF_BUF);   // [GQ][CAP]
-  float* tile_s = reinterpret_cast<float*>(smem + C::off_t(KP));    // [2][GQ][NT]
+  float* tile_s = reinterpret_cast<float*>(smem + C::off_t(KP));    // [TS][GQ][NT]
   __shared__ float qs[GQ][kD];
   __shared__ float us[GQ][P];
   __shared__ float qnu[GQ];
   __shared__ int visq[GQ];
   __shared__ int cnt_s[GQ];
   __shared__ unsigned long long cta_thr[GQ];
-  __shared__ __align__(8) uint64_t bars[2 * C::STAGES + 2 * C::NB + 2];
+  __shared__ __align__(8) uint64_t bars[2 * C::STAGES + 2 * C::NB + 2 + 2 * C::TS];
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_s;
   uint64_t* full = bars;
@@ -366,6 +367,8 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
   uint64_t* acce = accf + C::NB;
   uint64_t* uready = acce + C::NB;
   uint64_t* drain = uready + 1;
+  uint64_t* tfull = drain + 1;      // [TS] a score tile written by all four epilogue warps
+  uint64_t* tempty = tfull + C::TS;  // [TS] its queries read by all four
   volatile int* abort_f = &abort_s;
 
   const ScoreItem it = a.items[blockIdx.x];
@@ -386,6 +389,10 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
     }
     tc::mbar_init(uready, 128);
     tc::mbar_init(drain, 1);
+    for (int t = 0; t < C::TS; ++t) {
+      tc::mbar_init(tfull + t, 128);
+      tc::mbar_init(tempty + t, 128);
+    }
     *abort_f = 0;
     tc::fence_barrier_init();
   }
@@ -505,32 +512,36 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
     uint64_t thr[2] = {0ull, 0ull};
     float thr_f[2] = {-INFINITY, -INFINITY};   // score part of thr: a key can only pass if its score is >= thr_f
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
-    // Every epilogue warp runs every iteration and its barrier (a named barrier
-    // has no time limit): a warp that gave up waiting skips the work only.
+    // Scores pass through a ring of TS shared [query][key] tiles: every warp
+    // writes its quarter of the keys of tile i and reads all keys of its own
+    // queries, with mbarriers between writers and readers so that the warps can
+    // drift up to TS - 1 tiles apart (a warp whose queries take many appends on
+    // one tile no longer holds the others).  All waits are bounded.
     bool ok = true;
-    for (int i = 0; i < ntiles; ++i) {
-      const int b = i % C::NB;
-      ok = ok && __all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f));
-      // scores to the [query][key] tile (double-buffered: the barrier of tile
-      // i + 1 orders every warp's reads of tile i before the writes of tile i + 2)
-      float* T = tile_s + (i & 1) * GQ * C::NT;
-      if (ok) {
-        tc::fence_after_sync();
-        uint32_t r[16];
-        __syncwarp();
-        tc::tmem_ld16(tl + b * C::NQ, r);
-        tc::tmem_ld_wait(r);
-        tc::fence_before_sync();
-        tc::mbar_arrive(acce + b);
+    for (int i = 0; i < ntiles && ok; ++i) {
+      const int b = i % C::NB, ts = i % C::TS;
+      const uint32_t tph = (i / C::TS) & 1;
+      float* T = tile_s + ts * GQ * C::NT;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f) &&
+                                       tc::mbar_wait(tempty + ts, tph ^ 1, abort_f));
+      if (!ok) break;
+      tc::fence_after_sync();
+      uint32_t r[16];
+      __syncwarp();
+      tc::tmem_ld16(tl + b * C::NQ, r);
+      tc::tmem_ld_wait(r);
+      tc::fence_before_sync();
+      tc::mbar_arrive(acce + b);
 #pragma unroll
-        for (int q = 0; q < GQ; ++q)
-          if (q < nq) T[q * C::NT + quarter * 32 + lane] = __uint_as_float(r[q]);
-      }
-      epilogue_sync();
+      for (int q = 0; q < GQ; ++q)
+        if (q < nq) T[q * C::NT + quarter * 32 + lane] = __uint_as_float(r[q]);
+      tc::mbar_arrive(tfull + ts);   // release: the tile's quarter is written
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(tfull + ts, tph, abort_f));
+      if (!ok) break;
 #pragma unroll
       for (int x = 0; x < 2; ++x) {
         const int q = e + 4 * x;
-        if (ok && q < nq) {
+        if (q < nq) {
           const float4 v4 = reinterpret_cast<const float4*>(T + q * C::NT)[lane];   // keys 4 lane .. 4 lane + 3
           const float sv[4] = {v4.x, v4.y, v4.z, v4.w};
           const int jl0 = i * C::NT + 4 * lane;
@@ -555,6 +566,7 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
           }
         }
       }
+      tc::mbar_arrive(tempty + ts);   // this warp has read its queries of the tile
     }
     // each query's k best, from its owner warp
     for (int x = 0; x < 2; ++x) {
