@@ -225,6 +225,7 @@ def test_score_topk_tiny_causal(lib, tiny):
     (2, 2, 128, 100, "f32", (500, 90), ([-1, 250, 99], [-1, 3])),          # r = d, k > 64 (wide buffers)
     (8, 2, 64, 64, "bf16", (40, 17, 6000, 64), ([-1, 20], [-1], [-1] * 4, [-1, 63])),  # ragged, short seqs
     (4, 1, 24, 32, "bf16", (2500,), (list(range(2400, 2500)),)),            # many groups of one sequence
+    (2, 2, 128, 100, "bf16", (5000,), ([-1] * 6,)),                         # tensor-core decode, r = d, k > 64
 ])
 def test_score_topk_layouts(lib, case):
     Hq, Hk, r, k, dtype, lens, queries = case
@@ -233,6 +234,11 @@ def test_score_topk_layouts(lib, case):
 
 def test_score_topk_mean_term(lib):
     _score_case(lib, 4, 1, 32, 64, "bf16", (700,), ([-1, 300],), center=1)
+
+
+def test_score_topk_mean_term_decode_group(lib):
+    """The mean term on the tensor-core decode path (groups of at least four queries)."""
+    _score_case(lib, 4, 1, 32, 64, "bf16", (1500,), ([-1, -1, 1200, 700, 64],), center=1)
 
 
 def test_score_topk_unsorted_flag(lib):
