@@ -192,15 +192,33 @@ struct Plan {
   int nq = 1;   // launch width: smallest power of two >= the largest group
   std::vector<ScoreItem> items;
   std::vector<MergeItem> merges;
+  std::vector<ScoreItem> sitems;    // sample pass of the seeded groups
+  std::vector<MergeItem> smerges;   // its merges, which write the seeds
   std::vector<int32_t> vis;
-  int64_t cand_slots = 0;
+  int64_t cand_slots = 0, scand_slots = 0;
   // workspace offsets (bytes)
-  size_t off_items = 0, off_merges = 0, off_vis = 0, off_err = 0, off_cand = 0, bytes = 0, staged = 0;
+  size_t off_items = 0, off_merges = 0, off_sitems = 0, off_smerges = 0, off_vis = 0, off_err = 0, off_cand = 0,
+         off_scand = 0, off_seed = 0, bytes = 0, staged = 0;
 };
+
+constexpr int kSeedMinSplits = 8;    // groups cut into at least this many splits are seeded
+constexpr int64_t kSeedKeys = 1024;  // sample keys per split (at most an eighth of a split)
 
 // Groups of up to kGroupQ consecutive queries of one sequence; a group's visible
 // range is cut into splits so that the grid has several CTAs per SM.
-Plan make_plan(const saki_layout* L, int Hq, int kp) {
+//
+// Seeding (groups of the tensor-core decode kernel with many splits): a split
+// that starts from an empty candidate buffer admits every key until its
+// threshold has risen, and for a 27,648-key split and k = 64 that is about 800
+// appends and five re-sorts per query.  A sample pass first reads the first
+// kSeedKeys keys of every split and keeps, per query, the best score of each of
+// the split's 128 key groups (one key per tile and thread); the seed merge takes
+// the k-th largest of these group maxima over all splits of the row.  k distinct
+// visible keys reach it, so it bounds the row's k-th best score from below and
+// the main pass may start each query's threshold there (about 50 appends per
+// split and query in place of 800, no re-sort).  The result is unchanged: every
+// key of the row's top k scores at least the seed.
+Plan make_plan(const saki_layout* L, int Hq, int kp, int dtype, int P) {
   Plan p;
   const int64_t T = L->num_queries;
   struct G { int32_t b, n; int64_t vmax; int32_t seq; };
@@ -220,6 +238,9 @@ Plan make_plan(const saki_layout* L, int Hq, int kp) {
   const int64_t target_per_head = std::max<int64_t>(1, (int64_t)8 * kNumSMs / Hq);
   int64_t chunk = std::max<int64_t>(2048, (work + target_per_head - 1) / target_per_head);
   chunk = (chunk + 255) / 256 * 256;
+  // the tensor-core kernel takes groups of at least four queries
+  const bool seedable = decode_tc_eligible(dtype, P, p.nq);
+  const int64_t samp = std::min<int64_t>(kSeedKeys, chunk / 8 / 128 * 128);
   for (const G& g : groups) {
     const int64_t base = L->seq_offsets[g.seq];
     const int32_t S = g.vmax > 0 ? (int32_t)((g.vmax + chunk - 1) / chunk) : 1;
@@ -227,24 +248,63 @@ Plan make_plan(const saki_layout* L, int Hq, int kp) {
       p.items.push_back(ScoreItem{g.b, g.n, 0, (int32_t)g.vmax, base, -1, 0, 0});
       continue;
     }
+    const bool seeded = seedable && S >= kSeedMinSplits;
     const int64_t slot0 = p.cand_slots;
     p.cand_slots += (int64_t)g.n * S;
+    const int64_t sslot0 = p.scand_slots;
+    if (seeded) p.scand_slots += (int64_t)g.n * S;
     for (int32_t s = 0; s < S; ++s) {
       const int64_t lo = s * chunk, hi = std::min<int64_t>(g.vmax, lo + chunk);
-      p.items.push_back(ScoreItem{g.b, g.n, (int32_t)lo, (int32_t)hi, base, slot0 + s, S, 0});
+      p.items.push_back(ScoreItem{g.b, g.n, (int32_t)lo, (int32_t)hi, base, slot0 + s, S, seeded ? 1 : 0});
+      if (seeded)
+        p.sitems.push_back(ScoreItem{g.b, g.n, (int32_t)lo, (int32_t)std::min(hi, lo + samp), base, sslot0 + s, S, 0});
     }
-    for (int32_t b = 0; b < g.n; ++b) p.merges.push_back(MergeItem{g.b + b, S, slot0 + (int64_t)b * S});
+    for (int32_t b = 0; b < g.n; ++b) {
+      p.merges.push_back(MergeItem{g.b + b, S, slot0 + (int64_t)b * S});
+      if (seeded) p.smerges.push_back(MergeItem{g.b + b, S, sslot0 + (int64_t)b * S});
+    }
   }
   p.vis.resize(T);
   for (int64_t t = 0; t < T; ++t) p.vis[t] = (int32_t)L->q_visible[t];
   p.off_items = 0;
   p.off_merges = align_up(p.items.size() * sizeof(ScoreItem));
-  p.off_vis = p.off_merges + align_up(p.merges.size() * sizeof(MergeItem));
+  p.off_sitems = p.off_merges + align_up(p.merges.size() * sizeof(MergeItem));
+  p.off_smerges = p.off_sitems + align_up(p.sitems.size() * sizeof(ScoreItem));
+  p.off_vis = p.off_smerges + align_up(p.smerges.size() * sizeof(MergeItem));
   p.off_err = p.off_vis + align_up(p.vis.size() * sizeof(int32_t));   // zeroed by the upload
   p.staged = p.off_err + sizeof(int);
   p.off_cand = align_up(p.staged);
-  p.bytes = p.off_cand + align_up((size_t)p.cand_slots * Hq * kp * sizeof(uint64_t));
+  p.off_scand = p.off_cand + align_up((size_t)p.cand_slots * Hq * kp * sizeof(uint64_t));
+  p.off_seed = p.off_scand + align_up((size_t)p.scand_slots * Hq * kp * sizeof(uint64_t));
+  p.bytes = p.off_seed + (p.sitems.empty() ? 0 : align_up((size_t)Hq * T * sizeof(uint64_t)));
   return p;
+}
+
+// Score and merge the plan's items: the sample pass and its seed merge first when
+// the plan has seeded groups, then every split and the merge into idx / score.
+cudaError_t run_plan(ScoreArgs a, const Plan& p, char* ws, int dtype, int kp, cudaStream_t s) {
+  cudaError_t e;
+  a.seed = nullptr;
+  a.seed_out = nullptr;
+  a.sample = 0;
+  if (!p.sitems.empty()) {
+    ScoreArgs b = a;
+    b.items = reinterpret_cast<const ScoreItem*>(ws + p.off_sitems);
+    b.merges = reinterpret_cast<const MergeItem*>(ws + p.off_smerges);
+    b.n_items = (int32_t)p.sitems.size();
+    b.n_merges = (int32_t)p.smerges.size();
+    b.cand = reinterpret_cast<uint64_t*>(ws + p.off_scand);
+    b.cand_per_head = p.scand_slots;
+    b.idx = nullptr;
+    b.score = nullptr;
+    b.seed_out = reinterpret_cast<uint64_t*>(ws + p.off_seed);
+    b.sample = 1;
+    if ((e = launch_score_generic(b, dtype, kp, p.nq, s)) != cudaSuccess) return e;
+    if ((e = launch_merge(b, dtype, kp, s)) != cudaSuccess) return e;
+    a.seed = b.seed_out;
+  }
+  if ((e = launch_score_generic(a, dtype, kp, p.nq, s)) != cudaSuccess) return e;
+  return launch_merge(a, dtype, kp, s);
 }
 
 saki_status upload_plan(const Plan& p, char* ws, cudaStream_t s) {
@@ -253,6 +313,10 @@ saki_status upload_plan(const Plan& p, char* ws, cudaStream_t s) {
   if (!p.items.empty()) std::memcpy(host.data() + p.off_items, p.items.data(), p.items.size() * sizeof(ScoreItem));
   if (!p.merges.empty())
     std::memcpy(host.data() + p.off_merges, p.merges.data(), p.merges.size() * sizeof(MergeItem));
+  if (!p.sitems.empty())
+    std::memcpy(host.data() + p.off_sitems, p.sitems.data(), p.sitems.size() * sizeof(ScoreItem));
+  if (!p.smerges.empty())
+    std::memcpy(host.data() + p.off_smerges, p.smerges.data(), p.smerges.size() * sizeof(MergeItem));
   if (!p.vis.empty()) std::memcpy(host.data() + p.off_vis, p.vis.data(), p.vis.size() * sizeof(int32_t));
   return staging().upload(ws, host.data(), p.staged, s) == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA;
 }
@@ -440,7 +504,7 @@ size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout
       if (use_tc(cfg, layout, P))
         b = make_tc_plan(layout, cfg->num_q_heads, P, op == SAKI_OP_SCORE_TOPK).bytes;
       else
-        b = make_plan(layout, cfg->num_q_heads, kp_of(cfg->topk)).bytes;
+        b = make_plan(layout, cfg->num_q_heads, kp_of(cfg->topk), cfg->dtype, P).bytes;
       if (op == SAKI_OP_RECALL) b += recall_extra(cfg, layout->num_queries, true);
       return b;
     }
@@ -550,7 +614,7 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
     return run_tc(cfg, layout, tp, cfg->rank, false, Q, L, sketch, nu, idx, score, ws, s);
   }
   const int kp = kp_of(cfg->topk);
-  const Plan p = make_plan(layout, cfg->num_q_heads, kp);
+  const Plan p = make_plan(layout, cfg->num_q_heads, kp, cfg->dtype, cfg->rank);
   if (workspace_bytes < p.bytes) return SAKI_ERR_WORKSPACE;
   if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
   ScoreArgs a{};
@@ -568,8 +632,7 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
   a.n_items = (int32_t)p.items.size();
   a.n_merges = (int32_t)p.merges.size();
   KernelTimer kt(SAKI_KERNEL_SELECT, s);
-  if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, p.nq, s))) != SAKI_OK) return st;
-  return cuda_status(launch_merge(a, cfg->dtype, kp, s));
+  return cuda_status(run_plan(a, p, ws, cfg->dtype, kp, s));
 }
 
 saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64_t min_visible, const void* Q,
@@ -586,7 +649,7 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
     if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
   const int kp = kp_of(cfg->topk);
   const bool tc = use_tc(cfg, layout, kD);
-  const Plan p = tc ? Plan{} : make_plan(layout, cfg->num_q_heads, kp);
+  const Plan p = tc ? Plan{} : make_plan(layout, cfg->num_q_heads, kp, cfg->dtype, kD);
   const TcPlan tp = tc ? make_tc_plan(layout, cfg->num_q_heads, kD, false) : TcPlan{};
   const size_t base = tc ? tp.bytes : p.bytes;
   const size_t need = base + recall_extra(cfg, T, idx_exact == nullptr);
@@ -619,8 +682,7 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
     a.n_items = (int32_t)p.items.size();
     a.n_merges = (int32_t)p.merges.size();
     KernelTimer kt(SAKI_KERNEL_EXACT, s);
-    if ((st = cuda_status(launch_score_generic(a, cfg->dtype, kp, p.nq, s))) != SAKI_OK) return st;
-    if ((st = cuda_status(launch_merge(a, cfg->dtype, kp, s))) != SAKI_OK) return st;
+    if ((st = cuda_status(run_plan(a, p, ws, cfg->dtype, kp, s))) != SAKI_OK) return st;
   }
   const int32_t* vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
   return cuda_status(launch_recall(idx_approx, ie, vis, T, cfg->num_q_heads, cfg->topk, min_visible, counters,

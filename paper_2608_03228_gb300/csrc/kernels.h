@@ -50,7 +50,7 @@ struct ScoreItem {
   int64_t key_base;     // global row of the sequence's key 0
   int64_t cand;         // -1: write final lists; else candidate slot of (row 0, this split)
   int32_t cand_stride;  // slots between consecutive rows (= number of splits)
-  int32_t pad;
+  int32_t seeded;       // 1: start each query's threshold at ScoreArgs::seed of its row
 };
 
 // Merge of the per-split candidate lists of one query.
@@ -75,13 +75,18 @@ struct ScoreArgs {
   uint64_t* cand;       // candidate lists, kp keys per slot, per head: cand_per_head slots
   int64_t cand_per_head;
   int* err;             // zeroed workspace word; the tensor-core variant sets kStTimeout if a bounded wait gave up
+  const uint64_t* seed; // [Hq][T] per-row lower bound on the row's k-th best key (read by seeded items), or null
+  uint64_t* seed_out;   // merge only: write each merged row's k-th best key here instead of idx / score
   int64_t T, N;
   int32_t Hq, G, P, k, exact, n_items, n_merges;
+  int32_t sample;       // tensor-core variant only: write each query's kp best group maxima (a sample pass)
 };
 
 // generic CUDA-core scoring (any rank, f32 or bf16)
 // nq: query-group width of the launch (1, 2, 4 or 8), at least every item's q_count
 cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, cudaStream_t s);
+// true when launch_score_generic runs the tensor-core variant for these arguments
+bool decode_tc_eligible(int dtype, int P, int nq);
 cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s);
 size_t score_generic_smem(int P, int kp, int nq);
 

@@ -262,6 +262,16 @@ __global__ void __launch_bounds__(128) merge_kernel(const ScoreArgs a) {
     for (int e = 0; e < EK; ++e) other[e] = c[(int64_t)s * KP + e * 32 + lane];
     warp_merge_top<EK>(best, other);
   }
+  if (a.seed_out) {
+    // the row's k-th best key over the merged lists (0 while fewer than k)
+    uint64_t t = 0;
+#pragma unroll
+    for (int e = 0; e < EK; ++e)
+      if (e == (a.k - 1) >> 5) t = best[e];
+    t = shfl_u64(t, (a.k - 1) & 31);
+    if (lane == 0) a.seed_out[(int64_t)h * a.T + mi.t] = t;
+    return;
+  }
   float qnu = 0.f;
   if (a.nu) {
     const Tin* q = static_cast<const Tin*>(a.Q) + ((int64_t)h * a.T + mi.t) * kD;
@@ -286,10 +296,14 @@ __global__ void __launch_bounds__(128) merge_kernel(const ScoreArgs a) {
 // TMA), u = W^T q of the group's queries split into bf16 hi + lo the B operand
 // (N = 16, rows past the group zero), D[key][query] in a ring of TMEM
 // accumulators.  Each epilogue thread reads one key's scores for all queries (its
-// TMEM lane) and writes them to a shared [query][key] tile; each query then
-// belongs to one epilogue warp, which scans all 128 keys of the tile against
-// the query's running k-th best (score_generic_kernel's candidate buffer and
-// re-selection), so a query's threshold is built from every key of the split.
+// TMEM lane) into registers and compares them with its warp's running k-th best
+// of each query (score_generic_kernel's candidate buffer and re-selection, one
+// buffer per warp and query), one warp vote per tile for all queries; the four
+// warps' lists of a query are merged at the end.  A seeded item starts every
+// threshold at the row's seed, so after the first few keys almost no key is
+// appended.  With ScoreArgs::sample set, the kernel keeps per query the best
+// score each thread sees (a group maximum over the split) and writes the kp
+// largest of the CTA's 128 group maxima, from which the seeds are merged.
 // Roles: warp 0 TMA producer, warp 1 TMEM owner and MMA issuer, warps 2-5
 // projection and selection.  Every mbarrier wait is bounded; a CTA that gives
 // up sets kStTimeout in the error word.
@@ -308,10 +322,10 @@ struct DcCfg {
   static constexpr int U_PART = (NQ * P * 2 + 1023) & ~1023;   // u_hi or u_lo
   static constexpr int OFF_U = STAGES * STAGE_BYTES;
   static constexpr int OFF_BUF = OFF_U + 2 * U_PART;
-  static constexpr int cap(int kp) { return 4 * kp; }          // candidate slots per query
-  static constexpr int TS = 4;                                  // [query][key] score tiles in flight
-  static constexpr int off_t(int kp) { return OFF_BUF + kGroupQ * cap(kp) * 8; }   // [TS][query][key] scores
-  static int smem(int kp) { return off_t(kp) + TS * kGroupQ * NT * 4 + 1024; }
+  static constexpr int cap(int kp) { return 2 * kp; }          // candidate slots per warp and query
+  static constexpr int LANES = 4 * 32;                          // group maxima per query in a sample pass
+  static int smem(int kp) { return OFF_BUF + 4 * kGroupQ * cap(kp) * 8 + 1024; }   // [4 warps][query][cap]
+  static_assert(4 * cap(64) >= LANES, "a sample pass's group maxima fit the candidate buffers");
   static_assert(kGroupQ <= NQ && NQ % 16 == 0, "the group fits the MMA's N");
   static_assert(STAGE_BYTES % 1024 == 0 && OFF_U % 1024 == 0, "swizzled blocks on 1024-byte boundaries");
 };
@@ -350,15 +364,14 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
   uint8_t* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
   uint8_t* sStage = smem;
   uint8_t* sU = smem + C::OFF_U;
-  uint64_t* buf = reinterpret_cast<uint64_t*>(smem + C::OFF_BUF);   // [GQ][CAP]
-  float* tile_s = reinterpret_cast<float*>(smem + C::off_t(KP));    // [TS][GQ][NT]
+  uint64_t* buf = reinterpret_cast<uint64_t*>(smem + C::OFF_BUF);   // [4 warps][GQ][CAP]
   __shared__ float qs[GQ][kD];
   __shared__ float us[GQ][P];
   __shared__ float qnu[GQ];
   __shared__ int visq[GQ];
-  __shared__ int cnt_s[GQ];
+  __shared__ int cnt_s[4 * GQ];
   __shared__ unsigned long long cta_thr[GQ];
-  __shared__ __align__(8) uint64_t bars[2 * C::STAGES + 2 * C::NB + 2 + 2 * C::TS];
+  __shared__ __align__(8) uint64_t bars[2 * C::STAGES + 2 * C::NB + 2];
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_s;
   uint64_t* full = bars;
@@ -367,8 +380,6 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
   uint64_t* acce = accf + C::NB;
   uint64_t* uready = acce + C::NB;
   uint64_t* drain = uready + 1;
-  uint64_t* tfull = drain + 1;      // [TS] a score tile written by all four epilogue warps
-  uint64_t* tempty = tfull + C::TS;  // [TS] its queries read by all four
   volatile int* abort_f = &abort_s;
 
   const ScoreItem it = a.items[blockIdx.x];
@@ -389,10 +400,6 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
     }
     tc::mbar_init(uready, 128);
     tc::mbar_init(drain, 1);
-    for (int t = 0; t < C::TS; ++t) {
-      tc::mbar_init(tfull + t, 128);
-      tc::mbar_init(tempty + t, 128);
-    }
     *abort_f = 0;
     tc::fence_barrier_init();
   }
@@ -472,8 +479,8 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
       visq[et] = et < nq ? a.vis[it.q_begin + et] : 0;
       cta_thr[et] = 0ull;
     }
-    if (et < GQ) cnt_s[et] = 0;
-    for (int o = et; o < GQ * CAP; o += 128) buf[o] = 0ull;
+    if (et < 4 * GQ) cnt_s[et] = 0;
+    for (int o = et; o < 4 * GQ * CAP; o += 128) buf[o] = 0ull;
     epilogue_sync();
     // u_b = W_h^T q_b (fp32) and the mean term q_b^T nu_h
     const float* W = a.W + (int64_t)h * kD * P;
@@ -508,89 +515,137 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
     tc::fence_proxy_async_smem();
     tc::mbar_arrive(uready);
 
-    // this warp's queries are e and e + 4
-    uint64_t thr[2] = {0ull, 0ull};
-    float thr_f[2] = {-INFINITY, -INFINITY};   // score part of thr: a key can only pass if its score is >= thr_f
+    // Each thread owns one key of every tile (its TMEM lane) and holds that
+    // key's scores for all queries of the group in registers: one compare per
+    // query against the warp's running threshold and one warp vote per tile.
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
-    // Scores pass through a ring of TS shared [query][key] tiles: every warp
-    // writes its quarter of the keys of tile i and reads all keys of its own
-    // queries, with mbarriers between writers and readers so that the warps can
-    // drift up to TS - 1 tiles apart (a warp whose queries take many appends on
-    // one tile no longer holds the others).  All waits are bounded.
-    bool ok = true;
-    for (int i = 0; i < ntiles && ok; ++i) {
-      const int b = i % C::NB, ts = i % C::TS;
-      const uint32_t tph = (i / C::TS) & 1;
-      float* T = tile_s + ts * GQ * C::NT;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f) &&
-                                       tc::mbar_wait(tempty + ts, tph ^ 1, abort_f));
-      if (!ok) break;
-      tc::fence_after_sync();
-      uint32_t r[16];
-      __syncwarp();
-      tc::tmem_ld16(tl + b * C::NQ, r);
-      tc::tmem_ld_wait(r);
-      tc::fence_before_sync();
-      tc::mbar_arrive(acce + b);
+    int lim[GQ];   // keys of the split visible to query q (0 past the group)
+    int lim_min = nkeys;
+#pragma unroll
+    for (int q = 0; q < GQ; ++q) {
+      lim[q] = q < nq ? max(0, min(nkeys, visq[q] - it.key_lo)) : 0;
+      if (q < nq) lim_min = min(lim_min, lim[q]);
+    }
+    if (a.sample) {
+      // Sample pass: per query, the best score each thread sees over the split
+      // (a group of up to ntiles keys, one per tile).  The k-th largest group
+      // maximum over all splits is reached by k distinct visible keys, so it
+      // bounds the row's k-th best score from below.
+      float mx[GQ];
+#pragma unroll
+      for (int q = 0; q < GQ; ++q) mx[q] = -INFINITY;
+      for (int i = 0; i < ntiles; ++i) {
+        const int b = i % C::NB;
+        if (!__all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f))) break;
+        tc::fence_after_sync();
+        uint32_t r[8];
+        __syncwarp();
+        tc::tmem_ld8(tl + b * C::NQ, r);
+        tc::tmem_ld_wait(r);
+        tc::fence_before_sync();
+        tc::mbar_arrive(acce + b);
+        const int jl = i * C::NT + quarter * 32 + lane;
+#pragma unroll
+        for (int q = 0; q < GQ; ++q)
+          if (jl < lim[q]) mx[q] = fmaxf(mx[q], __uint_as_float(r[q]));
+      }
+      uint64_t* gm = buf;   // [GQ][LANES] group maxima as keys (0: the thread saw no visible key)
 #pragma unroll
       for (int q = 0; q < GQ; ++q)
-        if (q < nq) T[q * C::NT + quarter * 32 + lane] = __uint_as_float(r[q]);
-      tc::mbar_arrive(tfull + ts);   // release: the tile's quarter is written
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(tfull + ts, tph, abort_f));
-      if (!ok) break;
+        gm[q * C::LANES + quarter * 32 + lane] =
+            mx[q] > -INFINITY ? make_key(mx[q], (uint32_t)(it.key_lo + quarter * 32 + lane)) : 0ull;
+      epilogue_sync();
+      for (int q = e; q < nq; q += 4) {
+        int c = C::LANES;
+        reselect<KP, C::LANES>(gm + q * C::LANES, c, a.k);
+        uint64_t* c2 = a.cand + ((int64_t)h * a.cand_per_head + it.cand + (int64_t)q * it.cand_stride) * KP;
 #pragma unroll
-      for (int x = 0; x < 2; ++x) {
-        const int q = e + 4 * x;
-        if (q < nq) {
-          const float4 v4 = reinterpret_cast<const float4*>(T + q * C::NT)[lane];   // keys 4 lane .. 4 lane + 3
-          const float sv[4] = {v4.x, v4.y, v4.z, v4.w};
-          const int jl0 = i * C::NT + 4 * lane;
-          unsigned m = 0u;
+        for (int y = 0; y < EK; ++y) c2[y * 32 + lane] = gm[q * C::LANES + y * 32 + lane];
+      }
+    } else {
+      // a seeded item starts each query at its row's seed score: at least k
+      // visible keys of the row score that much, so every key of the row's
+      // top k still passes
+      uint64_t thr[GQ];
+      float thr_f[GQ];   // score part of thr: a key can only pass if its score is >= thr_f
 #pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            const bool ok = jl0 + t < nkeys && it.key_lo + jl0 + t < visq[q] && sv[t] >= thr_f[x];
-            m |= ok ? 1u << t : 0u;
-          }
-          const unsigned any = __reduce_or_sync(0xffffffffu, m);
+      for (int q = 0; q < GQ; ++q) {
+        thr[q] = 0ull;
+        thr_f[q] = q < nq ? -INFINITY : INFINITY;
+        const uint64_t sd = it.seeded && a.seed && q < nq ? a.seed[(int64_t)h * a.T + it.q_begin + q] : 0ull;
+        if (sd >> 32) {
+          thr[q] = (sd & 0xffffffff00000000ull) - 1ull;
+          thr_f[q] = key_score(sd);
+        }
+      }
+      uint64_t* wbuf = buf + e * GQ * CAP;
+      int* wcnt = cnt_s + e * GQ;
+      for (int i = 0; i < ntiles; ++i) {
+        const int b = i % C::NB;
+        if (!__all_sync(0xffffffffu, tc::mbar_wait(accf + b, (i / C::NB) & 1, abort_f))) break;
+        tc::fence_after_sync();
+        uint32_t r[8];
+        __syncwarp();
+        tc::tmem_ld8(tl + b * C::NQ, r);
+        tc::tmem_ld_wait(r);
+        tc::fence_before_sync();
+        tc::mbar_arrive(acce + b);
+        const int jl = i * C::NT + quarter * 32 + lane;
+        // one bit per query whose score clears its threshold; one vote for all
+        const bool inner = (i + 1) * C::NT <= lim_min;   // every key of the tile visible to every query
+        unsigned m = 0u;
 #pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            if (any & (1u << t)) {
-              const uint64_t key = make_key(sv[t], (uint32_t)(it.key_lo + jl0 + t));
-              const bool pass = ((m >> t) & 1u) && key > thr[x];
+        for (int q = 0; q < GQ; ++q) {
+          const bool ok = __uint_as_float(r[q]) >= thr_f[q] && (inner || jl < lim[q]);
+          m |= ok ? 1u << q : 0u;
+        }
+        const unsigned any = __reduce_or_sync(0xffffffffu, m);
+        if (any) {
+          const uint32_t j = (uint32_t)(it.key_lo + jl);
+#pragma unroll
+          for (int q = 0; q < GQ; ++q) {
+            if (any & (1u << q)) {
+              const uint64_t key = make_key(__uint_as_float(r[q]), j);
+              const bool pass = ((m >> q) & 1u) && key > thr[q];
               const unsigned mask = __ballot_sync(0xffffffffu, pass);
               if (mask) {
-                thr[x] = append_keys<KP, CAP>(buf + q * CAP, cnt_s + q, cta_thr + q, key, pass, mask, thr[x], a.k);
-                thr_f[x] = key_score(thr[x]);
+                thr[q] = append_keys<KP, CAP>(wbuf + q * CAP, wcnt + q, cta_thr + q, key, pass, mask, thr[q], a.k);
+                thr_f[q] = key_score(thr[q]);
               }
             }
           }
         }
       }
-      tc::mbar_arrive(tempty + ts);   // this warp has read its queries of the tile
-    }
-    // each query's k best, from its owner warp
-    for (int x = 0; x < 2; ++x) {
-      const int q = e + 4 * x;
-      if (q >= nq) continue;
-      int c = cnt_s[q];
-      reselect<KP, CAP>(buf + q * CAP, c, a.k);
-      uint64_t best[EK];
+      for (int q = 0; q < nq; ++q) {
+        int c = wcnt[q];
+        reselect<KP, CAP>(wbuf + q * CAP, c, a.k);
+      }
+      epilogue_sync();
+      // each query's k best: the four warps' sorted lists merged by one warp
+      for (int q = e; q < nq; q += 4) {
+        uint64_t best[EK], other[EK];
 #pragma unroll
-      for (int y = 0; y < EK; ++y) best[y] = buf[q * CAP + y * 32 + lane];
-      if (it.cand < 0) {
-        const int64_t row = ((int64_t)h * a.T + it.q_begin + q) * a.k;
+        for (int y = 0; y < EK; ++y) best[y] = buf[q * CAP + y * 32 + lane];
+        for (int w2 = 1; w2 < 4; ++w2) {
 #pragma unroll
-        for (int y = 0; y < EK; ++y) {
-          const int ii = y * 32 + lane;
-          if (ii < a.k) {
-            a.idx[row + ii] = key_index(best[y]);
-            if (a.score) a.score[row + ii] = best[y] ? key_score(best[y]) + qnu[q] : -INFINITY;
-          }
+          for (int y = 0; y < EK; ++y) other[y] = buf[(w2 * GQ + q) * CAP + y * 32 + lane];
+          warp_merge_top<EK>(best, other);
         }
-      } else {
-        uint64_t* c2 = a.cand + ((int64_t)h * a.cand_per_head + it.cand + (int64_t)q * it.cand_stride) * KP;
+        if (it.cand < 0) {
+          const int64_t row = ((int64_t)h * a.T + it.q_begin + q) * a.k;
 #pragma unroll
-        for (int y = 0; y < EK; ++y) c2[y * 32 + lane] = best[y];
+          for (int y = 0; y < EK; ++y) {
+            const int ii = y * 32 + lane;
+            if (ii < a.k) {
+              a.idx[row + ii] = key_index(best[y]);
+              if (a.score) a.score[row + ii] = best[y] ? key_score(best[y]) + qnu[q] : -INFINITY;
+            }
+          }
+        } else {
+          uint64_t* c2 = a.cand + ((int64_t)h * a.cand_per_head + it.cand + (int64_t)q * it.cand_stride) * KP;
+#pragma unroll
+          for (int y = 0; y < EK; ++y) c2[y * 32 + lane] = best[y];
+        }
       }
     }
   }
@@ -657,12 +712,16 @@ cudaError_t launch_nq(const ScoreArgs& a, int nq, cudaStream_t s) {
 }
 }  // namespace
 
+// bf16 keys or codes of a tensor-core width, in groups of at least four
+// queries, take the tensor-core variant (with one query per group the CUDA-core
+// kernel streams a decode step faster: 0.50 against 0.53 ms over 32 heads x 1M keys)
+bool decode_tc_eligible(int dtype, int P, int nq) {
+  return dtype == SAKI_BF16 && nq >= 4 && (P == 16 || P == 32 || P == 64 || P == 128);
+}
+
 cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, cudaStream_t s) {
   if (a.n_items == 0) return cudaSuccess;
-  // bf16 keys or codes of a tensor-core width, in groups of at least four
-  // queries, take the tensor-core variant (with one query per group the CUDA-core
-  // kernel streams a decode step faster: 0.50 against 0.53 ms over 32 heads x 1M keys)
-  if (dtype == SAKI_BF16 && a.err && nq >= 4 && (a.P == 16 || a.P == 32 || a.P == 64 || a.P == 128))
+  if (a.err && decode_tc_eligible(dtype, a.P, nq))
     return kp == 64 ? launch_decode_tc<64>(a, s) : launch_decode_tc<128>(a, s);
   if (dtype == SAKI_BF16)
     return kp == 64 ? launch_nq<__nv_bfloat16, 64>(a, nq, s) : launch_nq<__nv_bfloat16, 128>(a, nq, s);

@@ -232,6 +232,79 @@ def test_score_topk_layouts(lib, case):
     _score_case(lib, Hq, Hk, r, k, dtype, lens, queries, seed=int(sum(lens)) % 1000 + r)
 
 
+# A group whose keys are cut into eight or more splits is seeded: a sample pass
+# over the head of every split, merged per query, starts every split's threshold
+# at a score that at least k visible keys reach.  Mixed visibility covers rows
+# seeing exactly k, k + 1, k - 1 and no keys, and a second, unsplit sequence.
+@pytest.mark.parametrize("case", [
+    (4, 1, 32, 64, "bf16", (20000,), ([-1, 19999, 5000, 300, 64, 65, 63, 0],)),
+    (2, 2, 128, 100, "bf16", (30000,), ([-1] * 5,)),                        # r = d, k > 64
+    (4, 2, 16, 64, "bf16", (18000, 500), ([-1] * 4, [-1] * 4)),
+])
+def test_score_topk_seeded_decode(lib, case):
+    Hq, Hk, r, k, dtype, lens, queries = case
+    before = lib.saki_launch_count()
+    _score_case(lib, Hq, Hk, r, k, dtype, lens, queries, seed=int(sum(lens)) % 1000 + r)
+    # plan upload, sample pass, seed merge, main pass, merge
+    assert lib.saki_launch_count() - before == 5
+
+
+def test_score_topk_seeded_decode_ties(lib):
+    """Integer scores full of exact ties on the seeded path: the seed is a key
+    (score and index), so the lower-index rule must survive it exactly."""
+    torch = _torch()
+    Hq, Hk, r, k = 2, 1, 32, 64
+    rng = np.random.default_rng(19)
+    off, q_seq, q_vis = _layout_arrays((20000,), ([-1, 15000, 9000, 2047],))
+    T, N = len(q_seq), int(off[-1])
+    Q = np.zeros((Hq, T, D), np.float32)
+    Q[:, np.arange(T), np.arange(T) % D] = 1.0                  # one-hot queries: u = row of L
+    L = rng.integers(-1, 2, (Hq, D, r)).astype(np.float32)
+    sk = rng.integers(-2, 3, (Hq, N, r)).astype(np.float32)    # integer scores in [-64, 64]
+    cfg = lib.make_config(Hq, Hk, r, k, "bf16", flags=1)
+    lay = lib.HostLayout(off, q_seq, q_vis)
+    idx = torch.empty((Hq, T, k), dtype=torch.int32, device="cuda")
+    lib.saki_score_topk(cfg, lay, to_dev(Q, "bf16"), f32(L), to_dev(sk, "bf16"), idx)
+    idx = idx.cpu().numpy()
+    for h in range(Hq):
+        for t in range(T):
+            ref, _ = O.topk(O.approx_scores(Q[h, t], L[h], sk[h, :q_vis[t]]), k)
+            np.testing.assert_array_equal(idx[h, t], ref, err_msg=f"h{h} t{t}")
+
+
+def test_recall_seeded_decode(lib):
+    """Exact top-k through saki_recall on a seeded decode layout (keys as the
+    tensor-core operand, four query heads per KV head) and the head recall."""
+    torch = _torch()
+    Hq, Hk, r, k = 4, 1, 32, 64
+    rng = np.random.default_rng(23)
+    off, q_seq, q_vis = _layout_arrays((24000,), ([-1, -1, 20000, 3000, 65, 64],))
+    T, N = len(q_seq), int(off[-1])
+    Q = synth.round_to_bf16_grid(rng.standard_normal((Hq, T, D)).astype(np.float32))
+    K = synth.round_to_bf16_grid(rng.standard_normal((Hk, N, D)).astype(np.float32))
+    A = (rng.standard_normal((Hq, D, D)) / np.sqrt(D)).astype(np.float32)
+    ia = np.stack([np.stack([O.topk(rng.standard_normal(int(q_vis[t])), k)[0] for t in range(T)])
+                   for _ in range(Hq)]).astype(np.int32)
+    cfg = lib.make_config(Hq, Hk, r, k, "bf16", flags=1)
+    lay = lib.HostLayout(off, q_seq, q_vis)
+    ie = torch.empty((Hq, T, k), dtype=torch.int32, device="cuda")
+    rec = torch.empty((Hq,), device="cuda")
+    before = lib.saki_launch_count()
+    lib.saki_recall(cfg, lay, k + 1, to_dev(Q, "bf16"), f32(A), to_dev(K, "bf16"), torch.from_numpy(ia).cuda(), rec,
+                    idx_exact=ie)
+    # plan upload, sample pass, seed merge, main pass, merge, recall and its finish
+    assert lib.saki_launch_count() - before == 7
+    ie = ie.cpu().numpy()
+    waived = 0
+    for h in range(Hq):
+        rows = [O.exact_scores(Q[h, t], A[h], K[h // (Hq // Hk), :q_vis[t]]) for t in range(T)]
+        waived += check_topk_rows(ie[h], rows, k, label=f"exact h{h}")[1]
+    ref_ie = np.stack([np.stack([O.topk(O.exact_scores(Q[h, t], A[h], K[0, :q_vis[t]]), k)[0] for t in range(T)])
+                       for h in range(Hq)])
+    ref_rec = O.head_recall(ia, ref_ie, q_vis, k + 1, k)
+    np.testing.assert_allclose(rec.cpu().numpy(), ref_rec, atol=RECALL_ABS + waived / (k * T))
+
+
 def test_score_topk_mean_term(lib):
     _score_case(lib, 4, 1, 32, 64, "bf16", (700,), ([-1, 300],), center=1)
 
