@@ -376,12 +376,31 @@ def rooflines(w, pk, ktime, g):
                      "peak_source": f"{pk['source']} ({peak_name})", "model": note}
 
     alu = pk["alu_tops"]
-    entry("select", "alu", pairs, "Tops/s", alu,
-          "one threshold comparison per visible (head, query, key) pair; the scores come from a tensor-core "
-          f"contraction of 2r = {2 * r} flop per pair", "152 SMs x 128 lanes x max SM clock")
-    entry("exact", "alu", pairs, "Tops/s", alu,
-          "one comparison per visible pair; scores q^T A k from a tensor-core contraction of 2d flop per pair",
-          "152 SMs x 128 lanes x max SM clock")
+    # A selection has two floors: its bytes (queries, codes or keys and the
+    # projection read once, indices written) at the copy bandwidth, and one
+    # threshold comparison per visible pair at the lane rate (the scores come from
+    # the tensor core, far below its peak).  The larger floor is the bound: the
+    # bytes for decode-shaped calls (few queries over many keys), and for the
+    # batched causal workloads too, where the query and index bytes alone exceed
+    # the comparisons.
+    io = Hq * T * D * eb + Hq * T * w.topk * 4
+
+    def selection(name, nbytes, what):
+        t_hbm = nbytes / (pk["hbm_gbs"] * 1e9)
+        t_alu = pairs / (alu * 1e12)
+        if t_hbm >= t_alu:
+            entry(name, "hbm", nbytes, "GB/s", pk["hbm_gbs"],
+                  f"queries, {what} read once, indices written (the comparison floor, one per visible pair at "
+                  f"the lane rate, is lower)", "STREAM copy")
+        else:
+            entry(name, "alu", pairs, "Tops/s", alu,
+                  f"one threshold comparison per visible (head, query, key) pair (the byte floor, queries, {what} "
+                  f"read once, is lower)", "152 SMs x 128 lanes x max SM clock")
+        if name in out:
+            out[name]["floors_ms"] = {"hbm": t_hbm * 1e3, "alu": t_alu * 1e3}
+
+    selection("select", io + Hq * N * r * eb + Hq * D * r * 4, f"rank-{r} codes and L")
+    selection("exact", io + Hk * N * D * eb + Hq * D * D * 4, "keys and A")
     entry("moments", "hbm", (Hq + Hk) * n * D * eb + (Hq + Hk) * D * D * 4, "GB/s", pk["hbm_gbs"],
           "calibration queries and keys read once, fp32 moment matrices written", "STREAM copy")
     entry("build", "hbm", Hk * N * D * eb + Hq * N * r * eb, "GB/s", pk["hbm_gbs"],
