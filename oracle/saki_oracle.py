@@ -23,6 +23,9 @@ What it follows (sections and equations of arXiv 2608.03228, "SAKI"):
   ``c_j = R^T (k_j - mu)``; score ``s_hat = (L^T q)^T c_j + q^T A mu``.
 * Sec. 3 protocol: recall of the true top-k attended positions, i.e. the
   fraction of the exact top-k set (by ``q^T A k``) found by the index.
+* Tab. 1 / Sec. 4 comparison indexes: key PCA (the rank-r principal
+  projector of the keys, M = A P) and weight SVD (the operator's truncated
+  SVD, M = A_r).
 
 Readings where the paper is silent (each also listed in the design doc):
 
@@ -137,6 +140,60 @@ def fit(q_calib, k_calib, A, rank: int, center: bool, floor_rel: float = 1e-6) -
         out["nu"].append(np.asarray(A[h], F64) @ mu[g])
     res = {k: np.array(v) for k, v in out.items()}
     res.update(mu=np.array(mu), Sq=np.array(Sq), Sk=np.array(Sk))
+    return res
+
+
+# --------------------------------------------------------------------------
+# Tab. 1 comparison indexes: key PCA and weight SVD
+# --------------------------------------------------------------------------
+def key_pca_head(Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
+    """Key PCA for one head (Tab. 1; Sec. 4 states that PCA minimises
+    ``||(I - P) Sk^{1/2}||_F^2``): P = V_r V_r^T projects onto the r leading
+    eigenvectors of the key moment Sk, the score map is M = A P, and the
+    factors are L = A V_r, R = V_r, so a key's code is its principal
+    coordinates.  sigma are the square roots of Sk's eigenvalues (descending,
+    the App. A floor applied) and loss is the discarded key energy
+    ``sum_{i>r} lambda_i(Sk)``.  Directions whose eigenvalue is floored are
+    left out (zero columns)."""
+    lam, V = np.linalg.eigh(0.5 * (np.asarray(Sk, F64) + np.asarray(Sk, F64).T))
+    order = np.argsort(-lam, kind="stable")
+    lam, V = lam[order], V[:, order]
+    lmax = lam[0] if lam.size else 0.0
+    lam = np.where((lam > 0) & (lam >= floor_rel * lmax), lam, 0.0)
+    R = V[:, :r] * (lam[:r] > 0)
+    L = np.asarray(A, F64) @ R
+    L, R = canonical_signs(L, R)
+    return dict(L=L, R=R, M=L @ R.T, sigma=np.sqrt(lam), loss=float(np.sum(lam[r:])))
+
+
+def weight_svd_head(A, r: int) -> dict:
+    """Weight SVD for one head (Tab. 1; Sec. 4 (b)): the operator's own
+    truncated SVD, blind to the data.  A = U Sigma V^T, L = U_r Sigma_r^{1/2},
+    R = V_r Sigma_r^{1/2}, M = A_r; loss = ``sum_{i>r} sigma_i(A)^2``."""
+    U, sig, Vt = np.linalg.svd(np.asarray(A, F64))
+    sh = np.sqrt(sig[:r])
+    L, R = canonical_signs(U[:, :r] * sh, Vt[:r].T * sh)
+    return dict(L=L, R=R, M=(U[:, :r] * sig[:r]) @ Vt[:r], sigma=sig, loss=float(np.sum(sig[r:] ** 2)))
+
+
+def fit_baseline(method: str, k_calib, A, rank: int, center: bool, num_q_heads: int,
+                 floor_rel: float = 1e-6) -> dict:
+    """All heads of a comparison index, ``method`` "key_pca" or "weight_svd";
+    the keys' moments and means follow the same centering reading as ``fit``
+    (the mean term nu = A_h mu_g is unchanged).  Returns L, R, M, sigma, loss,
+    mu, nu like ``fit``."""
+    Hq, Hk = num_q_heads, len(k_calib)
+    G = Hq // Hk
+    Sk, mu = zip(*[moments(k_calib[g], center) for g in range(Hk)])
+    out = {k: [] for k in ("L", "R", "M", "sigma", "loss", "nu")}
+    for h in range(Hq):
+        g = h // G
+        res = key_pca_head(Sk[g], A[h], rank, floor_rel) if method == "key_pca" else weight_svd_head(A[h], rank)
+        for k in ("L", "R", "M", "sigma", "loss"):
+            out[k].append(res[k])
+        out["nu"].append(np.asarray(A[h], F64) @ mu[g])
+    res = {k: np.array(v) for k, v in out.items()}
+    res.update(mu=np.array(mu), Sk=np.array(Sk))
     return res
 
 

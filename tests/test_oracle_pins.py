@@ -51,13 +51,14 @@ def test_hand_examples(name):
         M = res["M"]
         np.testing.assert_allclose(M @ M, g["M_squared_over_M"] * M, atol=1e-12)
     if "pca_loss" in g:
-        lam, V = np.linalg.eigh(np.array(g["Sk"]))
-        P = np.outer(V[:, -1], V[:, -1])
-        assert abs(O.score_loss(np.array(g["A"]) @ P, g["A"], g["Sq"], g["Sk"]) - g["pca_loss"]) < 1e-12
+        pca = O.key_pca_head(np.array(g["Sk"]), np.array(g["A"]), g["r"])
+        assert abs(O.score_loss(pca["M"], g["A"], g["Sq"], g["Sk"]) - g["pca_loss"]) < 1e-12
     if "weight_svd_loss" in g:
-        U, s, Vt = np.linalg.svd(np.array(g["A"]))
-        W = s[0] * np.outer(U[:, 0], Vt[0])
-        assert abs(O.score_loss(W, g["A"], g["Sq"], g["Sk"]) - g["weight_svd_loss"]) < 1e-12
+        wsvd = O.weight_svd_head(np.array(g["A"]), g["r"])
+        assert abs(O.score_loss(wsvd["M"], g["A"], g["Sq"], g["Sk"]) - g["weight_svd_loss"]) < 1e-12
+    if np.allclose(g["Sq"], np.eye(len(g["A"]))) and np.allclose(g["Sk"], np.eye(len(g["A"]))):
+        # identity moments: the weight SVD is the optimum itself (Eckart-Young)
+        np.testing.assert_allclose(O.weight_svd_head(np.array(g["A"]), g["r"])["M"], g["M"], atol=1e-12)
 
 
 # ------------------------------------------------------- Prop. 1 identities
@@ -95,11 +96,8 @@ def test_saki_never_loses_to_key_pca_or_weight_svd(r):
     for seed in range(3):
         Sq, Sk, A = _case(seed=seed)
         res = O.fit_head(Sq, Sk, A, r)
-        lam, V = np.linalg.eigh(Sk)
-        Vr = V[:, ::-1][:, :r]
-        pca = O.score_loss(A @ Vr @ Vr.T, A, Sq, Sk)
-        U, s, Vt = np.linalg.svd(A)
-        wsvd = O.score_loss((U[:, :r] * s[:r]) @ Vt[:r], A, Sq, Sk)
+        pca = O.score_loss(O.key_pca_head(Sk, A, r)["M"], A, Sq, Sk)
+        wsvd = O.score_loss(O.weight_svd_head(A, r)["M"], A, Sq, Sk)
         assert res["loss"] <= pca * (1 + 1e-12)
         assert res["loss"] <= wsvd * (1 + 1e-12)
 
@@ -311,3 +309,82 @@ def test_predicted_mse_reduction_matches_independent_draws():
     # relative std of a mean of squared Gaussian bilinear forms is ~3/sqrt(n)
     tol = 5 * 3 / math.sqrt(n) * (1 - pred + 0.05)
     assert abs(meas - pred) < tol, (meas, pred, tol)
+
+
+# ------------------------------------------------- comparison indexes (Tab. 1)
+def _rotation(d, seed):
+    """An orthogonal matrix built from Givens rotations by fixed angles (no
+    factorisation routine involved)."""
+    Q = np.eye(d)
+    rng = np.random.default_rng(seed)
+    for i in range(d - 1):
+        for j in range(i + 1, d):
+            t = rng.uniform(0, 2 * np.pi)
+            G = np.eye(d)
+            G[i, i] = G[j, j] = np.cos(t)
+            G[i, j], G[j, i] = -np.sin(t), np.sin(t)
+            Q = Q @ G
+    return Q
+
+
+def test_weight_svd_closed_form():
+    """A = Q1 diag(4, 3, 2, 1) Q2^T: the rank-2 weight SVD keeps Q1 diag(4, 3, 0, 0)
+    Q2^T, sigma = (4, 3, 2, 1), loss = 2^2 + 1^2 = 5, and L R^T = M."""
+    Q1, Q2 = _rotation(4, 1), _rotation(4, 2)
+    A = Q1 @ np.diag([4.0, 3.0, 2.0, 1.0]) @ Q2.T
+    res = O.weight_svd_head(A, 2)
+    np.testing.assert_allclose(res["M"], Q1 @ np.diag([4.0, 3.0, 0.0, 0.0]) @ Q2.T, atol=1e-12)
+    np.testing.assert_allclose(res["sigma"], [4.0, 3.0, 2.0, 1.0], atol=1e-12)
+    assert abs(res["loss"] - 5.0) < 1e-12
+    np.testing.assert_allclose(res["L"] @ res["R"].T, res["M"], atol=1e-12)
+    # each R column is sqrt(sigma) times a unit right singular vector
+    np.testing.assert_allclose(np.sum(res["R"] ** 2, axis=0), [4.0, 3.0], atol=1e-12)
+
+
+def test_key_pca_closed_form():
+    """Sk = Q diag(9, 4, 1, 1/4) Q^T: rank-2 key PCA keeps the first two columns
+    of Q (R R^T = Q_2 Q_2^T, R orthonormal), L = A R, sigma = (3, 2, 1, 1/2),
+    loss = 1 + 1/4."""
+    Q = _rotation(4, 3)
+    Sk = Q @ np.diag([9.0, 4.0, 1.0, 0.25]) @ Q.T
+    A = _rotation(4, 4) @ np.diag([2.0, 1.0, 0.5, 0.1])
+    res = O.key_pca_head(Sk, A, 2)
+    np.testing.assert_allclose(res["R"] @ res["R"].T, Q[:, :2] @ Q[:, :2].T, atol=1e-12)
+    np.testing.assert_allclose(res["R"].T @ res["R"], np.eye(2), atol=1e-12)
+    np.testing.assert_allclose(res["L"], A @ res["R"], atol=1e-12)
+    np.testing.assert_allclose(res["M"], A @ Q[:, :2] @ Q[:, :2].T, atol=1e-12)
+    np.testing.assert_allclose(res["sigma"], [3.0, 2.0, 1.0, 0.5], atol=1e-12)
+    assert abs(res["loss"] - 1.25) < 1e-12
+
+
+def test_key_pca_drops_floored_directions():
+    """App. A floor: an eigenvalue below 1e-6 lambda_max counts as zero, so a
+    rank-3 key PCA of a rank-2 moment keeps two directions."""
+    Sk = np.diag([1.0, 0.5, 1e-9, 0.0])
+    res = O.key_pca_head(Sk, np.eye(4), 3)
+    np.testing.assert_allclose(res["M"], np.diag([1.0, 1.0, 0.0, 0.0]), atol=1e-15)
+    np.testing.assert_allclose(res["sigma"], [1.0, np.sqrt(0.5), 0.0, 0.0], atol=1e-15)
+
+
+def test_baselines_from_calibration_keys():
+    """fit_baseline on keys whose centered moment is diagonal by construction
+    (rows mu +- sqrt(n lambda_i / 2) e_i): key PCA picks the largest-variance
+    axes, nu = A mu; weight SVD ignores the data entirely."""
+    d, n = 6, 12
+    lam = np.array([0.5, 3.0, 0.25, 2.0, 1.0, 0.1])
+    mu = np.arange(1.0, d + 1.0)
+    K = np.tile(mu, (n, 1))
+    for i in range(d):
+        K[2 * i] += np.sqrt(n * lam[i] / 2) * np.eye(d)[i]
+        K[2 * i + 1] -= np.sqrt(n * lam[i] / 2) * np.eye(d)[i]
+    A = np.stack([_rotation(d, 5), _rotation(d, 6)])
+    res = O.fit_baseline("key_pca", K[None], A, 2, True, 2)
+    P = np.zeros((d, d))
+    P[1, 1] = P[3, 3] = 1.0
+    for h in range(2):
+        np.testing.assert_allclose(res["M"][h], A[h] @ P, atol=1e-12)
+        np.testing.assert_allclose(res["nu"][h], A[h] @ mu, atol=1e-12)
+    np.testing.assert_allclose(res["mu"][0], mu, atol=1e-12)
+    a = O.fit_baseline("weight_svd", K[None], A, 2, True, 2)
+    b = O.fit_baseline("weight_svd", 2.0 * K[None] + 1.0, A, 2, True, 2)
+    np.testing.assert_allclose(a["M"], b["M"], atol=1e-15)
