@@ -158,6 +158,23 @@ class GpuPath:
         if ev[4] is not None:
             ev[4].record()
 
+    def recall_with(self, method):
+        """Median recall of a Tab. 1 comparison index (key PCA, weight SVD) on the
+        same data through the same calls (untimed; overwrites the step's index,
+        selections and recall)."""
+        S, d, w, torch = self.saki, self.data, self.w, self.torch
+        cfg = S.make_config(w.num_q_heads, w.num_kv_heads, w.rank, w.topk, w.dtype, center=w.center, method=method)
+        need = S.saki_workspace_size(cfg, S.SAKI_OP_FIT, n_calib=w.n_calib)
+        ws = self.ws if need <= self.ws.numel() else torch.empty(need, device=self.dev, dtype=torch.uint8)
+        L, R = torch.empty_like(self.L), torch.empty_like(self.R)
+        S.saki_fit(cfg, d["q_calib"], d["k_calib"], d["A"], L, R, mu=self.mu, nu=self.nu, workspace=ws)
+        del ws
+        S.saki_build_index(cfg, d["K"], R, self.sketch, mu=self.mu, workspace=self.ws)
+        S.saki_score_topk(cfg, self.lay, d["Q"], L, self.sketch, self.idx, workspace=self.ws)
+        S.saki_recall(cfg, self.lay, w.topk + 1, d["Q"], d["A"], d["K"], self.idx, self.recall,
+                      idx_exact=self.idx_exact, workspace=self.ws)
+        return float(np.median(self.recall.cpu().numpy()))
+
 
 
 # kernel kinds timed inside the library (saki_kernel_timer_*)
@@ -253,6 +270,9 @@ def run_ours(args, w):
         "roofline": dict(roofs[dominant], kernel=dominant), "rooflines": roofs,
         "recall_median": float(np.median(g.recall.cpu().numpy())),
     }
+    if args.baselines:
+        line["recall_median_by_index"] = {"saki": line["recall_median"],
+                                          **{m: g.recall_with(m) for m in ("key_pca", "weight_svd")}}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
     if rank == 0:
@@ -493,6 +513,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--baselines", action="store_true",
+                    help="also report the median recall of the key-PCA and weight-SVD indexes (Tab. 1), untimed")
     ap.add_argument("--heads", type=int, default=0,
                     help="query heads (KV heads follow the workload's group size): a smaller case of the same "
                          "shapes, for profiler captures")

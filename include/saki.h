@@ -65,6 +65,13 @@ typedef enum saki_dtype { SAKI_F32 = 0, SAKI_BF16 = 1 } saki_dtype;
 /* saki_config.flags */
 #define SAKI_FLAG_SORTED 1 /* top-k lists in descending score (ties: lower index) */
 
+/* saki_config.method: which rank-r map saki_fit folds into L and R */
+#define SAKI_METHOD_SAKI 0       /* the exact optimum M_r of Prop. 1 (default) */
+#define SAKI_METHOD_KEY_PCA 1    /* Tab. 1 comparison: M = A_h V_r V_r^T, V_r the r leading
+                                    eigenvectors of Sk; L = A_h V_r, R = V_r */
+#define SAKI_METHOD_WEIGHT_SVD 2 /* Tab. 1 comparison: the truncated SVD of A_h itself,
+                                    L = U_r Sigma_r^{1/2}, R = V_r Sigma_r^{1/2} */
+
 typedef struct saki_config {
   int32_t num_q_heads;   /* Hq >= 1 */
   int32_t num_kv_heads;  /* Hk >= 1, Hq % Hk == 0 */
@@ -77,6 +84,7 @@ typedef struct saki_config {
                             (App. A, "Singular covariances"); the paper uses 1e-6 */
   int32_t max_sweeps;    /* Jacobi sweep limit of the fit; 0 selects 40 */
   int32_t flags;         /* SAKI_FLAG_* */
+  int32_t method;        /* SAKI_METHOD_*; 0 = SAKI */
 } saki_config;
 
 /* Which keys each query may rank (HOST memory).  Keys of sequence s are rows
@@ -118,7 +126,16 @@ SAKI_API size_t saki_workspace_size(const saki_config* cfg, int32_t op, const sa
  *   loss [Hq]       optimum sum_{i>r} sigma_i^2 (NULL = skip)
  * Moments are normalised by 1/n.  Synchronises `stream`; returns SAKI_ERR_NUMERIC
  * if a moment is not finite and SAKI_ERR_NOT_CONVERGED if a head's Jacobi SVD
- * reached max_sweeps (outputs are then still written from the last sweep). */
+ * reached max_sweeps (outputs are then still written from the last sweep).
+ * The comparison methods fold other rank-r maps into the same L, R, which the
+ * index and selection calls take unchanged:
+ *   SAKI_METHOD_KEY_PCA     R = V_r (unit columns), L = A_h V_r; sigma holds the
+ *                           square roots of Sk's eigenvalues and loss the
+ *                           discarded key energy sum_{i>r} lambda_i(Sk); the
+ *                           query calibration data is read but not used;
+ *   SAKI_METHOD_WEIGHT_SVD  sigma are A_h's singular values and loss
+ *                           sum_{i>r} sigma_i^2; the calibration data is only
+ *                           checked and, when center = 1, gives mu. */
 SAKI_API saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_calib,
                      const void* k_calib, const float* A, float* L, float* R, float* mu,
                      float* nu, float* sigma, float* loss, void* workspace,

@@ -164,6 +164,8 @@ saki_status check_cfg(const saki_config* c) {
   if (!(c->eig_floor_rel >= 0.f && c->eig_floor_rel < 1.f)) return SAKI_ERR_INVALID_ARGUMENT;
   if (c->max_sweeps < 0) return SAKI_ERR_INVALID_ARGUMENT;
   if (c->flags & ~SAKI_FLAG_SORTED) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->method != SAKI_METHOD_SAKI && c->method != SAKI_METHOD_KEY_PCA && c->method != SAKI_METHOD_WEIGHT_SVD)
+    return SAKI_ERR_INVALID_ARGUMENT;
   return SAKI_OK;
 }
 
@@ -447,7 +449,8 @@ BuildWs build_ws(const saki_config* c, int64_t N) {
 }
 
 // fit workspace: S, F, G [(Hq+Hk)][d][d], mu [Hk][d], status [Hq+Hk], C'^T scratch [Hq][d][d]
-struct FitWs { size_t S, F, G, mu, st, C, bytes; };
+struct FitWs { size_t S, F, G, mu, st, C, I, sig, bytes; };
+// Key PCA also needs an identity operator per query head and its own sigma.
 FitWs fit_ws(const saki_config* c) {
   const size_t nm = (size_t)c->num_q_heads + c->num_kv_heads;
   const size_t mat = nm * kD * kD * sizeof(float);
@@ -458,7 +461,13 @@ FitWs fit_ws(const saki_config* c) {
   w.mu = w.G + align_up(mat);
   w.st = w.mu + align_up((size_t)c->num_kv_heads * kD * sizeof(float));
   w.C = w.st + align_up(nm * sizeof(int));
-  w.bytes = w.C + align_up((size_t)c->num_q_heads * kD * kD * sizeof(float));
+  w.I = w.C + align_up((size_t)c->num_q_heads * kD * kD * sizeof(float));
+  w.sig = w.I;
+  w.bytes = w.I;
+  if (c->method == SAKI_METHOD_KEY_PCA) {
+    w.sig = w.I + align_up((size_t)c->num_q_heads * kD * kD * sizeof(float));
+    w.bytes = w.sig + align_up((size_t)c->num_q_heads * kD * sizeof(float));
+  }
   return w;
 }
 
@@ -542,15 +551,38 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
                                       s))) != SAKI_OK)
       return st;
   }
+  // The comparison indexes reuse the fit with other inputs: weight SVD whitens
+  // with identity factors (C' = A); key PCA keeps the key factors and sets the
+  // query factors and the operator to the identity (C' = F_k, whose left singular
+  // vectors are Sk's eigenvectors), then folds A into L.
+  const int method = cfg->method;
+  float* Iw = reinterpret_cast<float*>(ws + w.I);
+  float* sig = method == SAKI_METHOD_KEY_PCA && !sigma ? reinterpret_cast<float*>(ws + w.sig) : sigma;
   {
     KernelTimer kt(SAKI_KERNEL_FACTOR, s);
-    if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK) return st;
+    if (method == SAKI_METHOD_WEIGHT_SVD) {
+      if ((st = cuda_status(launch_identity(F, nm, s))) != SAKI_OK) return st;
+      if ((st = cuda_status(launch_identity(Gm, nm, s))) != SAKI_OK) return st;
+    } else {
+      if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK)
+        return st;
+    }
+    if (method == SAKI_METHOD_KEY_PCA) {
+      if ((st = cuda_status(launch_identity(F, Hq, s))) != SAKI_OK) return st;
+      if ((st = cuda_status(launch_identity(Gm, Hq, s))) != SAKI_OK) return st;
+      if ((st = cuda_status(launch_identity(Iw, Hq, s))) != SAKI_OK) return st;
+    }
   }
   {
     KernelTimer kt(SAKI_KERNEL_FIT, s);
-    if ((st = cuda_status(launch_fit(A, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
-                                     reinterpret_cast<float*>(ws + w.C), L, R, sigma, loss, nu, status, s))) !=
+    const float* Afit = method == SAKI_METHOD_KEY_PCA ? Iw : A;
+    if ((st = cuda_status(launch_fit(Afit, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
+                                     reinterpret_cast<float*>(ws + w.C), L, R, sig, loss, nu, status, s))) !=
         SAKI_OK)
+      return st;
+    if (method == SAKI_METHOD_KEY_PCA &&
+        (st = cuda_status(launch_key_pca_fold(A, sig, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, L, R, nu,
+                                              s))) != SAKI_OK)
       return st;
   }
   std::vector<int> hst(nm);

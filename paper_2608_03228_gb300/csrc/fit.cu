@@ -592,6 +592,48 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
   }
 }
 
+// ---------------------------------------------------------------- comparison indexes
+// Identity matrices [nmat][d][d]: the whitening factors of a comparison index
+// that ignores a moment (both for weight SVD, the query side for key PCA), and
+// the identity operator of the key-PCA fit.
+__global__ void identity_kernel(float* X) {
+  float* Xm = X + (int64_t)blockIdx.x * kD * kD;
+  for (int o = threadIdx.x; o < kD * kD; o += blockDim.x) Xm[o] = (o / kD == o % kD) ? 1.f : 0.f;
+}
+
+// Key PCA from the fit of C' = F_k (operator and query factors set to the
+// identity): that fit returns R = V Sigma^{-1/2} with V the leading eigenvectors
+// of Sk and Sigma = Lambda^{1/2}, signed like every fit.  Rescaled, R = V (unit
+// columns); the operator is folded into the query side, L = A_h V, and the mean
+// term recomputed, nu = A_h mu_g.  One CTA of d threads per head; thread i owns
+// row i of L and R, and reads the fit's R only from shared memory.
+__global__ void __launch_bounds__(kD) key_pca_fold_kernel(const float* A, const float* sigma, const float* mu,
+                                                         int Hq, int Hk, int r, float* L, float* R, float* nu) {
+  extern __shared__ float sm[];
+  float* As = sm;                    // A_h, row stride d + 1 (row i of thread i: conflict-free)
+  float* Vs = As + kD * (kD + 1);    // V [d][r]
+  __shared__ float mus[kD];
+  const int h = blockIdx.x, g = h / (Hq / Hk), i = threadIdx.x;
+  const float* Ah = A + (int64_t)h * kD * kD;
+  float* Lh = L + (int64_t)h * kD * r;
+  float* Rh = R + (int64_t)h * kD * r;
+  for (int o = i; o < kD * kD; o += kD) As[(o / kD) * (kD + 1) + o % kD] = Ah[o];
+  for (int o = i; o < kD * r; o += kD) Vs[o] = Rh[o] * sqrtf(fmaxf(sigma[(int64_t)h * kD + o % r], 0.f));
+  mus[i] = mu ? mu[(int64_t)g * kD + i] : 0.f;
+  __syncthreads();
+  for (int c = 0; c < r; ++c) {
+    float acc = 0.f;
+    for (int j = 0; j < kD; ++j) acc = fmaf(As[i * (kD + 1) + j], Vs[j * r + c], acc);
+    Lh[i * r + c] = acc;
+    Rh[i * r + c] = Vs[i * r + c];
+  }
+  if (nu) {
+    float v = 0.f;
+    for (int j = 0; j < kD; ++j) v = fmaf(As[i * (kD + 1) + j], mus[j], v);
+    nu[(int64_t)h * kD + i] = v;
+  }
+}
+
 constexpr float kTol = 1e-6f;
 constexpr size_t kSmem = sizeof(float) * kD * kLdS;         // factor kernel: L and L^{-1} share one buffer
 constexpr size_t kFitSmem = sizeof(float) * kD * kLdJ;      // fit kernel: the Jacobi matrix
@@ -614,6 +656,23 @@ cudaError_t launch_fit(const float* A, const float* F, const float* Gm, const fl
   note_launch();
   fit_kernel<<<Hq, kFitThreads, kFitSmem, s>>>(A, F, Gm, mu, Hq, Hk, r, max_sweeps, kTol, Cws, L, R, sigma, loss,
                                                nu, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_identity(float* X, int nmat, cudaStream_t s) {
+  if (nmat == 0) return cudaSuccess;
+  note_launch();
+  identity_kernel<<<nmat, 256, 0, s>>>(X);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_key_pca_fold(const float* A, const float* sigma, const float* mu, int Hq, int Hk, int r, float* L,
+                                float* R, float* nu, cudaStream_t s) {
+  const int smem = (int)(sizeof(float) * (kD * (kD + 1) + kD * r));
+  cudaError_t e = cudaFuncSetAttribute(key_pca_fold_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  note_launch();
+  key_pca_fold_kernel<<<Hq, kD, smem, s>>>(A, sigma, mu, Hq, Hk, r, L, R, nu);
   return cudaGetLastError();
 }
 

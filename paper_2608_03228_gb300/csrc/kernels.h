@@ -105,6 +105,11 @@ cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_swe
 cudaError_t launch_fit(const float* A, const float* F, const float* Gm, const float* mu, int Hq,
                        int Hk, int r, int max_sweeps, float* Cws, float* L, float* R, float* sigma,
                        float* loss, float* nu, int* status, cudaStream_t s);
+// comparison indexes: identity matrices [nmat][d][d]; the key-PCA rescale and
+// operator fold after a fit of C' = F_k (sigma of that fit, mu may be null)
+cudaError_t launch_identity(float* X, int nmat, cudaStream_t s);
+cudaError_t launch_key_pca_fold(const float* A, const float* sigma, const float* mu, int Hq, int Hk, int r, float* L,
+                                float* R, float* nu, cudaStream_t s);
 
 // key codes
 cudaError_t launch_build_generic(const void* K, const float* R, const float* mu, void* sketch,

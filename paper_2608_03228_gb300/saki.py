@@ -20,6 +20,8 @@ _lib = ctypes.CDLL(_LIB_PATH)
 
 SAKI_F32, SAKI_BF16 = 0, 1
 SAKI_FLAG_SORTED = 1
+SAKI_METHOD_SAKI, SAKI_METHOD_KEY_PCA, SAKI_METHOD_WEIGHT_SVD = 0, 1, 2
+METHODS = {"saki": SAKI_METHOD_SAKI, "key_pca": SAKI_METHOD_KEY_PCA, "weight_svd": SAKI_METHOD_WEIGHT_SVD}
 SAKI_OP_FIT, SAKI_OP_BUILD_INDEX, SAKI_OP_SCORE_TOPK, SAKI_OP_RECALL = 0, 1, 2, 3
 STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED", 3: "SAKI_ERR_CUDA",
           4: "SAKI_ERR_NUMERIC", 5: "SAKI_ERR_NOT_CONVERGED", 6: "SAKI_ERR_WORKSPACE", 7: "SAKI_ERR_TIMEOUT"}
@@ -35,7 +37,7 @@ class Config(ctypes.Structure):
     _fields_ = [("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("rank", ctypes.c_int32), ("topk", ctypes.c_int32), ("dtype", ctypes.c_int32),
                 ("center", ctypes.c_int32), ("eig_floor_rel", ctypes.c_float), ("max_sweeps", ctypes.c_int32),
-                ("flags", ctypes.c_int32)]
+                ("flags", ctypes.c_int32), ("method", ctypes.c_int32)]
 
 
 class Layout(ctypes.Structure):
@@ -78,9 +80,10 @@ def library_path() -> str:
 
 
 def make_config(num_q_heads, num_kv_heads, rank, topk, dtype="bf16", center=0, eig_floor_rel=1e-6,
-                max_sweeps=0, flags=0, head_dim=128) -> Config:
+                max_sweeps=0, flags=0, head_dim=128, method="saki") -> Config:
     dt = {"f32": SAKI_F32, "bf16": SAKI_BF16}.get(dtype, dtype)
-    return Config(num_q_heads, num_kv_heads, head_dim, rank, topk, dt, center, eig_floor_rel, max_sweeps, flags)
+    m = METHODS.get(method, method)
+    return Config(num_q_heads, num_kv_heads, head_dim, rank, topk, dt, center, eig_floor_rel, max_sweeps, flags, m)
 
 
 class HostLayout:

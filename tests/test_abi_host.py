@@ -47,12 +47,13 @@ def test_ctypes_layout_matches_c(lib, tmp_path):
     src = tmp_path / "layout.c"
     src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "saki.h"\nint main(void){'
                    'printf("%zu %zu %zu %zu %zu\\n", sizeof(saki_config), offsetof(saki_config, eig_floor_rel),'
-                   ' offsetof(saki_config, flags), sizeof(saki_layout), offsetof(saki_layout, q_visible));return 0;}')
+                   ' offsetof(saki_config, flags), sizeof(saki_layout), offsetof(saki_layout, q_visible));'
+                   'printf("%zu\\n", offsetof(saki_config, method));return 0;}')
     exe = tmp_path / "layout"
     subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
     vals = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True).stdout.split()]
     assert vals == [ctypes.sizeof(lib.Config), lib.Config.eig_floor_rel.offset, lib.Config.flags.offset,
-                    ctypes.sizeof(lib.Layout), lib.Layout.q_visible.offset]
+                    ctypes.sizeof(lib.Layout), lib.Layout.q_visible.offset, lib.Config.method.offset]
 
 
 def test_status_strings(lib):
@@ -73,7 +74,7 @@ def _cfg(lib, **kw):
 @pytest.mark.parametrize("kw,code", [
     (dict(num_kv_heads=3), 1), (dict(rank=0), 1), (dict(rank=129), 1), (dict(topk=0), 1), (dict(topk=129), 2),
     (dict(head_dim=64), 2), (dict(dtype=7), 1), (dict(center=2), 1), (dict(eig_floor_rel=-1.0), 1),
-    (dict(max_sweeps=-1), 1), (dict(flags=4), 1),
+    (dict(max_sweeps=-1), 1), (dict(flags=4), 1), (dict(method=3), 1), (dict(method=-1), 1),
 ])
 def test_config_validation(lib, kw, code):
     cfg = _cfg(lib, **kw)
@@ -128,3 +129,13 @@ def test_workspace_grows_with_splits(lib):
     long_ = _layout(lib, [1 << 20], [0] * 8, [1 << 20] * 8)
     assert lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_TOPK, long_) > \
         lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_TOPK, short)
+
+
+def test_key_pca_fit_needs_more_workspace(lib):
+    """Key PCA folds A into L after the fit: its workspace holds an identity
+    operator per head and sigma; the SAKI fit does not pay for that."""
+    saki = lib.saki_workspace_size(_cfg(lib), lib.SAKI_OP_FIT, n_calib=16)
+    pca = lib.saki_workspace_size(_cfg(lib, method="key_pca"), lib.SAKI_OP_FIT, n_calib=16)
+    wsvd = lib.saki_workspace_size(_cfg(lib, method="weight_svd"), lib.SAKI_OP_FIT, n_calib=16)
+    assert wsvd == saki
+    assert pca >= saki + 8 * 128 * 128 * 4

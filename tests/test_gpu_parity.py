@@ -25,11 +25,11 @@ def tiny():
     return w, data, ref
 
 
-def _gpu_fit(lib, w, data, center=None, rank=None):
+def _gpu_fit(lib, w, data, center=None, rank=None, method="saki"):
     torch = _torch()
     center = w.center if center is None else center
     r = w.rank if rank is None else rank
-    cfg = lib.make_config(w.num_q_heads, w.num_kv_heads, r, w.topk, w.dtype, center=center)
+    cfg = lib.make_config(w.num_q_heads, w.num_kv_heads, r, w.topk, w.dtype, center=center, method=method)
     Hq, Hk = w.num_q_heads, w.num_kv_heads
     L = torch.empty((Hq, D, r), device="cuda")
     R = torch.empty((Hq, D, r), device="cuda")
@@ -71,6 +71,60 @@ def test_fit_tiny(lib, tiny, center):
         if _rel_gap(s_ref, w.rank) >= 1e-3:
             assert map_rel_err(g["L"][h], g["R"][h], ref["M"][h]) <= MAP_REL
         np.testing.assert_allclose(g["nu"][h], ref["nu"][h], atol=1e-4 * max(1.0, np.abs(ref["nu"][h]).max()))
+
+
+@pytest.mark.parametrize("method", ["key_pca", "weight_svd"])
+@pytest.mark.parametrize("center", [0, 1])
+def test_fit_comparison_indexes(lib, tiny, method, center):
+    """The Tab. 1 comparison indexes through saki_fit: key PCA (L = A V_r, R = V_r
+    with V_r the leading eigenvectors of Sk) and weight SVD (A's truncated SVD)."""
+    w, data, _ = tiny
+    ref = O.fit_baseline(method, data["k_calib"], data["A"], w.rank, bool(center), w.num_q_heads)
+    g = _gpu_fit(lib, w, data, center=center, method=method)
+    for h in range(w.num_q_heads):
+        s_ref = ref["sigma"][h]
+        np.testing.assert_allclose(g["sigma"][h], s_ref, atol=1e-4 * s_ref[0], rtol=0)
+        assert abs(g["loss"][h] - ref["loss"][h]) <= 1e-4 * np.sum(s_ref ** 2)
+        if _rel_gap(s_ref, w.rank) >= 1e-3:
+            assert map_rel_err(g["L"][h], g["R"][h], ref["M"][h]) <= MAP_REL, h
+            if method == "key_pca":   # R = V_r itself: orthonormal, and L = A R
+                R = g["R"][h].astype(np.float64)
+                np.testing.assert_allclose(R.T @ R, np.eye(w.rank), atol=1e-4)
+                np.testing.assert_allclose(R @ R.T, ref["R"][h] @ ref["R"][h].T, atol=1e-4)
+                np.testing.assert_allclose(g["L"][h], data["A"][h].astype(np.float64) @ R,
+                                           atol=1e-5 * np.abs(g["L"][h]).max())
+            else:   # R = V_r Sigma^{1/2}, signed like the oracle
+                np.testing.assert_allclose(g["R"][h], ref["R"][h], atol=1e-4 * np.abs(ref["R"][h]).max())
+        np.testing.assert_allclose(g["nu"][h], ref["nu"][h], atol=1e-4 * max(1.0, np.abs(ref["nu"][h]).max()))
+
+
+def test_comparison_index_recall_end_to_end(lib, tiny):
+    """fit -> index -> select -> recall with each comparison index, against the
+    oracle's chain for the same index (the Tab. 1 measurement on synthetic data)."""
+    torch = _torch()
+    w, data, _ = tiny
+    G, T = w.group, len(data["q_seq"])
+    lay = lib.HostLayout(data["seq_offsets"], data["q_seq"], data["q_visible"])
+    Qd, Kd = to_dev(data["Q"], "f32"), to_dev(data["K"], "f32")
+    ie, _ = O.exact_topk(data["Q"], data["A"], data["K"], data["seq_offsets"], data["q_seq"], data["q_visible"],
+                         w.topk, G)
+    for method in ("key_pca", "weight_svd"):
+        g = _gpu_fit(lib, w, data, method=method)
+        cfg = g["cfg"]
+        sk = torch.empty((w.num_q_heads, data["K"].shape[1], w.rank), device="cuda")
+        lib.saki_build_index(cfg, Kd, f32(g["R"]), sk)
+        idx = torch.empty((w.num_q_heads, T, w.topk), dtype=torch.int32, device="cuda")
+        lib.saki_score_topk(cfg, lay, Qd, f32(g["L"]), sk, idx)
+        rec = torch.empty((w.num_q_heads,), device="cuda")
+        lib.saki_recall(cfg, lay, w.topk + 1, Qd, f32(data["A"]), Kd, idx, rec)
+        ref = O.fit_baseline(method, data["k_calib"], data["A"], w.rank, bool(w.center), w.num_q_heads)
+        sketch = O.build_index(data["K"], ref["R"], None, "f32", G)
+        ia, _ = O.score_topk(data["Q"], ref["L"], sketch, data["seq_offsets"], data["q_seq"], data["q_visible"],
+                             w.topk)
+        ref_rec = O.head_recall(ia, ie, data["q_visible"], w.topk + 1, w.topk)
+        # rows whose k-th and (k+1)-th scores nearly tie may swap a key under the
+        # fp32 fit (one swap moves a head's recall by 1/(64 x 448 rows)): allow ~100
+        np.testing.assert_allclose(rec.cpu().numpy(), ref_rec, atol=RECALL_ABS + 0.002, err_msg=method)
 
 
 def test_fit_full_rank_and_rank_one(lib, tiny):
