@@ -3,12 +3,12 @@
  *
  * SAKI (arXiv 2608.03228) indexes a KV cache with a per-head rank-r score map.
  * For query head h reading KV head g(h) = h / (Hq / Hk):
- *   - fit (Prop. 1, Eq. 3; Sec. 5; App. A): from calibration moments Sq (queries,
+ *   - fit (Prop. 1, Eq. 3, Sec. 5; Sec. 6; App. A): from calibration moments Sq (queries,
  *     uncentered) and Sk, mu (keys), form C = Sq^{1/2} A_h Sk^{1/2}, take its
  *     truncated SVD C_r = U_r Lambda_r V_r^T and fold M_r = Sq^{-1/2} C_r Sk^{-1/2}
  *     into L_h = Sq^{-1/2} U_r Lambda_r^{1/2} and R_h = Sk^{-1/2} V_r Lambda_r^{1/2};
- *   - index (Sec. 5): key codes c_j = R_h^T (k_j - mu_g);
- *   - select (Sec. 1, Sec. 5): s_hat_j = (L_h^T q)^T c_j over the keys a query
+ *   - index (Sec. 6): key codes c_j = R_h^T (k_j - mu_g);
+ *   - select (Sec. 1, Sec. 6): s_hat_j = (L_h^T q)^T c_j over the keys a query
  *     can see, keep the k largest;
  *   - evaluate (Sec. 3 protocol): exact s_j = q^T A_h k_j, its top-k, recall@k.
  *
@@ -111,7 +111,7 @@ typedef struct saki_layout {
 SAKI_API size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout* layout,
                            int64_t n_calib, int64_t total_keys);
 
-/* saki_fit -- Prop. 1 (Eq. 3), Sec. 5 and App. A: calibration moments, the exact
+/* saki_fit -- Prop. 1 (Eq. 3, Sec. 5), Sec. 6 and App. A: calibration moments, the exact
  * rank-r minimiser of the score distortion of Eq. (1), folded into factors.
  *   q_calib [Hq][n][d] dtype   calibration queries of each query head
  *   k_calib [Hk][n][d] dtype   calibration keys of each KV head
@@ -141,7 +141,7 @@ SAKI_API saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const voi
                      float* nu, float* sigma, float* loss, void* workspace,
                      size_t workspace_bytes, saki_stream stream);
 
-/* saki_build_index -- Sec. 5 key codes c_j = R_h^T (k_j - mu_g) for every query
+/* saki_build_index -- Sec. 6 key codes c_j = R_h^T (k_j - mu_g) for every query
  * head h and every key row j (all sequences at once).
  *   K      [Hk][total_keys][d] dtype
  *   R      [Hq][d][r] f32
@@ -151,7 +151,7 @@ SAKI_API saki_status saki_build_index(const saki_config* cfg, int64_t total_keys
                              const float* R, const float* mu, void* sketch, void* workspace,
                              size_t workspace_bytes, saki_stream stream);
 
-/* saki_score_topk -- Sec. 5 selection: per (head h, query t) the k keys of the
+/* saki_score_topk -- Sec. 6 selection: per (head h, query t) the k keys of the
  * visible prefix with the largest s_hat = (L_h^T q_t)^T c_j, never forming the
  * T x N score matrix.
  *   Q      [Hq][T][d] dtype      queries

@@ -16,14 +16,14 @@ What it follows (sections and equations of arXiv 2608.03228, "SAKI"):
   ``C_r = U_r Lambda_r V_r^T``, optimum ``M_r = Sq^{-1/2} C_r Sk^{-1/2}`` with
   ``L(M_r) = sum_{i>r} lambda_i(C)^2``; singular covariances use pseudoinverse
   roots, eigenvalues below ``1e-6 * lambda_max`` are treated as zero.
-* Sec. 5 (SAKI): ``Sq`` uncentered second moment of queries, ``Sk`` and ``mu``
+* Sec. 6 (SAKI): ``Sq`` uncentered second moment of queries, ``Sk`` and ``mu``
   from centered keys (uncentered keys are the ``mu = 0`` case, App. A
   "Centering"); factors ``B_q = Sq^{-1/2} U_r Lambda_r^{1/2}`` (called ``L``
   here) and ``B_k = Sk^{-1/2} V_r Lambda_r^{1/2}`` (called ``R``); key code
   ``c_j = R^T (k_j - mu)``; score ``s_hat = (L^T q)^T c_j + q^T A mu``.
 * Sec. 3 protocol: recall of the true top-k attended positions, i.e. the
   fraction of the exact top-k set (by ``q^T A k``) found by the index.
-* Tab. 1 / Sec. 4 comparison indexes: key PCA (the rank-r principal
+* Tab. 1 (Sec. 3 baselines) comparison indexes: key PCA (the rank-r principal
   projector of the keys, M = A P) and weight SVD (the operator's truncated
   SVD, M = A_r).
 
@@ -51,13 +51,13 @@ F64 = np.float64
 
 
 # --------------------------------------------------------------------------
-# Sec. 5: calibration moments
+# Sec. 6: calibration moments
 # --------------------------------------------------------------------------
 def moments(X, center: bool):
     """Second moment of the rows of X [n][d]: ``(1/n) sum_t x_t x_t^T``.
 
     ``center=True`` returns the covariance of the centered rows and their mean
-    (keys, Sec. 5 / App. A "Centering"); ``center=False`` the uncentered second
+    (keys, Sec. 6 / App. A "Centering"); ``center=False`` the uncentered second
     moment and a zero mean (queries, and the ``mu = 0`` special case)."""
     X = np.asarray(X, F64)
     n = X.shape[0]
@@ -97,7 +97,7 @@ def canonical_signs(L, R):
 
 
 def fit_head(Sq, Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
-    """Prop. 1 (Eq. 3) and the Sec. 5 factors for one head.
+    """Prop. 1 (Eq. 3, Sec. 5) and the Sec. 6 factors for one head.
 
     Returns L = B_q [d][r], R = B_k [d][r], the score map M_r = L R^T, the
     singular values of C (all d, descending) and the optimum
@@ -147,7 +147,7 @@ def fit(q_calib, k_calib, A, rank: int, center: bool, floor_rel: float = 1e-6) -
 # Tab. 1 comparison indexes: key PCA and weight SVD
 # --------------------------------------------------------------------------
 def key_pca_head(Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
-    """Key PCA for one head (Tab. 1; Sec. 4 states that PCA minimises
+    """Key PCA for one head (Tab. 1; Sec. 5 states that PCA minimises
     ``||(I - P) Sk^{1/2}||_F^2``): P = V_r V_r^T projects onto the r leading
     eigenvectors of the key moment Sk, the score map is M = A P, and the
     factors are L = A V_r, R = V_r, so a key's code is its principal
@@ -198,7 +198,7 @@ def fit_baseline(method: str, k_calib, A, rank: int, center: bool, num_q_heads: 
 
 
 # --------------------------------------------------------------------------
-# Sec. 5: key codes (the index)
+# Sec. 6: key codes (the index)
 # --------------------------------------------------------------------------
 def round_bf16(x):
     """Round fp64 values to the bf16 grid, nearest with ties to even.
@@ -227,7 +227,7 @@ def round_to(dtype: str, x):
 
 
 def build_index(K, R, mu, dtype: str, group: int):
-    """Key codes ``c_j = R_h^T (k_j - mu_g)`` for every query head h (Sec. 5).
+    """Key codes ``c_j = R_h^T (k_j - mu_g)`` for every query head h (Sec. 6).
 
     K [Hk][N][d]; R [Hq][d][r]; mu [Hk][d] or None.  Returns [Hq][N][r] rounded
     to the index dtype."""
@@ -245,7 +245,7 @@ def build_index(K, R, mu, dtype: str, group: int):
 # Selection: approximate and exact scores, top-k, recall
 # --------------------------------------------------------------------------
 def approx_scores(q, L, sketch):
-    """``s_hat_j = (L^T q)^T c_j`` for every code row of ``sketch`` (Sec. 5)."""
+    """``s_hat_j = (L^T q)^T c_j`` for every code row of ``sketch`` (Sec. 6)."""
     u = np.asarray(L, F64).T @ np.asarray(q, F64)
     return np.asarray(sketch, F64) @ u
 

@@ -1,4 +1,4 @@
-// Key codes of Sec. 5 on CUDA cores: sketch[h][j] = R_h^T (k_j - mu_g), fp32
+// Key codes of Sec. 6 on CUDA cores: sketch[h][j] = R_h^T (k_j - mu_g), fp32
 // accumulation, rounded to nearest-even into the index dtype.  Any rank; one
 // CTA per (128 keys, query head), R_h staged in shared memory.
 #include "common.cuh"

@@ -1,4 +1,4 @@
-// Key codes of Sec. 5 on the tensor cores: sketch[h][j] = R_h^T k_j for all query
+// Key codes of Sec. 6 on the tensor cores: sketch[h][j] = R_h^T k_j for all query
 // heads h of a GQA group at once (uncentered keys, mu = 0).
 //
 // One persistent CTA per SM walks items (KV head g, block of <= 128 output

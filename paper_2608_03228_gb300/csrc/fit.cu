@@ -1,4 +1,4 @@
-// The closed-form fit of Prop. 1 (Eq. 3), Sec. 5 and App. A, one CTA per matrix.
+// The closed-form fit of Prop. 1 (Eq. 3, Sec. 5), Sec. 6 and App. A, one CTA per matrix.
 //
 // factor_kernel: for each moment matrix S (query heads, then KV heads) a factor F
 //   with F F^T = S and G = F^{+T}.  Fast path: Cholesky S = F F^T, G = F^{-T},

@@ -1,4 +1,4 @@
-// Calibration moments of Sec. 5: Sq_h = (1/n) sum_t q_t q_t^T for every query
+// Calibration moments of Sec. 6: Sq_h = (1/n) sum_t q_t q_t^T for every query
 // head (uncentered) and Sk_g = (1/n) sum_t (k_t - mu_g)(k_t - mu_g)^T with
 // mu_g = (1/n) sum_t k_t for every KV head (centered keys, App. A "Centering";
 // mu = 0 when center = 0).

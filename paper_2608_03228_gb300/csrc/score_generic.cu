@@ -1,6 +1,6 @@
 // Generic fused score + top-k on CUDA cores (any rank, f32 or bf16 inputs).
 //
-// Serves the decode-shaped work of the selection step (Sec. 5: s_hat = (L^T q)^T c_j
+// Serves the decode-shaped work of the selection step (Sec. 6: s_hat = (L^T q)^T c_j
 // over the visible keys, keep the k largest) and, with W = A and X = K, the
 // exact top-k of the Sec. 3 recall protocol.  A work item is up to kGroupQ
 // queries of one sequence against one split of its keys; each lane scores one

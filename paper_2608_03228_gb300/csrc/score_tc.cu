@@ -3,7 +3,7 @@
 // One persistent CTA per SM walks work items (a tile of up to 128 consecutive
 // queries of one sequence, one query head), heaviest tiles first.  Per item:
 //   1. projection on the tensor core: u = W^T q for the 128 queries, with the
-//      fp32 projection W (L for Sec. 5's selection, A for the exact scores of the
+//      fp32 projection W (L for Sec. 6's selection, A for the exact scores of the
 //      Sec. 3 protocol) split exactly into three bf16 parts; the fp32 result in
 //      TMEM is split into u_hi + u_lo (bf16 each) and written, swizzled, as the
 //      A operand of the main loop (keeping u to ~16 bits, far below the score

@@ -59,7 +59,7 @@ def test_fit_tiny(lib, tiny, center):
     ref = O.fit(data["q_calib"], data["k_calib"], data["A"], w.rank, center=bool(center))
     g = _gpu_fit(lib, w, data, center=center)
     Hq = w.num_q_heads
-    for h in range(Hq):   # moments (Sec. 5): fp32 accumulation of n products
+    for h in range(Hq):   # moments (Sec. 6): fp32 accumulation of n products
         assert np.linalg.norm(g["S"][h] - ref["Sq"][h]) <= 1e-5 * np.linalg.norm(ref["Sq"][h])
     for gk in range(w.num_kv_heads):
         assert np.linalg.norm(g["S"][Hq + gk] - ref["Sk"][gk]) <= 1e-5 * np.linalg.norm(ref["Sk"][gk])
