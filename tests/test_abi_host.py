@@ -139,3 +139,23 @@ def test_key_pca_fit_needs_more_workspace(lib):
     wsvd = lib.saki_workspace_size(_cfg(lib, method="weight_svd"), lib.SAKI_OP_FIT, n_calib=16)
     assert wsvd == saki
     assert pca >= saki + 8 * 128 * 128 * 4
+
+
+def test_seeded_decode_reserves_the_sample_pass(lib):
+    """A bf16 decode group cut into eight or more splits runs the tensor-core
+    kernel with a sample pass first: its plan adds the sample lists and a seed
+    per row.  fp32 groups (CUDA-core kernel) and short sequences (fewer splits)
+    are not seeded, so the same layout needs less workspace there."""
+    lay = _layout(lib, [1 << 20], [0] * 8, [1 << 20] * 8)
+    bf = lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8), lib.SAKI_OP_SCORE_TOPK, lay)
+    f32 = lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8, dtype="f32"), lib.SAKI_OP_SCORE_TOPK,
+                                  lay)
+    # 38 splits x 8 rows of 64 keys per head for the sample lists, plus a seed per row
+    assert bf - f32 >= 32 * 38 * 8 * 64 * 8 + 32 * 8 * 8
+    short = _layout(lib, [9000], [0] * 8, [9000] * 8)
+    assert lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8), lib.SAKI_OP_SCORE_TOPK, short) == \
+        lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8, dtype="f32"), lib.SAKI_OP_SCORE_TOPK, short)
+    # groups of fewer than four queries take the CUDA-core kernel: no sample pass
+    one = _layout(lib, [1 << 20], [0], [1 << 20])
+    assert lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8), lib.SAKI_OP_SCORE_TOPK, one) == \
+        lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8, dtype="f32"), lib.SAKI_OP_SCORE_TOPK, one)
