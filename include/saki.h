@@ -107,7 +107,10 @@ typedef struct saki_layout {
 
 /* Bytes of device workspace `op` needs.  FIT uses n_calib; BUILD_INDEX uses
  * total_keys; SCORE_TOPK and RECALL use the layout.  Returns 0 if the arguments
- * are invalid. */
+ * are invalid.  For SCORE_TOPK and RECALL this is the size of the fastest plan;
+ * when a decode-shaped layout would run a sample pass (see saki_score_topk) and
+ * the workspace passed is too small for its lists but holds the plan without
+ * it, the call runs that plan instead (same results, slower). */
 SAKI_API size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout* layout,
                            int64_t n_calib, int64_t total_keys);
 
@@ -162,7 +165,11 @@ SAKI_API saki_status saki_build_index(const saki_config* cfg, int64_t total_keys
  *                                k keys are visible
  *   score  [Hq][T][k] f32 or NULL   s_hat (+ q^T nu) of each idx entry, -inf pad
  * Ranking is by descending s_hat with equal scores ordered by the lower index.
- * Without SAKI_FLAG_SORTED the k entries of a row come in unspecified order. */
+ * Without SAKI_FLAG_SORTED the k entries of a row come in unspecified order.
+ * Decode-shaped groups (at least four bf16 queries of one sequence whose keys
+ * are cut into eight or more splits) first run a sample pass over the head of
+ * every split, whose per-query bound starts each split's selection; the result
+ * is the same as without it. */
 SAKI_API saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, const void* Q,
                             const float* L, const void* sketch, const float* nu, int32_t* idx,
                             float* score, void* workspace, size_t workspace_bytes,

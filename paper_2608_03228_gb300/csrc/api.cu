@@ -220,7 +220,7 @@ constexpr int64_t kSeedKeys = 1024;  // sample keys per split (at most an eighth
 // the main pass may start each query's threshold there (about 50 appends per
 // split and query in place of 800, no re-sort).  The result is unchanged: every
 // key of the row's top k scores at least the seed.
-Plan make_plan(const saki_layout* L, int Hq, int kp, int dtype, int P) {
+Plan make_plan(const saki_layout* L, int Hq, int kp, int dtype, int P, bool seed = true) {
   Plan p;
   const int64_t T = L->num_queries;
   struct G { int32_t b, n; int64_t vmax; int32_t seq; };
@@ -241,7 +241,7 @@ Plan make_plan(const saki_layout* L, int Hq, int kp, int dtype, int P) {
   int64_t chunk = std::max<int64_t>(2048, (work + target_per_head - 1) / target_per_head);
   chunk = (chunk + 255) / 256 * 256;
   // the tensor-core kernel takes groups of at least four queries
-  const bool seedable = decode_tc_eligible(dtype, P, p.nq);
+  const bool seedable = seed && decode_tc_eligible(dtype, P, p.nq);
   const int64_t samp = std::min<int64_t>(kSeedKeys, chunk / 8 / 128 * 128);
   for (const G& g : groups) {
     const int64_t base = L->seq_offsets[g.seq];
@@ -307,6 +307,19 @@ cudaError_t run_plan(ScoreArgs a, const Plan& p, char* ws, int dtype, int kp, cu
   }
   if ((e = launch_score_generic(a, dtype, kp, p.nq, s)) != cudaSuccess) return e;
   return launch_merge(a, dtype, kp, s);
+}
+
+// The plan for a call: the seeded one, or the same splits without the sample
+// pass when the workspace holds only that (same results, slower; a caller with a
+// fixed scratch, such as saki_score_topk_noalloc, keeps working at sizes the
+// sample lists would push past it).
+Plan plan_for(const saki_layout* L, int Hq, int kp, int dtype, int P, size_t workspace_bytes, size_t extra) {
+  Plan p = make_plan(L, Hq, kp, dtype, P);
+  if (!p.sitems.empty() && workspace_bytes < p.bytes + extra) {
+    Plan q = make_plan(L, Hq, kp, dtype, P, false);
+    if (workspace_bytes >= q.bytes + extra) return q;
+  }
+  return p;
 }
 
 saki_status upload_plan(const Plan& p, char* ws, cudaStream_t s) {
@@ -646,7 +659,7 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
     return run_tc(cfg, layout, tp, cfg->rank, false, Q, L, sketch, nu, idx, score, ws, s);
   }
   const int kp = kp_of(cfg->topk);
-  const Plan p = make_plan(layout, cfg->num_q_heads, kp, cfg->dtype, cfg->rank);
+  const Plan p = plan_for(layout, cfg->num_q_heads, kp, cfg->dtype, cfg->rank, workspace_bytes, 0);
   if (workspace_bytes < p.bytes) return SAKI_ERR_WORKSPACE;
   if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
   ScoreArgs a{};
@@ -681,10 +694,11 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
     if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
   const int kp = kp_of(cfg->topk);
   const bool tc = use_tc(cfg, layout, kD);
-  const Plan p = tc ? Plan{} : make_plan(layout, cfg->num_q_heads, kp, cfg->dtype, kD);
+  const size_t extra = recall_extra(cfg, T, idx_exact == nullptr);
+  const Plan p = tc ? Plan{} : plan_for(layout, cfg->num_q_heads, kp, cfg->dtype, kD, workspace_bytes, extra);
   const TcPlan tp = tc ? make_tc_plan(layout, cfg->num_q_heads, kD, false) : TcPlan{};
   const size_t base = tc ? tp.bytes : p.bytes;
-  const size_t need = base + recall_extra(cfg, T, idx_exact == nullptr);
+  const size_t need = base + extra;
   if (workspace_bytes < need) return SAKI_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
