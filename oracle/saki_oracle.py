@@ -25,7 +25,10 @@ What it follows (sections and equations of arXiv 2608.03228, "SAKI"):
   fraction of the exact top-k set (by ``q^T A k``) found by the index.
 * Tab. 1 (Sec. 3 baselines) comparison indexes: key PCA (the rank-r principal
   projector of the keys, M = A P) and weight SVD (the operator's truncated
-  SVD, M = A_r).
+  SVD, M = A_r).  Sec. 6's projector variants SAP-svd (the raw span of C's
+  right singular vectors) and SAP-map (the optimum's key-side span,
+  orthonormalised): the paper names them without formulas; the readings are
+  the docstrings of ``sap_svd_head`` and ``sap_map_head``.
 
 Readings where the paper is silent (each also listed in the design doc):
 
@@ -174,6 +177,44 @@ def weight_svd_head(A, r: int) -> dict:
     sh = np.sqrt(sig[:r])
     L, R = canonical_signs(U[:, :r] * sh, Vt[:r].T * sh)
     return dict(L=L, R=R, M=(U[:, :r] * sig[:r]) @ Vt[:r], sigma=sig, loss=float(np.sum(sig[r:] ** 2)))
+
+
+def _orth(X):
+    """Orthonormal basis of the column span of X (d x r, full column rank) by
+    modified Gram-Schmidt."""
+    Q = np.array(X, F64)
+    for c in range(Q.shape[1]):
+        for p in range(c):
+            Q[:, c] -= (Q[:, p] @ Q[:, c]) * Q[:, p]
+        Q[:, c] /= np.linalg.norm(Q[:, c])
+    return Q
+
+
+def _projector_head(Q, A) -> dict:
+    L, R = canonical_signs(np.asarray(A, F64) @ Q, Q)
+    return dict(L=L, R=R, M=L @ R.T)
+
+
+def sap_svd_head(Sq, Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
+    """SAP-svd (Sec. 6, Tab. 1): the projector onto the raw span of the r
+    leading right singular vectors V_r of C = Sq^{1/2} A Sk^{1/2}, used directly
+    as key-space directions (the whitening is not undone); M = A V_r V_r^T,
+    L = A V_r, R = V_r."""
+    rq, _ = psd_roots(Sq, floor_rel)
+    rk, _ = psd_roots(Sk, floor_rel)
+    _, _, Vt = np.linalg.svd(rq @ np.asarray(A, F64) @ rk)
+    return _projector_head(Vt[:r].T, A)
+
+
+def sap_map_head(Sq, Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
+    """SAP-map (Sec. 6, Tab. 1): the orthogonal projector onto the key-side span
+    of the optimum M_r, i.e. span(Sk^{+1/2} V_r) = the column span of the factor
+    R of ``fit_head``, orthonormalised; M = A Q Q^T, L = A Q, R = Q."""
+    _, ik = psd_roots(Sk, floor_rel)
+    rq, _ = psd_roots(Sq, floor_rel)
+    rk, _ = psd_roots(Sk, floor_rel)
+    _, _, Vt = np.linalg.svd(rq @ np.asarray(A, F64) @ rk)
+    return _projector_head(_orth(ik @ Vt[:r].T), A)
 
 
 def fit_baseline(method: str, k_calib, A, rank: int, center: bool, num_q_heads: int,

@@ -388,3 +388,45 @@ def test_baselines_from_calibration_keys():
     a = O.fit_baseline("weight_svd", K[None], A, 2, True, 2)
     b = O.fit_baseline("weight_svd", 2.0 * K[None] + 1.0, A, 2, True, 2)
     np.testing.assert_allclose(a["M"], b["M"], atol=1e-15)
+
+
+# --------------------------------------------------- SAP projector variants (Sec. 6)
+def test_sap_variants_hand_example():
+    """A = [[1, 1], [0, 1]], Sq = I, Sk = diag(4, 1), r = 1.  C = A Sk^{1/2} =
+    [[2, 1], [0, 1]]; C^T C = [[4, 2], [2, 2]] has top eigenvalue 3 + sqrt5 with
+    eigenvector v = (2, sqrt5 - 1), |v|^2 = 10 - 2 sqrt5.  SAP-svd projects on v;
+    SAP-map on Sk^{-1/2} v = (1, sqrt5 - 1), |.|^2 = 7 - 2 sqrt5."""
+    A = np.array([[1.0, 1.0], [0.0, 1.0]])
+    Sq, Sk = np.eye(2), np.diag([4.0, 1.0])
+    s5 = math.sqrt(5.0)
+    v = np.array([2.0, s5 - 1.0])
+    w = np.array([1.0, s5 - 1.0])
+    P_svd = np.outer(v, v) / (10.0 - 2.0 * s5)
+    P_map = np.outer(w, w) / (7.0 - 2.0 * s5)
+    np.testing.assert_allclose(O.sap_svd_head(Sq, Sk, A, 1)["M"], A @ P_svd, atol=1e-12)
+    np.testing.assert_allclose(O.sap_map_head(Sq, Sk, A, 1)["M"], A @ P_map, atol=1e-12)
+
+
+def test_sap_variants_reduce_to_weight_svd_with_identity_moments():
+    """Sq = Sk = I: C = A, both spans are A's leading right singular vectors, and
+    A V_r V_r^T = A_r (rotated diagonal spectrum, kept part diag(4, 3))."""
+    Q1, Q2 = _rotation(4, 7), _rotation(4, 8)
+    A = Q1 @ np.diag([4.0, 3.0, 2.0, 1.0]) @ Q2.T
+    want = Q1 @ np.diag([4.0, 3.0, 0.0, 0.0]) @ Q2.T
+    for f in (O.sap_svd_head, O.sap_map_head):
+        np.testing.assert_allclose(f(np.eye(4), np.eye(4), A, 2)["M"], want, atol=1e-12)
+
+
+@pytest.mark.parametrize("r", [1, 3, 6])
+def test_sap_variants_are_projector_maps_that_never_beat_saki(r):
+    """Remark 1: an orthogonal projector P gives the rank-r map A P, so the exact
+    optimum's loss is no larger; R has orthonormal columns and P = R R^T."""
+    for seed in range(3):
+        Sq, Sk, A = _case(seed=seed + 20)
+        best = O.fit_head(Sq, Sk, A, r)["loss"]
+        for f in (O.sap_svd_head, O.sap_map_head):
+            res = f(Sq, Sk, A, r)
+            R = res["R"]
+            np.testing.assert_allclose(R.T @ R, np.eye(r), atol=1e-10)
+            np.testing.assert_allclose(res["M"], A @ R @ R.T, atol=1e-10)
+            assert best <= O.score_loss(res["M"], A, Sq, Sk) * (1 + 1e-12)
