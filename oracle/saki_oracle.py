@@ -30,7 +30,7 @@ What it follows (sections and equations of arXiv 2608.03228, "SAKI"):
   orthonormalised): the paper names them without formulas; the readings are
   the docstrings of ``sap_svd_head`` and ``sap_map_head``.
 
-Readings where the paper is silent (each also listed in the design doc):
+Readings where the paper is silent:
 
 * lambda_i(C) in Eq. (3) are the singular values of the (non-symmetric) C.
 * Moments are normalised by 1/n.
@@ -208,8 +208,10 @@ def sap_svd_head(Sq, Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
 
 def sap_map_head(Sq, Sk, A, r: int, floor_rel: float = 1e-6) -> dict:
     """SAP-map (Sec. 6, Tab. 1): the orthogonal projector onto the key-side span
-    of the optimum M_r, i.e. span(Sk^{+1/2} V_r) = the column span of the factor
-    R of ``fit_head``, orthonormalised; M = A Q Q^T, L = A Q, R = Q."""
+    of the optimum M_r, i.e. span((Sk^{1/2})^+ V_r), with (Sk^{1/2})^+ the
+    pseudo-inverse of the symmetric root (eigenvalues below the App. A floor
+    count as zero), which is the column span of the factor R of ``fit_head``,
+    orthonormalised; M = A Q Q^T, L = A Q, R = Q."""
     _, ik = psd_roots(Sk, floor_rel)
     rq, _ = psd_roots(Sq, floor_rel)
     rk, _ = psd_roots(Sk, floor_rel)

@@ -1,5 +1,10 @@
 """Helpers of the GPU parity tests: run the oracle and the CUDA library on the
-same seeded inputs and compare with the tolerances stated in the design doc."""
+same seeded inputs and compare them element by element.
+
+Tolerances: top-k sets must be identical wherever the oracle's k-th/(k+1)-th
+score gap exceeds GAP_REL x the row's largest |score|; reported scores agree
+within SCORE_REL x that maximum (fp32 accumulation of bf16 inputs); recall
+within RECALL_ABS; the rank-r map M_r within MAP_REL relative Frobenius."""
 from __future__ import annotations
 
 import numpy as np
@@ -52,8 +57,9 @@ def check_topk_rows(gpu_idx, rows_scores, k, gpu_scores=None, label=""):
                 assert set(valid.tolist()) == set(ref_idx.tolist()), (label, r, gap / mx)
                 exact += 1
             else:
-                # near-tie: every selected key must score within tolerance of the k-th
-                assert np.all(s[valid] >= srt[k - 1] - SCORE_REL * mx), (label, r)
+                # near-tie: the set is not unique at this margin, but every selected
+                # key must score within the same margin of the oracle's k-th
+                assert np.all(s[valid] >= srt[k - 1] - GAP_REL * mx), (label, r)
                 waived += 1
         if gpu_scores is not None:
             gs = np.asarray(gpu_scores[r])[:len(valid)]
@@ -64,3 +70,25 @@ def check_topk_rows(gpu_idx, rows_scores, k, gpu_scores=None, label=""):
 def map_rel_err(L_gpu, R_gpu, M_ref):
     M = np.asarray(L_gpu, np.float64) @ np.asarray(R_gpu, np.float64).T
     return np.linalg.norm(M - M_ref) / np.linalg.norm(M_ref)
+
+
+def recall_allowance(ref_rows, alt_rows, k, min_visible):
+    """How far a head's recall may move when the approximate scores change from
+    ``ref_rows`` (the oracle chain's) to ``alt_rows`` (the same formula evaluated
+    on the library's fitted factors), counted row by row (Prop. 2).
+
+    In a row where every score moved by at most e, a key can enter or leave the
+    top k only if it scores within 2 e of the oracle's k-th score; each such key
+    changes that row's recall by at most 1/k.  Returns the sum over qualifying
+    rows of min(k, #such keys) / k, divided by the number of qualifying rows."""
+    total, rows = 0.0, 0
+    for s, t in zip(ref_rows, alt_rows):
+        s = np.asarray(s, np.float64)
+        if len(s) < min_visible:
+            continue
+        rows += 1
+        e = float(np.max(np.abs(np.asarray(t, np.float64) - s)))
+        kth = np.sort(s)[::-1][k - 1]
+        m = int(np.sum(np.abs(s - kth) <= 2 * e)) if e > 0 else 0
+        total += min(k, m) / k
+    return total / max(1, rows)

@@ -97,10 +97,12 @@ def _check_rows(w, data, idx, sc, heads, rows, src, score_fn, label):
         e, wv = check_topk_rows(gi, vectors, w.topk, gpu_scores=gs, label=f"{label} h{h}")
         waived += wv
         total += len(rows)
-    # a row is waived (checked for validity only) when the oracle's own k-th/(k+1)-th
-    # gap is below 1e-4 of the row maximum: a property of the data, frequent over 1M
-    # random keys, so only a majority of exactly compared rows is required
-    assert waived <= total // 2, (label, waived, total)
+    # A row is waived when the oracle's own k-th/(k+1)-th gap is below 1e-4 of the
+    # row maximum; its selection is still checked key by key against that margin.
+    # The count depends on the data alone (a simulation of Gaussian scores: about
+    # 8 % of rows over 4096 keys, 12 % over 1M); the bound, 30 % of the rows or
+    # four, only keeps the exact comparison from becoming vacuous.
+    assert waived <= max(4, (3 * total + 9) // 10), (label, waived, total)
 
 
 # ------------------------------------------------------------------ Llama-3.1-8B shapes

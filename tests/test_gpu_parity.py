@@ -5,7 +5,8 @@ import pytest
 
 from oracle import saki_oracle as O
 from paper_2608_03228_gb300 import synth
-from tests.parity import (GAP_REL, MAP_REL, RECALL_ABS, check_topk_rows, f32, map_rel_err, to_dev)
+from tests.parity import (GAP_REL, MAP_REL, RECALL_ABS, check_topk_rows, f32, map_rel_err, recall_allowance,
+                          to_dev)
 
 pytestmark = pytest.mark.gpu
 D = 128
@@ -122,9 +123,21 @@ def test_comparison_index_recall_end_to_end(lib, tiny):
         ia, _ = O.score_topk(data["Q"], ref["L"], sketch, data["seq_offsets"], data["q_seq"], data["q_visible"],
                              w.topk)
         ref_rec = O.head_recall(ia, ie, data["q_visible"], w.topk + 1, w.topk)
-        # rows whose k-th and (k+1)-th scores nearly tie may swap a key under the
-        # fp32 fit (one swap moves a head's recall by 1/(64 x 448 rows)): allow ~100
-        np.testing.assert_allclose(rec.cpu().numpy(), ref_rec, atol=RECALL_ABS + 0.002, err_msg=method)
+        # The library's fp32 fit moves every approximate score a little; a key can
+        # change sides only in rows where it scores within twice that move of the
+        # oracle's k-th (Prop. 2).  Those keys are counted per head, with the same
+        # count on the exact side at the parity margin GAP_REL (fp32 exact scores).
+        alt_sketch = O.build_index(data["K"], g["R"].astype(np.float64), None, "f32", G)
+        got = rec.cpu().numpy()
+        for h in range(w.num_q_heads):
+            vis = data["q_visible"]
+            ref_rows = [O.approx_scores(data["Q"][h, t], ref["L"][h], sketch[h, :vis[t]]) for t in range(T)]
+            alt_rows = [O.approx_scores(data["Q"][h, t], g["L"][h], alt_sketch[h, :vis[t]]) for t in range(T)]
+            ex_rows = [O.exact_scores(data["Q"][h, t], data["A"][h], data["K"][h // G, :vis[t]]) for t in range(T)]
+            slack = [np.abs(r_).max() * GAP_REL if len(r_) else 0.0 for r_ in ex_rows]
+            allow = (recall_allowance(ref_rows, alt_rows, w.topk, w.topk + 1) +
+                     recall_allowance(ex_rows, [r_ + e for r_, e in zip(ex_rows, slack)], w.topk, w.topk + 1))
+            assert abs(got[h] - ref_rec[h]) <= RECALL_ABS + allow, (method, h, got[h], ref_rec[h], allow)
 
 
 def test_fit_full_rank_and_rank_one(lib, tiny):

@@ -430,3 +430,103 @@ def test_sap_variants_are_projector_maps_that_never_beat_saki(r):
             np.testing.assert_allclose(R.T @ R, np.eye(r), atol=1e-10)
             np.testing.assert_allclose(res["M"], A @ R @ R.T, atol=1e-10)
             assert best <= O.score_loss(res["M"], A, Sq, Sk) * (1 + 1e-12)
+
+
+# ------------------------------------------------------------ layouts and GQA
+def _two_sequence_layout():
+    """Two sequences in one key tensor: sequence 0 holds rows 0..4, sequence 1
+    rows 5..10.  Each query names its sequence and how many of that sequence's
+    keys it sees (the causal or decode prefix)."""
+    seq_offsets = np.array([0, 5, 11], np.int64)
+    #            t:  0  1  2  3  4  5
+    q_seq = np.array([0, 1, 1, 0, 1, 0], np.int32)
+    q_visible = np.array([3, 4, 6, 1, 0, 5], np.int64)
+    # one-dimensional codes (r = 1) chosen so that a visible prefix one key too
+    # long or too short, or a sequence read from the wrong base row, changes the
+    # top two
+    codes0 = [5.0, 1.0, 4.0, 9.0, 3.0]
+    codes1 = [0.0, 9.0, 7.0, 8.0, 6.0, 10.0]
+    u = np.array([1.0, 1.0, 1.0, 1.0, 1.0, -1.0])      # the last query ranks keys by -code
+    # the expected sequence-local top-2 of every query, worked out by hand:
+    #   t0: seq 0, keys 0..2, codes 5 1 4        -> 0, 2
+    #   t1: seq 1, keys 0..3, codes 0 9 7 8      -> 1, 3
+    #   t2: seq 1, keys 0..5, codes 0 9 7 8 6 10 -> 5, 1
+    #   t3: seq 0, key 0 only                    -> 0, -1
+    #   t4: seq 1, no key                        -> -1, -1
+    #   t5: seq 0, keys 0..4, scores -5 -1 -4 -9 -3 -> 1, 4
+    expected = np.array([[0, 2], [1, 3], [5, 1], [0, -1], [-1, -1], [1, 4]])
+    return seq_offsets, q_seq, q_visible, np.array(codes0 + codes1), u, expected
+
+
+def test_score_topk_slices_each_query_by_its_sequence_and_prefix():
+    off, q_seq, q_vis, codes, u, expected = _two_sequence_layout()
+    d = 4
+    Q = np.zeros((1, len(q_seq), d))
+    Q[0, :, 2] = u                                   # u = L^T q = q[2] with L = e_2
+    L = np.zeros((1, d, 1))
+    L[0, 2, 0] = 1.0
+    sketch = codes.reshape(1, -1, 1)
+    idx, val = O.score_topk(Q, L, sketch, off, q_seq, q_vis, 2)
+    np.testing.assert_array_equal(idx[0], expected)
+    assert list(val[0, 0]) == [5.0, 4.0] and list(val[0, 5]) == [-1.0, -3.0]
+    assert np.isneginf(val[0, 3, 1]) and np.all(np.isneginf(val[0, 4]))
+
+
+def test_exact_topk_slices_the_same_layout_and_maps_query_heads_to_kv_heads():
+    """Four query heads over two KV heads (G = 2): heads 0 and 1 must read KV head
+    0, heads 2 and 3 KV head 1.  KV head 1 holds the negated keys, so a wrong
+    head mapping reverses the ranking."""
+    off, q_seq, q_vis, codes, u, expected = _two_sequence_layout()
+    d = 3
+    K = np.zeros((2, len(codes), d))
+    K[0, :, 1] = codes
+    K[1, :, 1] = -codes
+    A = np.zeros((4, d, d))
+    A[:, 0, 1] = 1.0                                 # s = q[0] * k[1]
+    Q = np.zeros((4, len(q_seq), d))
+    Q[:, :, 0] = u
+    idx, _ = O.exact_topk(Q, A, K, off, q_seq, q_vis, 2, group=2)
+    for h in (0, 1):
+        np.testing.assert_array_equal(idx[h], expected)
+    # KV head 1: every query ranks by -code (the last one by +code), worked by hand
+    neg = np.array([[1, 2], [0, 2], [0, 4], [0, -1], [-1, -1], [3, 0]])
+    for h in (2, 3):
+        np.testing.assert_array_equal(idx[h], neg)
+
+
+def _diag_calibration(lams, d):
+    """n = d calibration rows whose uncentered second moment is exactly
+    diag(lams): row i = sqrt(d * lams[i]) e_i."""
+    X = np.zeros((d, d))
+    X[np.arange(d), np.arange(d)] = np.sqrt(d * np.asarray(lams, float))
+    return X
+
+
+def test_fit_maps_query_heads_to_their_own_kv_head():
+    """Hq = 4, Hk = 2.  With A = I and Sq = I exactly, the optimum is the
+    projector onto the r leading eigenvectors of the head's own Sk (Prop. 1:
+    C = Sk^{1/2}, M_r = Sk^{-1/2} C_r Sk^{-1/2}).  KV head 0 has its energy on
+    axes 0, 1 and KV head 1 on axes 2, 3, so heads 0, 1 must get diag(1, 1, 0,
+    ...) and heads 2, 3 diag(0, 0, 1, 1, 0, ...)."""
+    d, r = 8, 2
+    lam0 = [9.0, 4.0, 1.0, 0.5, 0.25, 0.2, 0.1, 0.05]
+    lam1 = [1.0, 0.5, 9.0, 4.0, 0.25, 0.2, 0.1, 0.05]
+    k_cal = np.stack([_diag_calibration(lam0, d), _diag_calibration(lam1, d)])
+    q_cal = np.stack([_diag_calibration(np.ones(d), d)] * 4)
+    A = np.stack([np.eye(d)] * 4)
+    res = O.fit(q_cal, k_cal, A, r, center=False)
+    P0 = np.diag([1.0, 1, 0, 0, 0, 0, 0, 0])
+    P1 = np.diag([0.0, 0, 1, 1, 0, 0, 0, 0])
+    for h, P in zip(range(4), (P0, P0, P1, P1)):
+        np.testing.assert_allclose(res["M"][h], P, atol=1e-12)
+    # loss = the discarded key energy of the head's own KV head
+    np.testing.assert_allclose(res["loss"], [1.0 + 0.5 + 0.25 + 0.2 + 0.1 + 0.05] * 2 +
+                               [1.0 + 0.5 + 0.25 + 0.2 + 0.1 + 0.05] * 2, rtol=1e-12)
+    for method in ("key_pca", "weight_svd"):
+        base = O.fit_baseline(method, k_cal, A, r, False, 4)
+        if method == "key_pca":      # R spans the two leading axes of the head's KV head
+            for h, P in zip(range(4), (P0, P0, P1, P1)):
+                np.testing.assert_allclose(base["R"][h] @ base["R"][h].T, P, atol=1e-12)
+            np.testing.assert_allclose(base["loss"], [2.1] * 4, rtol=1e-12)
+        else:                        # data-blind: every head keeps two unit directions of I
+            np.testing.assert_allclose(base["loss"], [d - r] * 4, rtol=1e-12)
