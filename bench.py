@@ -254,7 +254,6 @@ def run_ours(args, w):
     pk = peaks()
     names = ["fit", "build_index", "score_topk", "recall"]
     roofs = rooflines(w, pk, ktime, g)
-    dominant = max(roofs, key=lambda n: roofs[n]["ms_per_launch"] * roofs[n]["launches_per_step"])
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -267,12 +266,17 @@ def run_ours(args, w):
         "clocks": clk, "e2e": e2e, "gpu_launches": launches,
         "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
         "score_topk_keys_per_s": pairs / (stage_ms[2] / 1e3),
-        "roofline": dict(roofs[dominant], kernel=dominant), "rooflines": roofs,
+        "roofline": dict(roofs["select"], kernel="select: fused score + top-k (saki_score_topk)"),
+        "rooflines": roofs,
         "recall_median": float(np.median(g.recall.cpu().numpy())),
     }
     if args.baselines:
         line["recall_median_by_index"] = {"saki": line["recall_median"],
                                           **{m: g.recall_with(m) for m in ("key_pca", "weight_svd")}}
+    if not args.no_extras and world == 1 and args.workload == "llama31_8b_t4096_r32" and not args.heads:
+        del g
+        torch.cuda.empty_cache()
+        line["workloads"] = {name: measure_extra(name, what, args, pk, dev) for name, what in EXTRAS}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
     if rank == 0:
@@ -374,12 +378,32 @@ TRAFFIC_BYTES_PER_PAIR = {
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only
 
 
+def selection_model(w, pk, N, T, kind):
+    """The roofline of a selection kernel, as the survey's measurement plan sets
+    it: a batched causal layout is a dense (query x key x r) contraction on the
+    tensor core, 2 P flop per visible (head, query, key) pair against the bf16
+    peak (P = r for the index, d for the exact scores of the evaluation); a
+    decode-shaped or ragged layout is bound by reading the codes (or keys) once,
+    plus the queries and the written indices, against the copy bandwidth."""
+    pairs = visible_pairs(w)
+    Hq, Hk, r = w.num_q_heads, w.num_kv_heads, w.rank
+    eb = 2 if w.dtype == "bf16" else 4
+    P = r if kind == "select" else D
+    if w.queries == "causal":
+        return ("tensor", 2 * P * pairs, "TFLOP/s", pk["bf16_tflops"],
+                f"2 x {P} flop per visible (head, query, key) pair on the tensor core", "cuBLAS bf16 GEMM, burst")
+    x = Hq * N * r * eb if kind == "select" else Hk * N * D * eb
+    io = Hq * T * D * eb + Hq * T * w.topk * 4
+    what = f"rank-{r} codes" if kind == "select" else "keys"
+    return ("hbm", x + io, "GB/s", pk["hbm_gbs"], f"{what} read once, queries read, indices written",
+            "STREAM copy")
+
+
 def rooflines(w, pk, ktime, g):
     """Per timed kernel: algorithmic work per launch / event-measured launch time."""
     pairs = visible_pairs(w)
     N, Hq, Hk, r, n = g.N, w.num_q_heads, w.num_kv_heads, w.rank, w.n_calib
     eb = 2 if w.dtype == "bf16" else 4
-    T = g.T
     out = {}
 
     def entry(name, bound, work, unit, peak, note, peak_name):
@@ -395,32 +419,10 @@ def rooflines(w, pk, ktime, g):
                      "launches_per_step": cnt / max(1, ktime["_steps"]), "work_per_launch": work,
                      "peak_source": f"{pk['source']} ({peak_name})", "model": note}
 
-    alu = pk["alu_tops"]
-    # A selection has two floors: its bytes (queries, codes or keys and the
-    # projection read once, indices written) at the copy bandwidth, and one
-    # threshold comparison per visible pair at the lane rate (the scores come from
-    # the tensor core, far below its peak).  The larger floor is the bound: the
-    # bytes for decode-shaped calls (few queries over many keys), and for the
-    # batched causal workloads too, where the query and index bytes alone exceed
-    # the comparisons.
-    io = Hq * T * D * eb + Hq * T * w.topk * 4
-
-    def selection(name, nbytes, what):
-        t_hbm = nbytes / (pk["hbm_gbs"] * 1e9)
-        t_alu = pairs / (alu * 1e12)
-        if t_hbm >= t_alu:
-            entry(name, "hbm", nbytes, "GB/s", pk["hbm_gbs"],
-                  f"queries, {what} read once, indices written (the comparison floor, one per visible pair at "
-                  f"the lane rate, is lower)", "STREAM copy")
-        else:
-            entry(name, "alu", pairs, "Tops/s", alu,
-                  f"one threshold comparison per visible (head, query, key) pair (the byte floor, queries, {what} "
-                  f"read once, is lower)", "152 SMs x 128 lanes x max SM clock")
-        if name in out:
-            out[name]["floors_ms"] = {"hbm": t_hbm * 1e3, "alu": t_alu * 1e3}
-
-    selection("select", io + Hq * N * r * eb + Hq * D * r * 4, f"rank-{r} codes and L")
-    selection("exact", io + Hk * N * D * eb + Hq * D * D * 4, "keys and A")
+    entry("select", *selection_model(w, pk, N, g.T, "select"))
+    entry("exact", *selection_model(w, pk, N, g.T, "exact"))
+    if "exact" in out:
+        out["exact"]["model"] += " (evaluation only: the exact top-k of the recall protocol)"
     entry("moments", "hbm", (Hq + Hk) * n * D * eb + (Hq + Hk) * D * D * 4, "GB/s", pk["hbm_gbs"],
           "calibration queries and keys read once, fp32 moment matrices written", "STREAM copy")
     entry("build", "hbm", Hk * N * D * eb + Hq * N * r * eb, "GB/s", pk["hbm_gbs"],
@@ -429,6 +431,86 @@ def rooflines(w, pk, ktime, g):
           "model: 4 d^3 flop per head for C' plus 6 d^3 per one-sided Jacobi sweep at 8 sweeps", "fp32 FMA")
     entry("factor", "alu", (Hq + Hk) * (D ** 3 // 3 + D ** 3), "TFLOP/s", pk["fp32_tflops"],
           "model: Cholesky d^3/3 plus triangular inverse d^3 flop per moment matrix", "fp32 FMA")
+    return out
+
+
+# Workloads timed after the headline step, each under its own key of the JSON
+# line: what is timed, and why (the survey's measurement plan).
+EXTRAS = [
+    ("decode_n1m_b1_r32", "select"),          # 1M-token decode, one query: HBM-bound selection
+    ("decode_n1m_b8_r32", "select"),          # the same cache, eight queries
+    ("ragged64_mistral7b_r64", "build+select"),   # index build and selection in one timed step
+    ("qwen25_7b_t4096_r16", "select"),        # rank sweep at the Qwen2.5-7B shape (Tab. 2)
+    ("qwen25_7b_t4096_r32", "select"),
+    ("qwen25_7b_t4096_r64", "select"),
+    ("llama32_3b_t4096_r32", "select"),
+    ("qwen25_7b_t4096_r32_n512", "fit"),      # calibration-length sweep (Fig. 2A)
+    ("qwen25_7b_t4096_r32_n32768", "fit"),
+]
+
+
+def measure_extra(name, what, args, pk, dev):
+    """Time one call kind of a workload: W warm-up and max(K, 5) timed calls, CUDA
+    events on the launching stream, inputs resident (every input is larger than
+    L2, so consecutive calls do not reuse cached data).  One untimed full step
+    first produces the factors and codes and the median recall."""
+    import torch
+    w = synth.WORKLOADS[name]
+    g = GpuPath(w, dev)
+    g.step()
+    torch.cuda.synchronize()
+    S, d = g.saki, g.data
+    recall_median = float(np.median(g.recall.cpu().numpy()))
+
+    def call():
+        if what == "fit":
+            S.saki_fit(g.cfg, d["q_calib"], d["k_calib"], d["A"], g.L, g.R, mu=g.mu, nu=g.nu, sigma=g.sigma,
+                       loss=g.loss, workspace=g.ws)
+            return
+        if what == "build+select":
+            S.saki_build_index(g.cfg, d["K"], g.R, g.sketch, mu=g.mu, workspace=g.ws)
+        S.saki_score_topk(g.cfg, g.lay, d["Q"], g.L, g.sketch, g.idx, workspace=g.ws)
+
+    for _ in range(max(3, args.warmup)):
+        call()
+    torch.cuda.synchronize()
+    kinds = {"select": KINDS["select"], "build": KINDS["build"], "moments": KINDS["moments"], "fit": KINDS["fit"],
+             "factor": KINDS["factor"]}
+    for k in kinds.values():
+        S.saki_kernel_timer_start(k)
+    n = max(5, args.steps)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(n):
+        call()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / n
+    kt = {k: S.saki_kernel_timer_stop(v) for k, v in kinds.items()}
+    kt["_steps"] = n
+    roofs = rooflines(w, pk, kt, g)
+    pairs = visible_pairs(w)
+    out = {"timed": what, "ms_per_call": ms, "calls": n, "query_heads": w.num_q_heads, "kv_heads": w.num_kv_heads,
+           "T": g.T, "N": g.N, "rank": w.rank, "n_calib": w.n_calib, "recall_median": recall_median,
+           "kernel_ms": {k: round(v["ms_per_launch"] * v["launches_per_step"], 4) for k, v in roofs.items()}}
+    if what == "fit":
+        out["roofline"] = dict(roofs["moments"], kernel="moments") if "moments" in roofs else None
+    else:
+        out["scored_keys_per_s"] = pairs / (ms / 1e3)
+        out["roofline"] = dict(roofs["select"], kernel="select") if "select" in roofs else None
+        if what == "build+select":
+            # the whole timed step against the HBM floor of the step: keys read,
+            # codes written by the build and read back by the selection
+            eb = 2 if w.dtype == "bf16" else 4
+            nbytes = (w.num_kv_heads * g.N * D * eb + 2 * w.num_q_heads * g.N * w.rank * eb +
+                      w.num_q_heads * g.T * (D * eb + w.topk * 4))
+            out["step_roofline"] = {"bound": "hbm", "achieved": nbytes / (ms / 1e3) / 1e9, "peak": pk["hbm_gbs"],
+                                    "unit": "GB/s", "frac": nbytes / (ms / 1e3) / 1e9 / pk["hbm_gbs"],
+                                    "traffic": None, "work_per_step": nbytes,
+                                    "model": "keys read, codes written and read back, queries read, indices "
+                                             "written (build and selection not fused)"}
+    del g
+    torch.cuda.empty_cache()
     return out
 
 
@@ -513,6 +595,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the decode, ragged and rank/calibration-sweep workloads timed after the headline step")
     ap.add_argument("--baselines", action="store_true",
                     help="also report the median recall of the key-PCA and weight-SVD indexes (Tab. 1), untimed")
     ap.add_argument("--heads", type=int, default=0,

@@ -16,17 +16,32 @@
  *   Pointers.  Tensor arguments are DEVICE pointers on the current CUDA device,
  *     16-byte aligned, row-major with the last listed dimension fastest.  The
  *     layout description (saki_layout) is HOST memory.  The caller owns every
- *     buffer, including the workspace; the library keeps no state between calls
- *     and allocates no device memory.
- *   Streams.  Work is enqueued on `stream` (NULL = legacy default stream).
- *     saki_fit synchronises the stream once to report numeric status;
- *     saki_score_topk and saki_recall copy their small host-side work list into
- *     the workspace with cudaMemcpyAsync from pageable memory, which orders
- *     them after earlier work on the stream.  Other calls return at once.
+ *     buffer, including the workspace; the library allocates no device memory.
+ *   Host staging.  The library's own small transfers (the work list a call
+ *     builds on the host, status words read back) go through a ring of mapped
+ *     pinned host slots per device that the library allocates on first use
+ *     (cudaHostAlloc, at least 4 MB a slot) and keeps for the life of the
+ *     process; a copy kernel on `stream` moves them, so they never queue behind
+ *     the caller's large copies on other streams.  A slot is reused once the
+ *     copy that last read it has run; when none is free the ring grows by one
+ *     slot instead of blocking the host.  saki_score_topk_noalloc stages
+ *     through pageable memory instead and pins nothing.
+ *   Streams.  Work is enqueued on `stream` (NULL = legacy default stream) and
+ *     the calls return without waiting for it, except saki_fit, which
+ *     synchronises the stream once to report numeric status, and calls made
+ *     with SAKI_FLAG_CHECK.  A stream in capture mode is refused
+ *     (SAKI_ERR_UNSUPPORTED, nothing enqueued): each call uploads a work list
+ *     from host memory that lives only for the call.
  *   Errors.  Arguments are checked before any launch; on SAKI_ERR_INVALID_ARGUMENT,
  *     SAKI_ERR_UNSUPPORTED or SAKI_ERR_WORKSPACE nothing is launched and no
  *     output is touched.  SAKI_ERR_CUDA reports a failed launch or copy (the
- *     CUDA error is left for cudaGetLastError()).
+ *     CUDA error is left for cudaGetLastError()).  Every wait inside a kernel
+ *     is bounded (about two seconds); a kernel whose wait runs out stops,
+ *     leaves its outputs partly written and sets the error word in the first
+ *     bytes of the call's workspace.  saki_score_topk, saki_recall and
+ *     saki_build_index return before their kernels run, so that word is read
+ *     by saki_workspace_status (or by the call itself under SAKI_FLAG_CHECK),
+ *     which returns SAKI_ERR_TIMEOUT when it is set.
  *   dtype.  SAKI_F32 or SAKI_BF16 applies to queries, keys, calibration data and
  *     key codes; A, L, R, mu, nu, sigma, loss and scores are always float32.
  *   GQA.  Query head h uses KV head h / (num_q_heads / num_kv_heads).
@@ -64,6 +79,10 @@ typedef enum saki_dtype { SAKI_F32 = 0, SAKI_BF16 = 1 } saki_dtype;
 
 /* saki_config.flags */
 #define SAKI_FLAG_SORTED 1 /* top-k lists in descending score (ties: lower index) */
+#define SAKI_FLAG_CHECK 2  /* saki_score_topk, saki_recall, saki_build_index (and the
+                              no-alloc selection) synchronise `stream` before returning
+                              and report the device status of their kernels, as
+                              saki_workspace_status does */
 
 /* saki_config.method: which rank-r map saki_fit folds into L and R */
 #define SAKI_METHOD_SAKI 0       /* the exact optimum M_r of Prop. 1 (default) */
@@ -188,6 +207,16 @@ SAKI_API saki_status saki_recall(const saki_config* cfg, const saki_layout* layo
                         int32_t* idx_exact, float* recall, void* workspace,
                         size_t workspace_bytes, saki_stream stream);
 
+/* saki_workspace_status -- the device status of the last saki_score_topk,
+ * saki_recall or saki_build_index call that used `workspace` (the first 256 bytes
+ * of every workspace of these calls are a header holding the error word, which
+ * each call clears as it starts).  Synchronises `stream`, the stream that call
+ * ran on, then returns SAKI_OK, or SAKI_ERR_TIMEOUT if one of the call's kernels
+ * gave up a bounded wait (its outputs are then incomplete).  A call that
+ * launched nothing (no queries) leaves the header as it was.  saki_fit reports
+ * its status itself and keeps no header. */
+SAKI_API saki_status saki_workspace_status(const void* workspace, saki_stream stream);
+
 /* Bytes of the static device scratch array behind saki_score_topk_noalloc. */
 #define SAKI_NOALLOC_SCRATCH_BYTES (16u << 20)
 
@@ -202,9 +231,13 @@ SAKI_API saki_status saki_recall(const saki_config* cfg, const saki_layout* layo
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress) with that device current; make that first call
  *     before any stream capture.
- *   - A layout whose work plan needs more than SAKI_NOALLOC_SCRATCH_BYTES
- *     (saki_workspace_size with SAKI_OP_SCORE_TOPK reports the need) is rejected
- *     with SAKI_ERR_WORKSPACE before any launch.
+ *   - The call runs the fastest plan that fits the scratch: saki_workspace_size
+ *     (SAKI_OP_SCORE_TOPK) reports the fastest plan, and a decode-shaped layout
+ *     whose seeded plan (see saki_score_topk) exceeds SAKI_NOALLOC_SCRATCH_BYTES
+ *     runs without the sample pass when that fits (same results).  Only a layout
+ *     that even the plan without it does not fit is rejected, with
+ *     SAKI_ERR_WORKSPACE, before any launch.
+ *   - Its device status is read by saki_noalloc_status (or SAKI_FLAG_CHECK).
  *   - Every call shares the one array and it keeps the last call's contents;
  *     each call rewrites everything it later reads, so nothing needs clearing,
  *     but calls that overlap on the GPU (other streams, other host threads)
@@ -213,6 +246,11 @@ SAKI_API saki_status saki_score_topk_noalloc(const saki_config* cfg, const saki_
                                              const void* Q, const float* L, const void* sketch,
                                              const float* nu, int32_t* idx, float* score,
                                              saki_stream stream);
+
+/* saki_noalloc_status -- saki_workspace_status for the static scratch of
+ * saki_score_topk_noalloc on the current device (SAKI_OK before its first call);
+ * no counterpart in the paper. */
+SAKI_API saki_status saki_noalloc_status(saki_stream stream);
 
 /* Static description of a status code. */
 /* ---------------------------------------------------------------- profiling aids
@@ -238,6 +276,15 @@ SAKI_API saki_status saki_score_topk_noalloc(const saki_config* cfg, const saki_
 #define SAKI_KERNEL_BUILD 5   /* key-code kernel(s) of saki_build_index */
 #define SAKI_KERNEL_FACTOR 6  /* moment-factor kernel of saki_fit */
 SAKI_API int64_t saki_launch_count(void);
+/* saki_debug_inject_stall(kind): a test hook for the failure reporting.  Arms a
+ * one-shot stall for the next launch of a tensor-core kernel of that kind
+ * (SAKI_KERNEL_SELECT, SAKI_KERNEL_EXACT or SAKI_KERNEL_BUILD; 0 disarms): its
+ * TMA producer issues no loads, so the other roles' bounded waits run out
+ * (about two seconds), the kernel stops without faulting and the call's error
+ * word reports SAKI_ERR_TIMEOUT.  A launch of another path (CUDA-core kernels,
+ * which do not wait) leaves the stall armed.  SAKI_ERR_INVALID_ARGUMENT for
+ * other kinds. */
+SAKI_API saki_status saki_debug_inject_stall(int32_t kind);
 SAKI_API saki_status saki_kernel_timer_start(int32_t kind);
 SAKI_API saki_status saki_kernel_timer_stop(int32_t kind, double* total_ms, int64_t* launches);
 

@@ -2,7 +2,7 @@
 // host-side work plan of the selection kernels, and launches.  No device
 // memory is allocated here; every buffer belongs to the caller.
 #include <algorithm>
-#include <array>
+#include <atomic>
 #include <climits>
 #include <cstring>
 #include <map>
@@ -89,42 +89,58 @@ class Staging {
     size_t cap = 0;
     cudaEvent_t ev = nullptr;
   };
+  // A slot is free once the event recorded behind its last copy has completed
+  // (queried, never waited on).  When no slot of the device's ring is free the
+  // ring grows by one, so the host never blocks on the GPU here: the ring ends
+  // as deep as the most uploads the caller ever kept in flight.
   struct Ring {
-    std::array<Slot, 4> slot;
-    int next = 0;
+    std::vector<Slot*> slot;
+    size_t cap = size_t(4) << 20;   // capacity of every slot made from now on
   };
+  static bool idle(const Slot& sl) { return !sl.ev || cudaEventQuery(sl.ev) == cudaSuccess; }
+  static cudaError_t pin(Slot& sl, size_t cap) {
+    if (sl.p) cudaFreeHost(sl.p);
+    sl.p = sl.d = nullptr;
+    sl.cap = 0;
+    cudaError_t e = cudaHostAlloc(&sl.p, cap, cudaHostAllocMapped | cudaHostAllocPortable);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaHostGetDevicePointer(&sl.d, sl.p, 0)) != cudaSuccess) {
+      cudaFreeHost(sl.p);
+      sl.p = nullptr;
+      return e;
+    }
+    sl.cap = cap;
+    return cudaSuccess;
+  }
   cudaError_t take(size_t n, Slot** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     Ring& ring = rings_[dev];
-    Slot& sl = ring.slot[ring.next];
-    ring.next = (ring.next + 1) % (int)ring.slot.size();
-    if (sl.ev && (e = cudaEventSynchronize(sl.ev)) != cudaSuccess) return e;
-    if (!sl.ev && (e = cudaEventCreateWithFlags(&sl.ev, cudaEventDisableTiming)) != cudaSuccess) return e;
-    if (sl.cap < n) {
+    if (ring.cap < n) {
       // Pinning host memory stalls transfers in flight on the GPU's host link
       // (a caller's input copy of 2.75 GB took 174 ms instead of 13 ms when it
-      // overlapped one), so every slot of the ring grows at once, to a power of
-      // two of at least 4 MB: after the first calls nothing is pinned again.
-      size_t cap = size_t(4) << 20;
-      while (cap < n) cap <<= 1;
-      for (Slot& o : ring.slot) {
-        if (o.cap >= cap) continue;
-        if (o.ev && &o != &sl && (e = cudaEventSynchronize(o.ev)) != cudaSuccess) return e;
-        if (o.p) cudaFreeHost(o.p);
-        o.p = o.d = nullptr;
-        o.cap = 0;
-        if ((e = cudaHostAlloc(&o.p, cap, cudaHostAllocMapped | cudaHostAllocPortable)) != cudaSuccess) return e;
-        if ((e = cudaHostGetDevicePointer(&o.d, o.p, 0)) != cudaSuccess) {
-          cudaFreeHost(o.p);
-          o.p = nullptr;
-          return e;
-        }
-        o.cap = cap;
-      }
+      // overlapped one), so every idle slot grows at once, to a power of two of
+      // at least 4 MB: after the first calls nothing is pinned again.
+      while (ring.cap < n) ring.cap <<= 1;
+      for (Slot* o : ring.slot)
+        if (o->cap < ring.cap && idle(*o) && (e = pin(*o, ring.cap)) != cudaSuccess) return e;
     }
-    *out = &sl;
+    Slot* sl = nullptr;
+    for (Slot* o : ring.slot)
+      if (o->cap >= n && idle(*o)) { sl = o; break; }
+    if (!sl) {
+      for (Slot* o : ring.slot)   // an idle slot left small by an earlier growth
+        if (idle(*o)) { sl = o; break; }
+      if (sl && (e = pin(*sl, ring.cap)) != cudaSuccess) return e;
+    }
+    if (!sl) {
+      ring.slot.push_back(new Slot());
+      sl = ring.slot.back();
+      if ((e = pin(*sl, ring.cap)) != cudaSuccess) return e;
+    }
+    if (!sl->ev && (e = cudaEventCreateWithFlags(&sl->ev, cudaEventDisableTiming)) != cudaSuccess) return e;
+    *out = sl;
     return cudaSuccess;
   }
   std::mutex mu_;
@@ -144,7 +160,27 @@ Staging& staging() {
 }
 
 constexpr size_t kAlign = 256;
+// Every workspace of the selection, recall and index calls starts with this
+// header; its first word is the call's device error word (zeroed by the call's
+// plan upload, set by a kernel whose bounded wait gave up), which
+// saki_workspace_status reads.
+constexpr size_t kHeader = 256;
 constexpr int kNumSMs = 152;
+
+// One-shot stall for the failure-reporting test (saki_debug_inject_stall): the
+// next launch of the armed kernel kind gets a producer that issues no loads.
+std::atomic<int> g_stall_kind{0};
+int take_stall(int kind) {
+  int expect = kind;
+  return g_stall_kind.compare_exchange_strong(expect, 0) ? 1 : 0;
+}
+
+// Work lists are uploaded from host memory that lives only for the call, so a
+// captured call would replay a copy from freed memory: refuse stream capture.
+bool capturing(cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  return cudaStreamIsCapturing(s, &st) == cudaSuccess && st != cudaStreamCaptureStatusNone;
+}
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 inline saki_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA; }
 inline bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -163,7 +199,7 @@ saki_status check_cfg(const saki_config* c) {
   if (c->center != 0 && c->center != 1) return SAKI_ERR_INVALID_ARGUMENT;
   if (!(c->eig_floor_rel >= 0.f && c->eig_floor_rel < 1.f)) return SAKI_ERR_INVALID_ARGUMENT;
   if (c->max_sweeps < 0) return SAKI_ERR_INVALID_ARGUMENT;
-  if (c->flags & ~SAKI_FLAG_SORTED) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->flags & ~(SAKI_FLAG_SORTED | SAKI_FLAG_CHECK)) return SAKI_ERR_INVALID_ARGUMENT;
   if (c->method != SAKI_METHOD_SAKI && c->method != SAKI_METHOD_KEY_PCA && c->method != SAKI_METHOD_WEIGHT_SVD)
     return SAKI_ERR_INVALID_ARGUMENT;
   return SAKI_OK;
@@ -268,13 +304,13 @@ Plan make_plan(const saki_layout* L, int Hq, int kp, int dtype, int P, bool seed
   }
   p.vis.resize(T);
   for (int64_t t = 0; t < T; ++t) p.vis[t] = (int32_t)L->q_visible[t];
-  p.off_items = 0;
-  p.off_merges = align_up(p.items.size() * sizeof(ScoreItem));
+  p.off_err = 0;   // the header's error word, zeroed by the upload
+  p.off_items = kHeader;
+  p.off_merges = p.off_items + align_up(p.items.size() * sizeof(ScoreItem));
   p.off_sitems = p.off_merges + align_up(p.merges.size() * sizeof(MergeItem));
   p.off_smerges = p.off_sitems + align_up(p.sitems.size() * sizeof(ScoreItem));
   p.off_vis = p.off_smerges + align_up(p.smerges.size() * sizeof(MergeItem));
-  p.off_err = p.off_vis + align_up(p.vis.size() * sizeof(int32_t));   // zeroed by the upload
-  p.staged = p.off_err + sizeof(int);
+  p.staged = p.off_vis + p.vis.size() * sizeof(int32_t);
   p.off_cand = align_up(p.staged);
   p.off_scand = p.off_cand + align_up((size_t)p.cand_slots * Hq * kp * sizeof(uint64_t));
   p.off_seed = p.off_scand + align_up((size_t)p.scand_slots * Hq * kp * sizeof(uint64_t));
@@ -362,9 +398,9 @@ TcPlan make_tc_plan(const saki_layout* L, int Hq, int P, bool with_qnu) {
                    [](const TcTile& a, const TcTile& b) { return a.vis_max > b.vis_max; });
   p.vis.resize(T);
   for (int64_t t = 0; t < T; ++t) p.vis[t] = (int32_t)L->q_visible[t];
-  p.off_vis = align_up(p.tiles.size() * sizeof(TcTile));
-  p.off_err = p.off_vis + align_up(p.vis.size() * sizeof(int32_t));
-  p.staged = p.off_err + sizeof(int);
+  p.off_err = 0;   // the header's error word, zeroed by the upload
+  p.off_vis = kHeader + align_up(p.tiles.size() * sizeof(TcTile));
+  p.staged = p.off_vis + p.vis.size() * sizeof(int32_t);
   p.off_w = align_up(p.staged);
   p.off_qnu = p.off_w + align_up((size_t)Hq * 3 * P * kD * 2);
   p.bytes = p.off_qnu + (with_qnu ? align_up((size_t)Hq * T * sizeof(float)) : 0);
@@ -390,7 +426,7 @@ bool use_tc(const saki_config* c, const saki_layout* L, int P) {
 
 saki_status upload_tc_plan(const TcPlan& p, char* ws, cudaStream_t s) {
   std::vector<char> host(p.staged, 0);
-  if (!p.tiles.empty()) std::memcpy(host.data(), p.tiles.data(), p.tiles.size() * sizeof(TcTile));
+  if (!p.tiles.empty()) std::memcpy(host.data() + kHeader, p.tiles.data(), p.tiles.size() * sizeof(TcTile));
   if (!p.vis.empty()) std::memcpy(host.data() + p.off_vis, p.vis.data(), p.vis.size() * sizeof(int32_t));
   return staging().upload(ws, host.data(), p.staged, s) == cudaSuccess ? SAKI_OK : SAKI_ERR_CUDA;
 }
@@ -422,7 +458,7 @@ saki_status run_tc(const saki_config* cfg, const saki_layout* layout, const TcPl
   L.Hk = cfg->num_kv_heads;
   L.num_sms = num_sms();
   TcArgs& a = L.args;
-  a.tiles = reinterpret_cast<const TcTile*>(ws);
+  a.tiles = reinterpret_cast<const TcTile*>(ws + kHeader);
   a.vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
   a.qnu = qnu;
   a.idx = idx;
@@ -436,6 +472,7 @@ saki_status run_tc(const saki_config* cfg, const saki_layout* layout, const TcPl
   a.k = cfg->topk;
   a.exact = exact ? 1 : 0;
   a.sorted = (cfg->flags & SAKI_FLAG_SORTED) ? 1 : 0;
+  a.stall = take_stall(exact ? SAKI_KERNEL_EXACT : SAKI_KERNEL_SELECT);
   KernelTimer kt(exact ? SAKI_KERNEL_EXACT : SAKI_KERNEL_SELECT, s);
   return cuda_status(launch_score_tc(L, s));
 }
@@ -448,15 +485,15 @@ BuildWs build_ws(const saki_config* c, int64_t N) {
   BuildWs w{};
   const int G = c->num_q_heads / c->num_kv_heads;
   w.tc = c->dtype == SAKI_BF16 && !c->center && build_tc_supported(c->rank, G) && N > 0;
-  if (!w.tc) { w.bytes = kAlign; return w; }
+  w.off_err = 0;
+  if (!w.tc) { w.bytes = kHeader; return w; }
   const int ncb = (G * c->rank + 127) / 128;
   const int64_t tiles = (N + 127) / 128;
   for (int g = 0; g < c->num_kv_heads; ++g)
     for (int cb = 0; cb < ncb; ++cb)
       for (int64_t t = 0; t < tiles; t += 32)
         w.items.push_back(BuildItem{g, cb, (int32_t)t, (int32_t)std::min<int64_t>(tiles, t + 32)});
-  w.off_err = align_up(w.items.size() * sizeof(BuildItem));
-  w.off_w = w.off_err + kAlign;
+  w.off_w = kHeader + align_up(w.items.size() * sizeof(BuildItem));
   w.bytes = w.off_w + align_up(build_tc_workspace(c->num_q_heads, c->rank));
   return w;
 }
@@ -489,9 +526,37 @@ size_t recall_extra(const saki_config* c, int64_t T, bool with_idx) {
          (with_idx ? align_up((size_t)c->num_q_heads * T * c->topk * sizeof(int32_t)) : 0);
 }
 
+// Read the header's error word once the stream has run up to here.
+saki_status read_status(const void* workspace, cudaStream_t s) {
+  int word = 0;
+  if (staging().download_sync(&word, workspace, sizeof(int), s) != cudaSuccess) return SAKI_ERR_CUDA;
+  return word ? SAKI_ERR_TIMEOUT : SAKI_OK;
+}
+
+// A call's return: its launch status, then, with SAKI_FLAG_CHECK, the device
+// status of what it launched.
+saki_status finish(const saki_config* cfg, saki_status st, const void* workspace, cudaStream_t s) {
+  if (st != SAKI_OK || !(cfg->flags & SAKI_FLAG_CHECK)) return st;
+  return read_status(workspace, s);
+}
+
 }  // namespace
 
 extern "C" {
+
+saki_status saki_workspace_status(const void* workspace, saki_stream stream) {
+  if (!workspace || !al16(workspace)) return SAKI_ERR_INVALID_ARGUMENT;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
+  return read_status(workspace, s);
+}
+
+saki_status saki_debug_inject_stall(int32_t kind) {
+  if (kind != 0 && kind != SAKI_KERNEL_SELECT && kind != SAKI_KERNEL_EXACT && kind != SAKI_KERNEL_BUILD)
+    return SAKI_ERR_INVALID_ARGUMENT;
+  g_stall_kind.store(kind);
+  return SAKI_OK;
+}
 
 const char* saki_status_string(saki_status s) {
   switch (s) {
@@ -547,6 +612,7 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
   const FitWs w = fit_ws(cfg);
   if (workspace_bytes < w.bytes) return SAKI_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
   char* ws = static_cast<char*>(workspace);
   const int Hq = cfg->num_q_heads, Hk = cfg->num_kv_heads, nm = Hq + Hk;
   float* S = reinterpret_cast<float*>(ws + w.S);
@@ -622,20 +688,34 @@ saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const v
   if (w.tc) {
     if (!workspace) return SAKI_ERR_INVALID_ARGUMENT;
     if (workspace_bytes < w.bytes) return SAKI_ERR_WORKSPACE;
+    if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
     char* ws = static_cast<char*>(workspace);
-    std::vector<char> host(w.off_w, 0);
-    std::memcpy(host.data(), w.items.data(), w.items.size() * sizeof(BuildItem));
+    std::vector<char> host(kHeader + w.items.size() * sizeof(BuildItem), 0);
+    std::memcpy(host.data() + kHeader, w.items.data(), w.items.size() * sizeof(BuildItem));
     if ((st = cuda_status(staging().upload(ws, host.data(), host.size(), s))) != SAKI_OK) return st;
-    KernelTimer kt(SAKI_KERNEL_BUILD, s);
-    return cuda_status(launch_build_tc(K, R, sketch, total_keys, cfg->num_q_heads,
+    {
+      KernelTimer kt(SAKI_KERNEL_BUILD, s);
+      st = cuda_status(launch_build_tc(K, R, sketch, total_keys, cfg->num_q_heads,
                                        cfg->num_q_heads / cfg->num_kv_heads, cfg->rank,
-                                       reinterpret_cast<const BuildItem*>(ws), (int)w.items.size(), ws + w.off_w,
-                                       reinterpret_cast<int*>(ws + w.off_err), num_sms(), s));
+                                       reinterpret_cast<const BuildItem*>(ws + kHeader), (int)w.items.size(),
+                                       ws + w.off_w, reinterpret_cast<int*>(ws + w.off_err),
+                                       take_stall(SAKI_KERNEL_BUILD), num_sms(), s));
+    }
+    return finish(cfg, st, workspace, s);
   }
-  KernelTimer kt(SAKI_KERNEL_BUILD, s);
-  return cuda_status(launch_build_generic(K, R, cfg->center ? mu : nullptr, sketch, total_keys, cfg->num_q_heads,
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
+  // the CUDA-core build has no bounded wait: its status is always ok, and a
+  // workspace passed along gets a zeroed header so that it reads so
+  if (workspace && workspace_bytes >= kHeader &&
+      (st = cuda_status(cudaMemsetAsync(workspace, 0, sizeof(int), s))) != SAKI_OK)
+    return st;
+  {
+    KernelTimer kt(SAKI_KERNEL_BUILD, s);
+    st = cuda_status(launch_build_generic(K, R, cfg->center ? mu : nullptr, sketch, total_keys, cfg->num_q_heads,
                                           cfg->num_q_heads / cfg->num_kv_heads, cfg->rank, cfg->center,
                                           cfg->dtype, s));
+  }
+  return workspace ? finish(cfg, st, workspace, s) : st;
 }
 
 saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, const void* Q, const float* L,
@@ -656,11 +736,13 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
   if (use_tc(cfg, layout, cfg->rank)) {
     const TcPlan tp = make_tc_plan(layout, cfg->num_q_heads, cfg->rank, true);
     if (workspace_bytes < tp.bytes) return SAKI_ERR_WORKSPACE;
-    return run_tc(cfg, layout, tp, cfg->rank, false, Q, L, sketch, nu, idx, score, ws, s);
+    if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
+    return finish(cfg, run_tc(cfg, layout, tp, cfg->rank, false, Q, L, sketch, nu, idx, score, ws, s), ws, s);
   }
   const int kp = kp_of(cfg->topk);
   const Plan p = plan_for(layout, cfg->num_q_heads, kp, cfg->dtype, cfg->rank, workspace_bytes, 0);
   if (workspace_bytes < p.bytes) return SAKI_ERR_WORKSPACE;
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
   if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
   ScoreArgs a{};
   a.Q = Q; a.X = sketch; a.W = L; a.nu = nu;
@@ -676,8 +758,12 @@ saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, c
   a.exact = 0;
   a.n_items = (int32_t)p.items.size();
   a.n_merges = (int32_t)p.merges.size();
-  KernelTimer kt(SAKI_KERNEL_SELECT, s);
-  return cuda_status(run_plan(a, p, ws, cfg->dtype, kp, s));
+  a.stall = take_stall(SAKI_KERNEL_SELECT);
+  {
+    KernelTimer kt(SAKI_KERNEL_SELECT, s);
+    st = cuda_status(run_plan(a, p, ws, cfg->dtype, kp, s));
+  }
+  return finish(cfg, st, ws, s);
 }
 
 saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64_t min_visible, const void* Q,
@@ -701,6 +787,7 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
   const size_t need = base + extra;
   if (workspace_bytes < need) return SAKI_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;   // after every host-side check above
   char* ws = static_cast<char*>(workspace);
   unsigned long long* counters = reinterpret_cast<unsigned long long*>(ws + base);
   int32_t* ie = idx_exact ? idx_exact
@@ -708,9 +795,12 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
                                                                             sizeof(unsigned long long)));
   if (tc) {
     if ((st = run_tc(cfg, layout, tp, kD, true, Q, A, K, nullptr, ie, nullptr, ws, s)) != SAKI_OK) return st;
-    return cuda_status(launch_recall(idx_approx, ie, reinterpret_cast<const int32_t*>(ws + tp.off_vis), T,
-                                     cfg->num_q_heads, cfg->topk, min_visible, counters, recall, s));
+    return finish(cfg,
+                  cuda_status(launch_recall(idx_approx, ie, reinterpret_cast<const int32_t*>(ws + tp.off_vis), T,
+                                            cfg->num_q_heads, cfg->topk, min_visible, counters, recall, s)),
+                  ws, s);
   }
+  if (T == 0 && (st = cuda_status(cudaMemsetAsync(ws, 0, sizeof(int), s))) != SAKI_OK) return st;
   if (T > 0) {
     if ((st = upload_plan(p, ws, s)) != SAKI_OK) return st;
     ScoreArgs a{};
@@ -727,12 +817,15 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
     a.exact = 1;
     a.n_items = (int32_t)p.items.size();
     a.n_merges = (int32_t)p.merges.size();
+    a.stall = take_stall(SAKI_KERNEL_EXACT);
     KernelTimer kt(SAKI_KERNEL_EXACT, s);
     if ((st = cuda_status(run_plan(a, p, ws, cfg->dtype, kp, s))) != SAKI_OK) return st;
   }
   const int32_t* vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
-  return cuda_status(launch_recall(idx_approx, ie, vis, T, cfg->num_q_heads, cfg->topk, min_visible, counters,
-                                   recall, s));
+  return finish(cfg,
+                cuda_status(launch_recall(idx_approx, ie, vis, T, cfg->num_q_heads, cfg->topk, min_visible, counters,
+                                          recall, s)),
+                ws, s);
 }
 
 }  // extern "C"

@@ -37,7 +37,7 @@ __device__ __forceinline__ bool wait_noabort(uint64_t* bar, uint32_t parity) {
 __global__ void __launch_bounds__(192, 1)
     build_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmB,
                     const BuildItem* items, int n_items, int64_t N, int ncol_total, int r, int G,
-                    __nv_bfloat16* sketch, int* err) {
+                    __nv_bfloat16* sketch, int* err, int stall) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
   uint8_t* sA = smem;
@@ -89,7 +89,7 @@ __global__ void __launch_bounds__(192, 1)
       int nb = 0;          // B loads issued
       int prev_g = -1, prev_cb = -1;
       bool ok = true;
-      for (int item = i_begin; item < i_end && ok; ++item) {
+      for (int item = stall ? i_end : i_begin; item < i_end && ok; ++item) {
         const BuildItem it = items[item];
         if (it.g != prev_g || it.cb != prev_cb) {
           if (nb > 0 && !(ok = tc::mbar_wait(bfree, (nb - 1) & 1, abort_f))) break;
@@ -271,8 +271,8 @@ bool build_tc_supported(int r, int G) {
 size_t build_tc_workspace(int Hq, int r) { return (size_t)Hq * 3 * r * kD * 2; }
 
 cudaError_t launch_build_tc(const void* K, const float* R, void* sketch, int64_t N, int Hq, int G, int r,
-                            const BuildItem* items, int n_items, void* wsplit, int* err, int num_sms,
-                            cudaStream_t s) {
+                            const BuildItem* items, int n_items, void* wsplit, int* err, int stall,
+                            int num_sms, cudaStream_t s) {
   if (n_items == 0) return cudaSuccess;
   const int64_t n = (int64_t)Hq * r * kD;
   const int blocks = (int)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
@@ -290,7 +290,7 @@ cudaError_t launch_build_tc(const void* K, const float* R, void* sketch, int64_t
   const int grid = n_items < num_sms ? n_items : num_sms;
   note_launch();
   build_tc_kernel<<<grid, 192, kBuildSmem, s>>>(mK, mB, items, n_items, N, ncol_total, r, G,
-                                                static_cast<__nv_bfloat16*>(sketch), err);
+                                                static_cast<__nv_bfloat16*>(sketch), err, stall);
   return cudaGetLastError();
 }
 

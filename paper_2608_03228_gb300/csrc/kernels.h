@@ -80,6 +80,7 @@ struct ScoreArgs {
   int64_t T, N;
   int32_t Hq, G, P, k, exact, n_items, n_merges;
   int32_t sample;       // tensor-core variant only: write each query's kp best group maxima (a sample pass)
+  int32_t stall;        // test hook: the tensor-core variant's producer issues no loads (its waits run out)
 };
 
 // generic CUDA-core scoring (any rank, f32 or bf16)
@@ -141,6 +142,7 @@ struct TcArgs {
   int* err;             // set to 1 if a bounded wait gave up
   int64_t T, N;
   int32_t n_items, Hq, G, k, exact, sorted;
+  int32_t stall;        // test hook: the producer issues no loads, so the consumers' bounded waits run out
 };
 
 struct TcLaunch {
@@ -165,7 +167,7 @@ struct BuildItem {
 bool build_tc_supported(int r, int G);
 size_t build_tc_workspace(int Hq, int r);
 cudaError_t launch_build_tc(const void* K, const float* R, void* sketch, int64_t N, int Hq, int G, int r,
-                            const BuildItem* items, int n_items, void* wsplit, int* err, int num_sms,
-                            cudaStream_t s);
+                            const BuildItem* items, int n_items, void* wsplit, int* err, int stall,
+                            int num_sms, cudaStream_t s);
 
 }  // namespace saki

@@ -418,7 +418,7 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
       tc::prefetch_tmap(&tmX);
       const int64_t xrow = (int64_t)(a.exact ? h / a.G : h) * a.N + it.key_base + it.key_lo;
       int issued = 0;
-      for (int i = 0; i < ntiles; ++i) {
+      for (int i = 0; i < (a.stall ? 0 : ntiles); ++i) {
         const int st = i % C::STAGES;
         if (!tc::mbar_wait(empty + st, ((i / C::STAGES) & 1) ^ 1, abort_f)) break;
         tc::mbar_arrive_expect_tx(full + st, C::STAGE_BYTES);

@@ -659,7 +659,7 @@ __global__ void __launch_bounds__(192, 1)
       tc::prefetch_tmap(&tmX);
       uint32_t sc = 0;
       int it = 0, q_issued = 0;
-      for (int item = blockIdx.x; item < a.n_items; item += gridDim.x, ++it) {
+      for (int item = a.stall ? a.n_items : blockIdx.x; item < a.n_items; item += gridDim.x, ++it) {
         const TcTile t = a.tiles[item / Hq];
         const int h = item % Hq;
         if (it > 0 && !tc::mbar_wait(afree, (it - 1) & 1, abort_f)) break;

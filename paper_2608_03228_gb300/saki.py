@@ -19,7 +19,7 @@ if not os.path.exists(_LIB_PATH):
 _lib = ctypes.CDLL(_LIB_PATH)
 
 SAKI_F32, SAKI_BF16 = 0, 1
-SAKI_FLAG_SORTED = 1
+SAKI_FLAG_SORTED, SAKI_FLAG_CHECK = 1, 2
 SAKI_METHOD_SAKI, SAKI_METHOD_KEY_PCA, SAKI_METHOD_WEIGHT_SVD = 0, 1, 2
 METHODS = {"saki": SAKI_METHOD_SAKI, "key_pca": SAKI_METHOD_KEY_PCA, "weight_svd": SAKI_METHOD_WEIGHT_SVD}
 SAKI_OP_FIT, SAKI_OP_BUILD_INDEX, SAKI_OP_SCORE_TOPK, SAKI_OP_RECALL = 0, 1, 2, 3
@@ -27,7 +27,8 @@ STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED
           4: "SAKI_ERR_NUMERIC", 5: "SAKI_ERR_NOT_CONVERGED", 6: "SAKI_ERR_WORKSPACE", 7: "SAKI_ERR_TIMEOUT"}
 EXPORTS = ("saki_workspace_size", "saki_fit", "saki_build_index", "saki_score_topk", "saki_recall",
            "saki_status_string", "saki_version", "saki_score_topk_noalloc", "saki_launch_count",
-           "saki_kernel_timer_start", "saki_kernel_timer_stop")
+           "saki_kernel_timer_start", "saki_kernel_timer_stop", "saki_workspace_status", "saki_noalloc_status",
+           "saki_debug_inject_stall")
 SAKI_KERNEL_SELECT, SAKI_KERNEL_EXACT, SAKI_KERNEL_FIT, SAKI_KERNEL_MOMENTS, SAKI_KERNEL_BUILD, SAKI_KERNEL_FACTOR = (
     1, 2, 3, 4, 5, 6)
 SAKI_NOALLOC_SCRATCH_BYTES = 16 << 20
@@ -58,6 +59,12 @@ _lib.saki_recall.restype = ctypes.c_int
 _lib.saki_recall.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout), _i64] + [_vp] * 7 + [_sz, _vp]
 _lib.saki_score_topk_noalloc.restype = ctypes.c_int
 _lib.saki_score_topk_noalloc.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout)] + [_vp] * 6 + [_vp]
+_lib.saki_workspace_status.restype = ctypes.c_int
+_lib.saki_workspace_status.argtypes = [_vp, _vp]
+_lib.saki_noalloc_status.restype = ctypes.c_int
+_lib.saki_noalloc_status.argtypes = [_vp]
+_lib.saki_debug_inject_stall.restype = ctypes.c_int
+_lib.saki_debug_inject_stall.argtypes = [_i32]
 _lib.saki_status_string.restype = ctypes.c_char_p
 _lib.saki_status_string.argtypes = [ctypes.c_int]
 _lib.saki_version.restype = ctypes.c_char_p
@@ -148,6 +155,21 @@ def saki_kernel_timer_stop(kind: int) -> tuple[float, int]:
     ms, n = ctypes.c_double(0.0), _i64(0)
     _check(_lib.saki_kernel_timer_stop(kind, ctypes.byref(ms), ctypes.byref(n)), "saki_kernel_timer_stop")
     return ms.value, int(n.value)
+
+
+def saki_workspace_status(workspace, stream=None) -> None:
+    """Raise SakiError(SAKI_ERR_TIMEOUT) if a kernel of the last selection, recall
+    or index call on this workspace gave up a bounded wait (synchronises stream)."""
+    _check(_lib.saki_workspace_status(_ptr(workspace), _stream(stream)), "saki_workspace_status")
+
+
+def saki_noalloc_status(stream=None) -> None:
+    _check(_lib.saki_noalloc_status(_stream(stream)), "saki_noalloc_status")
+
+
+def saki_debug_inject_stall(kind: int) -> None:
+    """Test hook: the next tensor-core launch of this kernel kind stalls its producer."""
+    _check(_lib.saki_debug_inject_stall(kind), "saki_debug_inject_stall")
 
 
 def saki_workspace_size(cfg: Config, op: int, layout: HostLayout | None = None, n_calib: int = 0,

@@ -79,6 +79,20 @@ WORKLOADS = {
     "qwen25_7b_t4096_r32": Workload("qwen25_7b_t4096_r32", 28 * 28, 28 * 4, rank=32,
                                     n_calib=4096, seq_lens=(4096,), spikes=(2, 16),
                                     seed=2, layers=28),
+    # the rank sweep at that shape (Tab. 2 reports r = 16, 32, 64)
+    "qwen25_7b_t4096_r16": Workload("qwen25_7b_t4096_r16", 28 * 28, 28 * 4, rank=16,
+                                    n_calib=4096, seq_lens=(4096,), spikes=(2, 16),
+                                    seed=2, layers=28),
+    "qwen25_7b_t4096_r64": Workload("qwen25_7b_t4096_r64", 28 * 28, 28 * 4, rank=64,
+                                    n_calib=4096, seq_lens=(4096,), spikes=(2, 16),
+                                    seed=2, layers=28),
+    # the calibration-length sweep at r = 32 (Fig. 2A: 512 to 32,768 tokens)
+    "qwen25_7b_t4096_r32_n512": Workload("qwen25_7b_t4096_r32_n512", 28 * 28, 28 * 4, rank=32,
+                                         n_calib=512, seq_lens=(4096,), spikes=(2, 16),
+                                         seed=2, layers=28),
+    "qwen25_7b_t4096_r32_n32768": Workload("qwen25_7b_t4096_r32_n32768", 28 * 28, 28 * 4, rank=32,
+                                           n_calib=32768, seq_lens=(4096,), spikes=(2, 16),
+                                           seed=2, layers=28),
     # Llama-3.2-3B shape: 28 layers x 24 query heads / 8 KV heads
     "llama32_3b_t4096_r32": Workload("llama32_3b_t4096_r32", 28 * 24, 28 * 8, rank=32,
                                      n_calib=4096, seq_lens=(4096,), spikes=(2, 16),

@@ -56,6 +56,13 @@ def test_ctypes_layout_matches_c(lib, tmp_path):
                     ctypes.sizeof(lib.Layout), lib.Layout.q_visible.offset, lib.Config.method.offset]
 
 
+def test_status_and_stall_hook_argument_checks(lib):
+    assert lib._lib.saki_workspace_status(None, None) == 1      # no workspace: rejected before any CUDA call
+    for kind in (4, 6, 99, -1):                                # only the tensor-core kernels with a producer
+        assert lib._lib.saki_debug_inject_stall(kind) == 1
+    assert lib._lib.saki_debug_inject_stall(0) == 0            # disarm
+
+
 def test_status_strings(lib):
     for code in range(8):
         assert lib.saki_status_string(code)
