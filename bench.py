@@ -407,7 +407,7 @@ def rooflines(w, pk, ktime, g):
     out = {}
 
     def entry(name, bound, work, unit, peak, note, peak_name):
-        tot, cnt = ktime[name]
+        tot, cnt = ktime.get(name, (0.0, 0))
         if cnt == 0:
             return
         ms = tot / cnt
