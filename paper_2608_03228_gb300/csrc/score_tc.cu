@@ -8,16 +8,18 @@
 //      TMEM is split into u_hi + u_lo (bf16 each) and written, swizzled, as the
 //      A operand of the main loop (keeping u to ~16 bits, far below the score
 //      tolerance);
-//   2. main loop over key tiles of the visible range: TMA brings NT key rows
-//      (codes, or raw keys for the exact scores) into a ring of shared-memory
-//      stages; one thread issues tcgen05.mma (M = 128 queries, N = NT keys,
-//      K = P, twice: u_hi and u_lo) into one of two TMEM accumulators;
+//   2. main loop over 64-key tiles of the visible range: TMA brings the key
+//      rows (codes, or raw keys for the exact scores) into a ring of
+//      shared-memory stages; one thread issues tcgen05.mma (M = 128 queries,
+//      N = 64 keys, K = P, twice: u_hi and u_lo) into a ring of four TMEM
+//      accumulators;
 //   3. four epilogue warps own one query row per thread (TMEM lane = row) and
 //      select in two passes over the same scores (the key tiles are multiplied
-//      twice; the tensor core has ample headroom): pass 1 keeps per-row maxima
-//      of 128 key groups and derives a certified lower bound tau on the row's
-//      k-th best score; pass 2 appends the visible keys scoring >= tau to the
-//      row's candidate column in shared memory.  The T x N score matrix is never
+//      twice; the tensor core has ample headroom): pass 1 folds every score
+//      into the row's 128 key-group maxima (one three-input maximum per two
+//      scores) and derives a certified lower bound tau on the row's k-th best
+//      score; pass 2 appends the visible keys scoring >= tau to the row's
+//      candidate column in shared memory.  The T x N score matrix is never
 //      stored.
 //   4. exact top-k of the remaining candidates per row, written coalesced.
 // Roles: warp 0 = TMA producer, warp 1 = TMEM owner + MMA issuer, warps 2-5 =
@@ -37,7 +39,7 @@ namespace saki {
 namespace {
 
 constexpr int kLdc = 129;   // candidate column stride (words): conflict-free per-row scans and row reads
-constexpr int kGroups = 64;   // pass-1 key groups per row (key offset mod 64); two maxima kept per group
+constexpr int kGroups = 128;  // pass-1 key groups per row, one maximum each
 constexpr int kScr = 36;      // per-row scratch stride (words): 32 scores + pad, conflict-free 16-byte stores
 
 template <int P>
@@ -53,7 +55,12 @@ struct TcCfg {
   // the room for its operands and keeps 16-bit indices in their own array
   static constexpr bool WIDE = P <= 64;
   static constexpr int STAGES = P == 128 ? 2 : 4;
-  static constexpr int CAP = P == 128 ? 144 : 136;               // candidate slots per row (multiple of 8)
+  // candidate slots per row: as many as the shared-memory budget leaves (a
+  // multiple of 8); bytes per slot and row: a 4-byte score plus a 4-byte (ranks
+  // up to 64) or 2-byte (rank 128) key index
+  static constexpr int FIXED_BYTES = (2 * 128 * P * 2 > 32768 ? 2 * 128 * P * 2 : 32768) + STAGES * 64 * P * 2 +
+                                     128 * kScr * 4 + 256 + 1024;
+  static constexpr int CAP = P == 128 ? 144 : ((232448 - FIXED_BYTES) / (kLdc * 8)) / 8 * 8;
   static constexpr int KB = P == 128 ? 2 : 1;                 // 64-wide K blocks
   static constexpr int KW = P == 128 ? 64 : P;                // K width of one block
   static constexpr int KK = KW / 16;                          // MMA K steps per block
@@ -73,7 +80,7 @@ struct TcCfg {
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
   static_assert(STAGE_BYTES >= P * 128, "a projection chunk must fit a stage");
   static_assert(CAP % 8 == 0 && CAP >= 64 + 32, "candidate capacity: k + one chunk of appends");
-  static_assert(NT % 64 == 0, "a key tile covers whole key groups");
+  static_assert(NT == 64, "pass 1 folds a tile's two 32-key halves into one block of 32 groups");
   static_assert(NT <= BUFC && P <= BUFC && TMEM_COLS <= 512, "a ring buffer holds a tile's or a projection's columns");
   static_assert(SMEM <= 232448, "shared memory budget");
   static_assert(OFF_STAGE % 1024 == 0 && STAGE_BYTES % 1024 == 0, "swizzled TMA tiles sit on 1024-byte boundaries");
@@ -422,106 +429,111 @@ __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int
   }
 }
 
-// Pass 1: fold 32 scores of a row (keys j0 .. j0+31, key groups gb .. gb+31)
-// into the two highest scores of each group (g1 >= g2); keys the row cannot see
-// count as -inf.  Called from fully unrolled loops, so gb is a constant and the
-// maxima stay in registers.
-__device__ __forceinline__ void fold32(const uint32_t (&r)[32], float (&g1)[kGroups], float (&g2)[kGroups], int gb,
-                                       int j0, int vis) {
-  float v[32];
-#pragma unroll
-  for (int u = 0; u < 32; ++u) v[u] = __uint_as_float(r[u]);
-  if (j0 + 32 > vis) {
-#pragma unroll
-    for (int u = 0; u < 32; ++u)
-      if (j0 + u >= vis) v[u] = -INFINITY;
-  }
+// Three-input maximum (one instruction on sm_100 and later).
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Scores of a key tile (keys j0 .. j0+63 of the row: ra holds the first 32, rb
+// the last 32) at or past the row's visible count become -inf.  Only tiles that
+// cross some row's visibility boundary take this path.
+__device__ __forceinline__ void mask_tile(uint32_t (&ra)[32], uint32_t (&rb)[32], int j0, int vis) {
+  const uint32_t ninf = __float_as_uint(-INFINITY);
 #pragma unroll
   for (int u = 0; u < 32; ++u) {
-    const float hi = fmaxf(g1[gb + u], v[u]);
-    g2[gb + u] = fmaxf(g2[gb + u], fminf(g1[gb + u], v[u]));
-    g1[gb + u] = hi;
+    ra[u] = j0 + u < vis ? ra[u] : ninf;
+    rb[u] = j0 + 32 + u < vis ? rb[u] : ninf;
   }
 }
 
-// The certified bound of pass 1: a value tau with at least k of the 128 kept
-// values >= tau, taken from a sorted sample of 32 of them (the highest sample
-// that qualifies), or -inf if none does (then every visible key is a candidate).
-__device__ __forceinline__ float select_tau(const float (&g1)[kGroups], const float (&g2)[kGroups], int k) {
+// Pass 1: fold a tile into 32 of the row's 128 group maxima.  Key j belongs to
+// group 32 ((j / 64) mod 4) + (j mod 32), so a tile's keys j and j + 32 share a
+// group and one three-input maximum folds both (half an instruction per
+// score).  Called from a loop unrolled over the tile index mod 4, so gb is a
+// constant and the maxima stay in registers.
+__device__ __forceinline__ void fold64(const uint32_t (&ra)[32], const uint32_t (&rb)[32], float (&g)[kGroups],
+                                       int gb) {
+#pragma unroll
+  for (int u = 0; u < 32; ++u) g[gb + u] = max3f(g[gb + u], __uint_as_float(ra[u]), __uint_as_float(rb[u]));
+}
+
+// The certified bound of pass 1.  The 128 group maxima are scores of distinct
+// visible keys, so any value tau with at least k of them >= tau bounds the row's
+// k-th best score from below.  32 of them, sorted, give pivots; one counting
+// pass tries the three around the expected rank of the k-th and keeps the
+// highest that qualifies (lower pivots on the rare rows where none does, -inf
+// as the last resort: every visible key is then a candidate).
+__device__ __forceinline__ float select_tau(const float (&g)[kGroups], int k) {
   float s[32];
 #pragma unroll
-  for (int u = 0; u < 16; ++u) {
-    s[u] = g1[4 * u + 1];
-    s[16 + u] = g2[4 * u + 3];
-  }
+  for (int u = 0; u < 32; ++u) s[u] = g[4 * u + 1];
   sort_desc<32>(s);
-  // sample q (0-based) has about (q + 1) * 128 / 33 values at or above it
-  int q = (33 * k) / (2 * kGroups);
-  q = q > 31 ? 31 : q;
+  // sample q (0-based, descending) has about (q + 1) * 128 / 33 maxima at or above it
+  int q = (33 * k + 127) / kGroups - 1;
+  q = q < 1 ? 1 : (q > 30 ? 30 : q);
   float tau = -INFINITY;
   bool pending = true;
-  for (int attempt = 0; attempt < 6; ++attempt) {
-    const float p = pick<32>(s, q);
-    int n0 = 0, n1 = 0;
+  for (int attempt = 0; attempt < 4; ++attempt) {
+    const float p0 = pick<32>(s, q - 1), p1 = pick<32>(s, q), p2 = pick<32>(s, q + 1);
+    int n0 = 0, n1 = 0, n2 = 0;
 #pragma unroll
-    for (int g = 0; g < kGroups; ++g) {
-      n0 += g1[g] >= p ? 1 : 0;
-      n1 += g2[g] >= p ? 1 : 0;
+    for (int i = 0; i < kGroups; ++i) {
+      n0 += g[i] >= p0 ? 1 : 0;
+      n1 += g[i] >= p1 ? 1 : 0;
+      n2 += g[i] >= p2 ? 1 : 0;
     }
-    if (pending && n0 + n1 >= k) {
-      tau = p;
-      pending = false;
+    if (pending) {
+      if (n0 >= k) tau = p0;
+      else if (n1 >= k) tau = p1;
+      else if (n2 >= k) tau = p2;
+      pending = !(n2 >= k);
     }
-    if (q == 31) pending = false;
-    q = q < 31 ? q + 1 : 31;
     if (!__any_sync(0xffffffffu, pending)) break;
+    q = q + 3 > 30 ? 30 : q + 3;
   }
   return tau;
 }
 
-// Pass 2: append the keys of 32 scores of a row (keys j0 .. j0+31) that score
-// above thr and are visible.  A column whose chunk of appends would not fit is
-// first cut to between k and CAP - 32 entries at a sampled pivot (which raises
-// thr to the pivot), together with every column of the warp that is close to
-// the capacity.  The appends are predicated stores at a running slot pointer:
-// no mask, no scratch, no data-dependent loop.
+// Rare path of pass 2: lanes whose column is within one chunk of the capacity
+// and would overflow with this chunk's appends are cut to between k and CAP - 32
+// entries at a sampled pivot (raising thr to it), together with every lane of
+// the warp close to the capacity; the exact cut only where no pivot qualifies.
 template <int CAP, class Col>
-__device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vis, float& thr, float* scr,
-                                         const Col& c, int& cnt, int k) {
-  float v[32];
+__device__ __forceinline__ void make_room(const uint32_t (&r)[32], float& thr, float* scr, const Col& c, int& cnt,
+                                          int k) {
+  int n = 0;
 #pragma unroll
-  for (int u = 0; u < 32; ++u) v[u] = __uint_as_float(r[u]);
-  if (j0 + 32 > vis) {
-#pragma unroll
-    for (int u = 0; u < 32; ++u)
-      if (j0 + u >= vis) v[u] = -INFINITY;
+  for (int u = 0; u < 32; ++u) n += __uint_as_float(r[u]) > thr ? 1 : 0;
+  const bool over = cnt + n > CAP;
+  const int near = (k + 8 > CAP - 40) ? k + 8 : CAP - 40;
+  if (__any_sync(0xffffffffu, over)) {
+    pivot_cut(c, cnt, thr, k, k + 8, CAP - 32, over || cnt > near);
+    const bool still = over && cnt > CAP - 32;
+    if (__any_sync(0xffffffffu, still)) cut_to_k(c, cnt, thr, k, scr, still);
   }
-  if (__any_sync(0xffffffffu, cnt > CAP - 32)) {
-    int n = 0;
-#pragma unroll
-    for (int u = 0; u < 32; ++u) n += v[u] > thr ? 1 : 0;
-    const bool over = cnt + n > CAP;
-    // a cut costs the warp about the same for one row as for all 32: when one
-    // row must be cut, every row close to the capacity is cut in the same call
-    const int near = (k + 8 > CAP - 40) ? k + 8 : CAP - 40;
-    if (__any_sync(0xffffffffu, over)) {
-      // a pivot cut (two passes) leaves between k and CAP - 32 entries; the
-      // exact cut only for lanes where no sampled pivot qualifies
-      pivot_cut(c, cnt, thr, k, k + 8, CAP - 32, over || cnt > near);
-      const bool still = over && cnt > CAP - 32;
-      if (__any_sync(0xffffffffu, still)) cut_to_k(c, cnt, thr, k, scr, still);
-    }
-    __syncwarp();
-  }
+  __syncwarp();
+}
+
+// Pass 2: append the keys of 32 scores of a row (keys j0 .. j0+31; keys the row
+// cannot see are -inf already) that score above thr.  The appends are
+// predicated stores at a running slot pointer: no mask, no scratch, no
+// data-dependent loop; the capacity check is one warp vote.
+template <int CAP, class Col>
+__device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, float& thr, float* scr, const Col& c,
+                                         int& cnt, int k) {
+  if (__any_sync(0xffffffffu, cnt > CAP - 32)) make_room<CAP>(r, thr, scr, c, cnt, k);
   float* ps = c.bs + cnt * kLdc + c.row;
   if constexpr (Col::kWide) {
     // score and index through one slot pointer; the count is the pointer's advance
     float* const p0 = ps;
 #pragma unroll
     for (int u = 0; u < 32; ++u) {
-      const bool t = v[u] > thr;
+      const float v = __uint_as_float(r[u]);
+      const bool t = v > thr;
       if (t) {
-        ps[0] = v[u];
+        ps[0] = v;
         ps[Col::kIOff] = __int_as_float(j0 + u);
       }
       ps += t ? kLdc : 0;
@@ -532,9 +544,10 @@ __device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, int vi
     int added = 0;
 #pragma unroll
     for (int u = 0; u < 32; ++u) {
-      const bool t = v[u] > thr;
+      const float v = __uint_as_float(r[u]);
+      const bool t = v > thr;
       if (t) {
-        *ps = v[u];
+        *ps = v;
         *pi = (uint16_t)(j0 + u);
       }
       ps += t ? kLdc : 0;
@@ -794,39 +807,37 @@ __global__ void __launch_bounds__(192, 1)
         tc::mbar_arrive(aready);
       }
       const int vis = m < t.nrows ? a.vis[t.q0 + m] : 0;
+      const int wmin = __reduce_min_sync(0xffffffffu, vis);   // tiles past it need masking
       const int ntiles = (t.vis_max + C::NT - 1) / C::NT;
-      // pass 1: the two highest scores per key group, then the certified bound
-      float g1[kGroups], g2[kGroups];
+      // pass 1: the maxima of the 128 key groups, then the certified bound
+      float g[kGroups];
 #pragma unroll
-      for (int g = 0; g < kGroups; ++g) {
-        g1[g] = -INFINITY;
-        g2[g] = -INFINITY;
-      }
-      for (int i = 0; i < ntiles; ++i) {
-        const uint32_t buf = ac % C::NB;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
-        if (!ok) break;
-        tc::fence_after_sync();
-        // chunk c + 1 is read from TMEM while chunk c is folded
-        uint32_t ra[32], rb[32];
-        __syncwarp();
-        tc::tmem_ld32(tl + buf * C::BUFC, ra);
-        tc::tmem_ld_wait(ra);
+      for (int u = 0; u < kGroups; ++u) g[u] = -INFINITY;
+      for (int i0 = 0; i0 < ntiles && ok; i0 += 4) {
 #pragma unroll
-        for (int c = 0; c < C::NT / 32; ++c) {
-          uint32_t(&cur)[32] = (c & 1) ? rb : ra;
-          uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
-          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::BUFC + (c + 1) * 32, nxt);
-          fold32(cur, g1, g2, (c % 2) * 32, i * C::NT + c * 32, vis);
-          if (c + 1 < C::NT / 32) tc::tmem_ld_wait(nxt);
+        for (int sub = 0; sub < 4; ++sub) {
+          const int i = i0 + sub;
+          if (i >= ntiles) break;
+          const uint32_t buf = ac % C::NB;
+          ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
+          if (!ok) break;
+          tc::fence_after_sync();
+          uint32_t ra[32], rb[32];
+          __syncwarp();
+          tc::tmem_ld32(tl + buf * C::BUFC, ra);
+          tc::tmem_ld32(tl + buf * C::BUFC + 32, rb);
+          tc::tmem_ld_wait(ra);
+          tc::reg_fence(rb);
+          tc::fence_before_sync();
+          tc::mbar_arrive(acce + buf);   // the scores are in registers: the MMA may reuse the buffer
+          ++ac;
+          if (i * C::NT + C::NT > wmin) mask_tile(ra, rb, i * C::NT, vis);
+          fold64(ra, rb, g, sub * 32);
         }
-        tc::fence_before_sync();
-        tc::mbar_arrive(acce + buf);
-        ++ac;
       }
       if (!ok) break;
       int cnt = 0;
-      float thr = below(select_tau(g1, g2, a.k));
+      float thr = below(select_tau(g, a.k));
       // pass 2: candidates scoring >= tau
       for (int i = 0; i < ntiles; ++i) {
         const uint32_t buf = ac % C::NB;
@@ -836,18 +847,15 @@ __global__ void __launch_bounds__(192, 1)
         uint32_t ra[32], rb[32];
         __syncwarp();
         tc::tmem_ld32(tl + buf * C::BUFC, ra);
+        tc::tmem_ld32(tl + buf * C::BUFC + 32, rb);
         tc::tmem_ld_wait(ra);
-#pragma unroll
-        for (int c = 0; c < C::NT / 32; ++c) {
-          uint32_t(&cur)[32] = (c & 1) ? rb : ra;
-          uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
-          if (c + 1 < C::NT / 32) tc::tmem_ld32(tl + buf * C::BUFC + (c + 1) * 32, nxt);
-          append32<C::CAP>(cur, i * C::NT + c * 32, vis, thr, scr, col, cnt, a.k);
-          if (c + 1 < C::NT / 32) tc::tmem_ld_wait(nxt);
-        }
+        tc::reg_fence(rb);
         tc::fence_before_sync();
         tc::mbar_arrive(acce + buf);
         ++ac;
+        if (i * C::NT + C::NT > wmin) mask_tile(ra, rb, i * C::NT, vis);
+        append32<C::CAP>(ra, i * C::NT, thr, scr, col, cnt, a.k);
+        append32<C::CAP>(rb, i * C::NT + 32, thr, scr, col, cnt, a.k);
       }
       if (!ok) break;
       // convert the next item's projection now, so the tensor core can move on
