@@ -369,11 +369,11 @@ def run_e2e(g, args, torch):
 # the heads, as the pairs do, so bench.py scales these to the workload; a kernel
 # changed after its capture is left out (traffic null).
 TRAFFIC_BYTES_PER_PAIR = {
-    "select": (554087936 + 225715712) / 2148007936,
-    "exact": (868380928 + 238369792) / 2148007936,
-    "moments": (335566848 + 3014400) / 2148007936,
-    "build": (73444608 + 13551872) / 2148007936,
-    "fit": (59018496 + 30720) / 2148007936,
+    "select": (542111744 + 225285632) / 2148007936,
+    "exact": (889242624 + 236534016) / 2148007936,
+    "moments": (335588864 + 3024640) / 2148007936,
+    "build": (73442048 + 13277184) / 2148007936,
+    "fit": (58813440 + 44288) / 2148007936,
 }
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only
 

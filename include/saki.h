@@ -207,6 +207,23 @@ SAKI_API saki_status saki_recall(const saki_config* cfg, const saki_layout* layo
                         int32_t* idx_exact, float* recall, void* workspace,
                         size_t workspace_bytes, saki_stream stream);
 
+/* saki_merge_topk -- the exchange step of a selection split by key ranges
+ * (several GPUs each holding a contiguous range of a long cache, Sec. 1's
+ * 1M-token setting): the k best of the union of per-part top-k lists.
+ *   idx_parts   [P][rows][k] int32  part-local key indices, -1 padding
+ *   score_parts [P][rows][k] f32    their scores (the ranking key)
+ *   part_offsets [P] HOST int64     first key of each part's range, in [0, 2^31)
+ *   idx   [rows][k] int32           global indices (local + offset), -1 padding
+ *   score [rows][k] f32 or NULL
+ * Output lists are in descending score, equal scores by the lower global index,
+ * which is the ranking saki_score_topk applies over the whole range, so merging
+ * the parts' lists reproduces its result.  k = cfg->topk; P <= 64
+ * (SAKI_ERR_UNSUPPORTED above).  Stream-ordered, no workspace. */
+SAKI_API saki_status saki_merge_topk(const saki_config* cfg, int32_t num_parts, int64_t num_rows,
+                                     const int32_t* idx_parts, const float* score_parts,
+                                     const int64_t* part_offsets, int32_t* idx, float* score,
+                                     saki_stream stream);
+
 /* saki_workspace_status -- the device status of the last saki_score_topk,
  * saki_recall or saki_build_index call that used `workspace` (the first 256 bytes
  * of every workspace of these calls are a header holding the error word, which

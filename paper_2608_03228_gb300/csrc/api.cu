@@ -551,6 +551,25 @@ saki_status saki_workspace_status(const void* workspace, saki_stream stream) {
   return read_status(workspace, s);
 }
 
+saki_status saki_merge_topk(const saki_config* cfg, int32_t num_parts, int64_t num_rows, const int32_t* idx_parts,
+                            const float* score_parts, const int64_t* part_offsets, int32_t* idx, float* score,
+                            saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  if (num_parts < 1 || num_rows < 0 || !part_offsets) return SAKI_ERR_INVALID_ARGUMENT;
+  if (num_parts > kMaxParts) return SAKI_ERR_UNSUPPORTED;
+  if (num_rows > 0 && (!idx_parts || !score_parts || !idx)) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {(const void*)idx_parts, (const void*)score_parts, (const void*)idx, (const void*)score})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  PartOffsets po{};
+  for (int p = 0; p < num_parts; ++p) {
+    if (part_offsets[p] < 0 || part_offsets[p] > INT32_MAX) return SAKI_ERR_INVALID_ARGUMENT;
+    po.off[p] = part_offsets[p];
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return cuda_status(launch_merge_parts(idx_parts, score_parts, po, num_parts, num_rows, cfg->topk, idx, score, s));
+}
+
 saki_status saki_debug_inject_stall(int32_t kind) {
   if (kind != 0 && kind != SAKI_KERNEL_SELECT && kind != SAKI_KERNEL_EXACT && kind != SAKI_KERNEL_BUILD)
     return SAKI_ERR_INVALID_ARGUMENT;

@@ -170,4 +170,14 @@ cudaError_t launch_build_tc(const void* K, const float* R, void* sketch, int64_t
                             const BuildItem* items, int n_items, void* wsplit, int* err, int stall,
                             int num_sms, cudaStream_t s);
 
+// ---------------------------------------------------------------- merge of per-part lists
+constexpr int kMaxParts = 64;
+struct PartOffsets {
+  int64_t off[kMaxParts];   // key offset of each part's range (added to its local indices)
+};
+// idx_in, score_in [parts][rows][k] (part-local indices, -1 padding); idx, score
+// [rows][k]: the k best of the union, descending, global indices
+cudaError_t launch_merge_parts(const int32_t* idx_in, const float* score_in, const PartOffsets& po, int parts,
+                               int64_t rows, int k, int32_t* idx, float* score, cudaStream_t s);
+
 }  // namespace saki

@@ -28,7 +28,7 @@ STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED
 EXPORTS = ("saki_workspace_size", "saki_fit", "saki_build_index", "saki_score_topk", "saki_recall",
            "saki_status_string", "saki_version", "saki_score_topk_noalloc", "saki_launch_count",
            "saki_kernel_timer_start", "saki_kernel_timer_stop", "saki_workspace_status", "saki_noalloc_status",
-           "saki_debug_inject_stall")
+           "saki_debug_inject_stall", "saki_merge_topk")
 SAKI_KERNEL_SELECT, SAKI_KERNEL_EXACT, SAKI_KERNEL_FIT, SAKI_KERNEL_MOMENTS, SAKI_KERNEL_BUILD, SAKI_KERNEL_FACTOR = (
     1, 2, 3, 4, 5, 6)
 SAKI_NOALLOC_SCRATCH_BYTES = 16 << 20
@@ -65,6 +65,8 @@ _lib.saki_noalloc_status.restype = ctypes.c_int
 _lib.saki_noalloc_status.argtypes = [_vp]
 _lib.saki_debug_inject_stall.restype = ctypes.c_int
 _lib.saki_debug_inject_stall.argtypes = [_i32]
+_lib.saki_merge_topk.restype = ctypes.c_int
+_lib.saki_merge_topk.argtypes = [ctypes.POINTER(Config), _i32, _i64, _vp, _vp, _vp, _vp, _vp, _vp]
 _lib.saki_status_string.restype = ctypes.c_char_p
 _lib.saki_status_string.argtypes = [ctypes.c_int]
 _lib.saki_version.restype = ctypes.c_char_p
@@ -170,6 +172,16 @@ def saki_noalloc_status(stream=None) -> None:
 def saki_debug_inject_stall(kind: int) -> None:
     """Test hook: the next tensor-core launch of this kernel kind stalls its producer."""
     _check(_lib.saki_debug_inject_stall(kind), "saki_debug_inject_stall")
+
+
+def saki_merge_topk(cfg: Config, idx_parts, score_parts, part_offsets, idx, score=None, stream=None) -> None:
+    """The k best of per-part top-k lists (idx_parts, score_parts [P][rows][k] on
+    the device, part-local indices); part_offsets: host sequence of P ints."""
+    offs = np.ascontiguousarray(part_offsets, np.int64)
+    P = idx_parts.shape[0]
+    rows = idx_parts.numel() // (P * cfg.topk) if P else 0
+    _check(_lib.saki_merge_topk(ctypes.byref(cfg), P, rows, _ptr(idx_parts), _ptr(score_parts), offs.ctypes.data,
+                                _ptr(idx), _ptr(score), _stream(stream)), "saki_merge_topk")
 
 
 def saki_workspace_size(cfg: Config, op: int, layout: HostLayout | None = None, n_calib: int = 0,
