@@ -83,6 +83,11 @@ typedef enum saki_dtype { SAKI_F32 = 0, SAKI_BF16 = 1 } saki_dtype;
                               no-alloc selection) synchronise `stream` before returning
                               and report the device status of their kernels, as
                               saki_workspace_status does */
+#define SAKI_FLAG_SHRINK 4 /* saki_fit: Ledoit-Wolf shrinkage of both moments (Sec. 7):
+                              S <- (1 - rho) S + rho (tr S / d) I, rho = min(b2, d2) / d2,
+                              d2 = ||S - (tr S / d) I||_F^2,
+                              b2 = (1/n^2) sum_t ||x_t x_t^T - S||_F^2 (keys centered
+                              when center = 1) */
 
 /* saki_config.method: which rank-r map saki_fit folds into L and R */
 #define SAKI_METHOD_SAKI 0       /* the exact optimum M_r of Prop. 1 (default) */
@@ -90,6 +95,14 @@ typedef enum saki_dtype { SAKI_F32 = 0, SAKI_BF16 = 1 } saki_dtype;
                                     eigenvectors of Sk; L = A_h V_r, R = V_r */
 #define SAKI_METHOD_WEIGHT_SVD 2 /* Tab. 1 comparison: the truncated SVD of A_h itself,
                                     L = U_r Sigma_r^{1/2}, R = V_r Sigma_r^{1/2} */
+#define SAKI_METHOD_SAP_SVD 3    /* Sec. 6 projector variant: M = A_h Q Q^T with Q the r
+                                    leading right singular vectors of C = Sq^{1/2} A_h Sk^{1/2}
+                                    (symmetric roots), used directly as key directions;
+                                    L = A_h Q, R = Q */
+#define SAKI_METHOD_SAP_MAP 4    /* Sec. 6 projector variant: M = A_h Q Q^T with Q an
+                                    orthonormal basis (Gram-Schmidt, in column order) of the
+                                    optimum's key-side span, span(Sk^{+1/2} V_r);
+                                    L = A_h Q, R = Q */
 
 typedef struct saki_config {
   int32_t num_q_heads;   /* Hq >= 1 */
@@ -123,6 +136,8 @@ typedef struct saki_layout {
 #define SAKI_OP_BUILD_INDEX 1
 #define SAKI_OP_SCORE_TOPK 2
 #define SAKI_OP_RECALL 3
+#define SAKI_OP_KEY_SPECTRUM 4
+#define SAKI_OP_SCORE_MSE 5
 
 /* Bytes of device workspace `op` needs.  FIT uses n_calib; BUILD_INDEX uses
  * total_keys; SCORE_TOPK and RECALL use the layout.  Returns 0 if the arguments
@@ -157,7 +172,13 @@ SAKI_API size_t saki_workspace_size(const saki_config* cfg, int32_t op, const sa
  *                           query calibration data is read but not used;
  *   SAKI_METHOD_WEIGHT_SVD  sigma are A_h's singular values and loss
  *                           sum_{i>r} sigma_i^2; the calibration data is only
- *                           checked and, when center = 1, gives mu. */
+ *                           checked and, when center = 1, gives mu;
+ *   SAKI_METHOD_SAP_SVD,
+ *   SAKI_METHOD_SAP_MAP     the projector variants; sigma and loss are those of
+ *                           the SAKI optimum they are derived from (the
+ *                           variant's own distortion is larger, Prop. 1).
+ *                           Each column of R (= Q) is signed so that its
+ *                           largest-|.| entry is positive. */
 SAKI_API saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_calib,
                      const void* k_calib, const float* A, float* L, float* R, float* mu,
                      float* nu, float* sigma, float* loss, void* workspace,
@@ -206,6 +227,35 @@ SAKI_API saki_status saki_recall(const saki_config* cfg, const saki_layout* layo
                         const void* Q, const float* A, const void* K, const int32_t* idx_approx,
                         int32_t* idx_exact, float* recall, void* workspace,
                         size_t workspace_bytes, saki_stream stream);
+
+/* saki_key_spectrum -- Sec. 7's random-matrix diagnostic: per KV head, the
+ * eigenvalues of the key correlation matrix D^{-1/2} Sk D^{-1/2} (D = diag(Sk);
+ * Sk centered when cfg->center = 1, from the n_calib rows of k_calib
+ * [Hk][n][d]) in descending order, and how many lie above the Marchenko-Pastur
+ * upper edge (1 + sqrt(q_eff))^2, q_eff = d tau_int / n_calib (tau_int >= 1,
+ * the token autocorrelation time; 1 for independent draws).
+ *   eig [Hk][d] f32, spikes [Hk] int32 (device); workspace of
+ *   saki_workspace_size(SAKI_OP_KEY_SPECTRUM).
+ * Synchronises `stream`; SAKI_ERR_NOT_CONVERGED if a Jacobi eigensolve reached
+ * max_sweeps (outputs written from the last sweep). */
+SAKI_API saki_status saki_key_spectrum(const saki_config* cfg, int64_t n_calib, const void* k_calib,
+                                       float tau_int, float* eig, int32_t* spikes, void* workspace,
+                                       size_t workspace_bytes, saki_stream stream);
+
+/* saki_score_mse -- App. C's measured score-MSE reduction: per query head, over
+ * every key_stride-th visible key of every query of the layout (key_stride >= 1;
+ * 1 = all causal pairs), out[h] = { sum s^2, sum (s - s_hat)^2, pairs } in fp64
+ * with s = q^T A_h k and s_hat = (L_h^T q)^T c + q^T nu_h (the index's score,
+ * mean term included when nu is given).  The measured reduction is
+ * 1 - out[h][1] / out[h][0], to compare with the predicted
+ * 1 - sum_{i>r} sigma_i^2 / sum_i sigma_i^2 of saki_fit.
+ *   Q [Hq][T][d], K [Hk][total_keys][d], sketch [Hq][total_keys][r] (dtype),
+ *   A [Hq][d][d], L [Hq][d][r], nu [Hq][d] f32 or NULL, out [Hq][3] double.
+ * Stream-ordered (workspace header as the selection calls). */
+SAKI_API saki_status saki_score_mse(const saki_config* cfg, const saki_layout* layout, int64_t key_stride,
+                                    const void* Q, const float* A, const void* K, const float* L,
+                                    const void* sketch, const float* nu, double* out, void* workspace,
+                                    size_t workspace_bytes, saki_stream stream);
 
 /* saki_merge_topk -- the exchange step of a selection split by key ranges
  * (several GPUs each holding a contiguous range of a long cache, Sec. 1's

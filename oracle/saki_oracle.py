@@ -125,15 +125,36 @@ def score_loss(M, A, Sq, Sk) -> float:
     return float(np.trace(E @ np.asarray(Sk, F64) @ E.T @ np.asarray(Sq, F64)))
 
 
-def fit(q_calib, k_calib, A, rank: int, center: bool, floor_rel: float = 1e-6) -> dict:
+def ledoit_wolf(X, center: bool):
+    """Ledoit-Wolf shrinkage of the second moment of the rows of X [n][d] (Sec. 7
+    applies it to both moments; Ledoit & Wolf 2004): S* = (1 - rho) S + rho m I
+    with m = tr(S) / d, rho = min(b2, d2) / d2, d2 = ||S - m I||_F^2 and
+    b2 = (1/n^2) sum_t ||x_t x_t^T - S||_F^2 (x_t centered when ``center``).
+    Returns (S*, rho, mu)."""
+    S, mu = moments(X, center)
+    Xc = np.asarray(X, F64) - mu
+    n, d = Xc.shape
+    m = np.trace(S) / d
+    d2 = float(np.sum((S - m * np.eye(d)) ** 2))
+    b2 = sum(float(np.sum((np.outer(x, x) - S) ** 2)) for x in Xc) / n ** 2
+    rho = min(b2, d2) / d2 if d2 > 0 else 0.0
+    return (1 - rho) * S + rho * m * np.eye(d), rho, mu
+
+
+def fit(q_calib, k_calib, A, rank: int, center: bool, floor_rel: float = 1e-6, shrink: bool = False) -> dict:
     """All heads: q_calib [Hq][n][d], k_calib [Hk][n][d], A [Hq][d][d].
+    ``shrink`` replaces both moments by their Ledoit-Wolf shrinkage.
 
     Returns L, R [Hq][d][r]; M [Hq][d][d]; mu [Hk][d]; nu = A_h mu_g [Hq][d];
     sigma [Hq][d]; loss [Hq]; Sq [Hq][d][d]; Sk [Hk][d][d]."""
     Hq, Hk = len(q_calib), len(k_calib)
     G = Hq // Hk
-    Sk, mu = zip(*[moments(k_calib[g], center) for g in range(Hk)])
-    Sq = [moments(q_calib[h], False)[0] for h in range(Hq)]
+    if shrink:
+        Sk, _, mu = zip(*[ledoit_wolf(k_calib[g], center) for g in range(Hk)])
+        Sq = [ledoit_wolf(q_calib[h], False)[0] for h in range(Hq)]
+    else:
+        Sk, mu = zip(*[moments(k_calib[g], center) for g in range(Hk)])
+        Sq = [moments(q_calib[h], False)[0] for h in range(Hq)]
     out = {k: [] for k in ("L", "R", "M", "sigma", "loss", "nu")}
     for h in range(Hq):
         g = h // G
@@ -381,3 +402,51 @@ def head_recall(idx_approx, idx_exact, q_visible, min_visible: int, k: int):
 def median_over_heads(recall):
     """Median across heads (Tab. 1 reports medians over all heads)."""
     return float(np.median(np.asarray(recall, F64)))
+
+
+# --------------------------------------------------------------------------
+# Sec. 7: a random-matrix view of the key moments, and App. C's measured
+# score-MSE reduction
+# --------------------------------------------------------------------------
+def correlation_spectrum(S):
+    """Eigenvalues (descending) of the correlation matrix D^{-1/2} S D^{-1/2},
+    D = diag(S) (a zero diagonal entry leaves its row and column zero)."""
+    S = np.asarray(S, F64)
+    dg = np.diag(S)
+    inv = np.where(dg > 0, 1.0 / np.sqrt(np.where(dg > 0, dg, 1.0)), 0.0)
+    Rm = S * inv[:, None] * inv[None, :]
+    return np.sort(np.linalg.eigvalsh(0.5 * (Rm + Rm.T)))[::-1]
+
+
+def mp_upper_edge(d: int, n: int, tau_int: float = 1.0) -> float:
+    """Marchenko-Pastur upper edge (1 + sqrt(q_eff))^2 with q_eff = d / T_eff and
+    T_eff = n / tau_int (Sec. 7)."""
+    return (1.0 + np.sqrt(d * tau_int / n)) ** 2
+
+
+def mp_spike_count(S, n: int, tau_int: float = 1.0) -> int:
+    """Eigenvalues of the correlation matrix of S above the MP upper edge."""
+    lam = correlation_spectrum(S)
+    return int(np.sum(lam > mp_upper_edge(len(lam), n, tau_int)))
+
+
+def score_mse(Q, A, K, L, codes, nu, seq_offsets, q_seq, q_visible, group: int, key_stride: int = 1):
+    """App. C measurement: per query head, over the causal (query, key) pairs
+    (every key_stride-th visible key of each query), the sums of s^2 and
+    (s - s_hat)^2 with s = q^T A k and s_hat = (L^T q)^T c + q^T nu.
+    Returns [Hq][3]: sum s^2, sum (s - s_hat)^2, pairs.  The measured
+    reduction is 1 - column 1 / column 0."""
+    Hq, T = Q.shape[0], Q.shape[1]
+    out = np.zeros((Hq, 3))
+    for h in range(Hq):
+        g = h // group
+        for t in range(T):
+            base, vis = int(seq_offsets[q_seq[t]]), int(q_visible[t])
+            keys = np.arange(0, vis, key_stride)
+            if len(keys) == 0:
+                continue
+            q = np.asarray(Q[h, t], F64)
+            s = exact_scores(q, A[h], K[g, base + keys])
+            sh = approx_scores(q, L[h], codes[h, base + keys]) + (0.0 if nu is None else q @ np.asarray(nu[h], F64))
+            out[h] += (np.sum(s ** 2), np.sum((s - sh) ** 2), len(keys))
+    return out

@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <atomic>
 #include <climits>
+#include <cmath>
 #include <cstring>
 #include <map>
 #include <mutex>
@@ -199,9 +200,8 @@ saki_status check_cfg(const saki_config* c) {
   if (c->center != 0 && c->center != 1) return SAKI_ERR_INVALID_ARGUMENT;
   if (!(c->eig_floor_rel >= 0.f && c->eig_floor_rel < 1.f)) return SAKI_ERR_INVALID_ARGUMENT;
   if (c->max_sweeps < 0) return SAKI_ERR_INVALID_ARGUMENT;
-  if (c->flags & ~(SAKI_FLAG_SORTED | SAKI_FLAG_CHECK)) return SAKI_ERR_INVALID_ARGUMENT;
-  if (c->method != SAKI_METHOD_SAKI && c->method != SAKI_METHOD_KEY_PCA && c->method != SAKI_METHOD_WEIGHT_SVD)
-    return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->flags & ~(SAKI_FLAG_SORTED | SAKI_FLAG_CHECK | SAKI_FLAG_SHRINK)) return SAKI_ERR_INVALID_ARGUMENT;
+  if (c->method < SAKI_METHOD_SAKI || c->method > SAKI_METHOD_SAP_MAP) return SAKI_ERR_INVALID_ARGUMENT;
   return SAKI_OK;
 }
 
@@ -499,7 +499,7 @@ BuildWs build_ws(const saki_config* c, int64_t N) {
 }
 
 // fit workspace: S, F, G [(Hq+Hk)][d][d], mu [Hk][d], status [Hq+Hk], C'^T scratch [Hq][d][d]
-struct FitWs { size_t S, F, G, mu, st, C, I, sig, bytes; };
+struct FitWs { size_t S, F, G, mu, st, C, I, sig, acc4, bytes; };
 // Key PCA also needs an identity operator per query head and its own sigma.
 FitWs fit_ws(const saki_config* c) {
   const size_t nm = (size_t)c->num_q_heads + c->num_kv_heads;
@@ -518,6 +518,12 @@ FitWs fit_ws(const saki_config* c) {
     w.sig = w.I + align_up((size_t)c->num_q_heads * kD * kD * sizeof(float));
     w.bytes = w.sig + align_up((size_t)c->num_q_heads * kD * sizeof(float));
   }
+  if (c->method == SAKI_METHOD_SAP_SVD) {   // the fold reads sigma_r even when the caller asks for none
+    w.sig = w.I;
+    w.bytes = w.sig + align_up((size_t)c->num_q_heads * kD * sizeof(float));
+  }
+  w.acc4 = w.bytes;   // Ledoit-Wolf: sum_t ||x_t||^4 per moment matrix
+  if (c->flags & SAKI_FLAG_SHRINK) w.bytes = w.acc4 + align_up(nm * sizeof(double));
   return w;
 }
 
@@ -549,6 +555,75 @@ saki_status saki_workspace_status(const void* workspace, saki_stream stream) {
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
   return read_status(workspace, s);
+}
+
+saki_status saki_key_spectrum(const saki_config* cfg, int64_t n_calib, const void* k_calib, float tau_int,
+                              float* eig, int32_t* spikes, void* workspace, size_t workspace_bytes,
+                              saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  if (n_calib < 1 || !k_calib || !eig || !spikes || !workspace || !(tau_int >= 1.f)) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {k_calib, (const void*)eig, (const void*)spikes, (const void*)workspace})
+    if (!al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  const int Hk = cfg->num_kv_heads;
+  const size_t off_mu = align_up((size_t)Hk * kD * kD * sizeof(float));
+  const size_t off_st = off_mu + align_up((size_t)Hk * kD * sizeof(float));
+  if (workspace_bytes < off_st + align_up((size_t)Hk * sizeof(int))) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
+  char* ws = static_cast<char*>(workspace);
+  float* S = reinterpret_cast<float*>(ws);
+  int* status = reinterpret_cast<int*>(ws + off_st);
+  if ((st = cuda_status(cudaMemsetAsync(status, 0, Hk * sizeof(int), s))) != SAKI_OK) return st;
+  // key moments only (Hq = 0), centered as cfg->center says
+  if ((st = cuda_status(launch_gram(nullptr, k_calib, n_calib, 0, Hk, cfg->center, cfg->dtype, S,
+                                    reinterpret_cast<float*>(ws + off_mu), status, s))) != SAKI_OK)
+    return st;
+  const double q_eff = (double)kD * tau_int / (double)n_calib;
+  const float edge = (float)((1.0 + std::sqrt(q_eff)) * (1.0 + std::sqrt(q_eff)));
+  const int sweeps = cfg->max_sweeps > 0 ? cfg->max_sweeps : 40;
+  if ((st = cuda_status(launch_spectrum(S, Hk, edge, sweeps, eig, spikes, status, s))) != SAKI_OK) return st;
+  std::vector<int> hst(Hk);
+  if ((st = cuda_status(staging().download_sync(hst.data(), status, Hk * sizeof(int), s))) != SAKI_OK) return st;
+  int acc = 0;
+  for (int v : hst) acc |= v;
+  if (acc & kStTimeout) return SAKI_ERR_TIMEOUT;
+  if (acc & kStNotConverged) return SAKI_ERR_NOT_CONVERGED;
+  return SAKI_OK;
+}
+
+saki_status saki_score_mse(const saki_config* cfg, const saki_layout* layout, int64_t key_stride, const void* Q,
+                           const float* A, const void* K, const float* L, const void* sketch, const float* nu,
+                           double* out, void* workspace, size_t workspace_bytes, saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  int64_t N = 0;
+  if ((st = check_layout(layout, &N)) != SAKI_OK) return st;
+  const int64_t T = layout->num_queries;
+  if (key_stride < 1 || !out || !workspace || (T > 0 && (!Q || !A || !L || (N > 0 && (!K || !sketch)))))
+    return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {Q, (const void*)A, K, (const void*)L, sketch, (const void*)nu, (const void*)out,
+                        (const void*)workspace})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  const size_t need = kHeader + align_up((size_t)T * 2 * sizeof(int64_t));
+  if (workspace_bytes < need) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
+  char* ws = static_cast<char*>(workspace);
+  std::vector<char> host(kHeader + (size_t)T * 2 * sizeof(int64_t), 0);
+  int64_t* qi = reinterpret_cast<int64_t*>(host.data() + kHeader);
+  for (int64_t t = 0; t < T; ++t) {
+    qi[2 * t] = layout->seq_offsets[layout->q_seq[t]];
+    qi[2 * t + 1] = layout->q_visible[t];
+  }
+  if ((st = cuda_status(staging().upload(ws, host.data(), host.size(), s))) != SAKI_OK) return st;
+  const int Hq = cfg->num_q_heads;
+  if ((st = cuda_status(cudaMemsetAsync(out, 0, (size_t)Hq * 3 * sizeof(double), s))) != SAKI_OK) return st;
+  return finish(cfg,
+                cuda_status(launch_score_mse(Q, A, K, L, sketch, nu, reinterpret_cast<const int64_t*>(ws + kHeader), T,
+                                             N, Hq, Hq / cfg->num_kv_heads, cfg->rank, key_stride, cfg->dtype, out,
+                                             s)),
+                ws, s);
 }
 
 saki_status saki_merge_topk(const saki_config* cfg, int32_t num_parts, int64_t num_rows, const int32_t* idx_parts,
@@ -601,6 +676,15 @@ size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout
       return n_calib >= 1 ? fit_ws(cfg).bytes : 0;
     case SAKI_OP_BUILD_INDEX:
       return total_keys >= 0 ? build_ws(cfg, total_keys).bytes : 0;
+    case SAKI_OP_KEY_SPECTRUM:
+      return align_up((size_t)cfg->num_kv_heads * kD * kD * sizeof(float)) +
+             align_up((size_t)cfg->num_kv_heads * kD * sizeof(float)) +
+             align_up((size_t)cfg->num_kv_heads * sizeof(int));
+    case SAKI_OP_SCORE_MSE: {
+      int64_t n = 0;
+      if (check_layout(layout, &n) != SAKI_OK) return 0;
+      return kHeader + align_up((size_t)layout->num_queries * 2 * sizeof(int64_t));
+    }
     case SAKI_OP_SCORE_TOPK:
     case SAKI_OP_RECALL: {
       int64_t n = 0;
@@ -649,20 +733,32 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
                                       s))) != SAKI_OK)
       return st;
   }
+  if (cfg->flags & SAKI_FLAG_SHRINK) {   // Sec. 7: Ledoit-Wolf shrinkage of both moments
+    double* acc4 = reinterpret_cast<double*>(ws + w.acc4);
+    if ((st = cuda_status(cudaMemsetAsync(acc4, 0, nm * sizeof(double), s))) != SAKI_OK) return st;
+    if ((st = cuda_status(launch_fourth_moment(q_calib, k_calib, n_calib, Hq, Hk, cfg->center ? muw : nullptr,
+                                               cfg->dtype, acc4, s))) != SAKI_OK)
+      return st;
+    if ((st = cuda_status(launch_shrink(S, acc4, n_calib, nm, nullptr, s))) != SAKI_OK) return st;
+  }
   // The comparison indexes reuse the fit with other inputs: weight SVD whitens
   // with identity factors (C' = A); key PCA keeps the key factors and sets the
   // query factors and the operator to the identity (C' = F_k, whose left singular
   // vectors are Sk's eigenvectors), then folds A into L.
   const int method = cfg->method;
   float* Iw = reinterpret_cast<float*>(ws + w.I);
-  float* sig = method == SAKI_METHOD_KEY_PCA && !sigma ? reinterpret_cast<float*>(ws + w.sig) : sigma;
+  float* sig = (method == SAKI_METHOD_KEY_PCA || method == SAKI_METHOD_SAP_SVD) && !sigma
+                   ? reinterpret_cast<float*>(ws + w.sig) : sigma;
   {
     KernelTimer kt(SAKI_KERNEL_FACTOR, s);
     if (method == SAKI_METHOD_WEIGHT_SVD) {
       if ((st = cuda_status(launch_identity(F, nm, s))) != SAKI_OK) return st;
       if ((st = cuda_status(launch_identity(Gm, nm, s))) != SAKI_OK) return st;
     } else {
-      if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s))) != SAKI_OK)
+      // SAP-svd needs the symmetric key roots (the right singular vectors of C itself)
+      const int sym_from = method == SAKI_METHOD_SAP_SVD ? Hq : (1 << 30);
+      if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s, sym_from))) !=
+          SAKI_OK)
         return st;
     }
     if (method == SAKI_METHOD_KEY_PCA) {
@@ -681,6 +777,10 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
     if (method == SAKI_METHOD_KEY_PCA &&
         (st = cuda_status(launch_key_pca_fold(A, sig, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, L, R, nu,
                                               s))) != SAKI_OK)
+      return st;
+    if ((method == SAKI_METHOD_SAP_SVD || method == SAKI_METHOD_SAP_MAP) &&
+        (st = cuda_status(launch_sap_fold(A, F, sig, Hq, Hk, cfg->rank, method == SAKI_METHOD_SAP_SVD, L, R, s))) !=
+            SAKI_OK)
       return st;
   }
   std::vector<int> hst(nm);

@@ -313,8 +313,13 @@ __device__ void column_norms(const float* X, float* out, int ld = kLdS) {
 // One d x d buffer in shared memory (two CTAs per SM): the Cholesky factor L
 // in its lower triangle, L^{-1} transposed in its strict upper triangle with
 // L^{-1}'s diagonal in dinv; or, on the fallback path, the Jacobi matrix.
+// Matrices m >= sym_from take the eigen path whatever their spectrum and store
+// the symmetric roots F = S^{1/2} = V Lambda^{1/2} V^T and G = S^{+1/2} (the
+// projector variant SAP-svd needs the right singular vectors of the
+// symmetric-root C itself).
 __global__ void __launch_bounds__(kFitThreads, 2) factor_kernel(const float* S, float floor_rel, int max_sweeps,
-                                                                float tol, float* Fout, float* Gout, int* status) {
+                                                                float tol, float* Fout, float* Gout, int* status,
+                                                                int sym_from) {
   extern __shared__ __align__(16) float sm[];
   float* Sb = sm;   // row-major
   float* Xb = sm;   // the Jacobi matrix of the fallback path
@@ -346,8 +351,11 @@ __global__ void __launch_bounds__(kFitThreads, 2) factor_kernel(const float* S, 
   }
   const float trace = red[0];
 
+  const bool sym = m >= sym_from;
+  if (sym && tid == 0) flag = 3;   // skip the Cholesky path
+  __syncthreads();
   // Cholesky, right-looking, in place
-  for (int j = 0; j < kD; ++j) {
+  for (int j = 0; j < kD && !sym; ++j) {
     const float piv = Sb[j * kLdS + j];
     const bool ok = piv > 0.f && isfinite(piv);
     if (!ok) { if (tid == 0) flag = 1; }
@@ -365,7 +373,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) factor_kernel(const float* S, 
     __syncthreads();
   }
 
-  bool chol_ok = (flag == 0);
+  bool chol_ok = (flag == 0) && !sym;
   if (chol_ok) {
     // Linv = F^{-1} by right-looking substitution on the identity: row i is
     // divided by F_ii, then subtracted (times F_ri) from every row below it.
@@ -432,6 +440,25 @@ __global__ void __launch_bounds__(kFitThreads, 2) factor_kernel(const float* S, 
   }
   __syncthreads();
   const float lmax = red[0];
+  if (sym) {
+    // F = sum_c v_c v_c^T sqrt(l_c), G = sum_c v_c v_c^T / sqrt(l_c) over the kept
+    // eigenpairs (v_c = w_c / l_c from the Jacobi columns w_c = v_c l_c)
+    for (int o = tid; o < kD * kD; o += kFitThreads) {
+      const int i = o / kD, j = o % kD;
+      float f = 0.f, gg = 0.f;
+      for (int c = 0; c < kD; ++c) {
+        const float l = lam[c];
+        if (!(l > 0.f && l >= floor_rel * lmax)) continue;
+        const float vv = (Xb[c * kLdS + i] / l) * (Xb[c * kLdS + j] / l);
+        const float sl = sqrtf(l);
+        f = fmaf(vv, sl, f);
+        gg = fmaf(vv, 1.f / sl, gg);
+      }
+      F[o] = f;
+      G[o] = gg;
+    }
+    return;
+  }
   for (int o = tid; o < kD * kD; o += kFitThreads) {
     const int i = o / kD, c = o % kD;
     const float l = lam[c];
@@ -634,17 +661,147 @@ __global__ void __launch_bounds__(kD) key_pca_fold_kernel(const float* A, const 
   }
 }
 
+// The projector variants of Sec. 6 (SAP-svd, SAP-map) from a SAKI fit: an
+// orthonormal basis Q of an r-dimensional key subspace, the map M = A_h Q Q^T
+// folded as R = Q, L = A_h Q (nu = A_h mu is the fit's).  SAP-map takes the
+// optimum's key-side span, span(Sk^{+1/2} V_r): the columns of the fit's R
+// (Sk^{+1/2} V_r Sigma_r^{1/2} whatever factor of Sk whitened it), in order.
+// SAP-svd takes the raw right singular vectors V_r of C: with the symmetric key
+// root F_k = Sk^{1/2} (factor kernel, sym_from) the fit's R gives
+// V_r = F_k R Sigma_r^{-1/2}.  Either basis is orthonormalised by modified
+// Gram-Schmidt in column order and each column signed so that its largest-|.|
+// entry (the first of equal ones) is positive.  One CTA of d threads per head;
+// thread i owns row i.
+__global__ void __launch_bounds__(kD) sap_fold_kernel(const float* A, const float* Fm, const float* sigma, int Hq,
+                                                      int Hk, int r, int svd, float* L, float* R) {
+  extern __shared__ float sm[];
+  float* As = sm;                    // A_h or F_k, row stride d + 1
+  float* Qs = As + kD * (kD + 1);    // [d][r]
+  __shared__ float red[kD / 32];
+  __shared__ int redi[kD / 32];
+  const int h = blockIdx.x, g = h / (Hq / Hk), i = threadIdx.x, lane = i & 31, warp = i >> 5;
+  float* Lh = L + (int64_t)h * kD * r;
+  float* Rh = R + (int64_t)h * kD * r;
+  if (svd) {
+    const float* Fk = Fm + (int64_t)(Hq + g) * kD * kD;
+    for (int o = i; o < kD * kD; o += kD) As[(o / kD) * (kD + 1) + o % kD] = Fk[o];
+    __syncthreads();
+    for (int c = 0; c < r; ++c) {
+      float acc = 0.f;
+      for (int j = 0; j < kD; ++j) acc = fmaf(As[i * (kD + 1) + j], Rh[j * r + c], acc);
+      const float sg = sigma[(int64_t)h * kD + c];
+      Qs[i * r + c] = sg > 0.f ? acc * rsqrtf(sg) : 0.f;
+    }
+  } else {
+    for (int c = 0; c < r; ++c) Qs[i * r + c] = Rh[i * r + c];
+  }
+  __syncthreads();
+  auto block_sum = [&](float v) {
+    v = warp_sum(v);
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kD / 32; ++w) t += red[w];
+    __syncthreads();
+    return t;
+  };
+  for (int c = 0; c < r; ++c) {
+    float x = Qs[i * r + c];
+    for (int p = 0; p < c; ++p) {
+      const float qp = Qs[i * r + p];
+      const float dot = block_sum(qp * x);
+      x = fmaf(-dot, qp, x);
+    }
+    const float nrm = sqrtf(block_sum(x * x));
+    x = nrm > 0.f ? x / nrm : 0.f;
+    // sign: the largest-|.| entry (first of equal ones) positive
+    float best = fabsf(x);
+    int bi = i;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ob > best || (ob == best && oi < bi)) { best = ob; bi = oi; }
+    }
+    if (lane == 0) { red[warp] = best; redi[warp] = bi; }
+    __syncthreads();
+    float b = red[0];
+    int bidx = redi[0];
+    for (int w = 1; w < kD / 32; ++w)
+      if (red[w] > b || (red[w] == b && redi[w] < bidx)) { b = red[w]; bidx = redi[w]; }
+    __syncthreads();
+    if (i == bidx) red[0] = x;
+    __syncthreads();
+    if (red[0] < 0.f) x = -x;
+    __syncthreads();
+    Qs[i * r + c] = x;
+    __syncthreads();
+  }
+  // L = A_h Q, R = Q
+  const float* Ah = A + (int64_t)h * kD * kD;
+  for (int o = i; o < kD * kD; o += kD) As[(o / kD) * (kD + 1) + o % kD] = Ah[o];
+  __syncthreads();
+  for (int c = 0; c < r; ++c) {
+    float acc = 0.f;
+    for (int j = 0; j < kD; ++j) acc = fmaf(As[i * (kD + 1) + j], Qs[j * r + c], acc);
+    Lh[i * r + c] = acc;
+    Rh[i * r + c] = Qs[i * r + c];
+  }
+}
+
+// Sec. 7 diagnostic: the eigenvalues (descending) of each key correlation
+// matrix D^{-1/2} S D^{-1/2} (D = diag(S); a zero diagonal entry leaves its row
+// and column zero), from one-sided Jacobi on it, and the number above the
+// Marchenko-Pastur upper edge.  The column norms of the converged Jacobi matrix
+// are the eigenvalues of the PSD input; a rank sort (ties by position) orders them.
+__global__ void __launch_bounds__(kFitThreads, 2) spectrum_kernel(const float* S, float edge, int max_sweeps,
+                                                                  float tol, float* lam_out, int* spikes,
+                                                                  int* status) {
+  extern __shared__ __align__(16) float sm[];
+  float* Xb = sm;   // column-major, ld kLdS
+  __shared__ float lam[kD];
+  __shared__ float dg[kD];
+  __shared__ int counter, above;
+  const int m = blockIdx.x, tid = threadIdx.x;
+  const float* Sm = S + (int64_t)m * kD * kD;
+  if (tid < kD) {
+    const float v = Sm[tid * kD + tid];
+    dg[tid] = v > 0.f ? rsqrtf(v) : 0.f;
+  }
+  if (tid == 0) above = 0;
+  __syncthreads();
+  for (int o = tid; o < kD * kD; o += kFitThreads) {
+    const int i = o / kD, c = o % kD;
+    Xb[c * kLdS + i] = Sm[o] * dg[i] * dg[c];
+  }
+  __syncthreads();
+  const bool conv = jacobi_columns(Xb, max_sweeps, tol, &counter);
+  if (!conv && tid == 0) status[m] |= kStNotConverged;
+  column_norms(Xb, lam);
+  __syncthreads();
+  if (tid < kD) {
+    const float l = lam[tid];
+    int rank = 0;
+    for (int j = 0; j < kD; ++j) rank += (lam[j] > l || (lam[j] == l && j < tid)) ? 1 : 0;
+    lam_out[(int64_t)m * kD + rank] = l;
+    if (l > edge) atomicAdd(&above, 1);
+  }
+  __syncthreads();
+  if (tid == 0) spikes[m] = above;
+}
+
 constexpr float kTol = 1e-6f;
 constexpr size_t kSmem = sizeof(float) * kD * kLdS;         // factor kernel: L and L^{-1} share one buffer
 constexpr size_t kFitSmem = sizeof(float) * kD * kLdJ;      // fit kernel: the Jacobi matrix
 }  // namespace
 
 cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps, float* F, float* Gm,
-                          int* status, cudaStream_t s) {
+                          int* status, cudaStream_t s, int sym_from) {
   cudaError_t e = cudaFuncSetAttribute(factor_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
   if (e != cudaSuccess) return e;
   note_launch();
-  factor_kernel<<<nmat, kFitThreads, kSmem, s>>>(S, floor_rel, max_sweeps, kTol, F, Gm, status);
+  factor_kernel<<<nmat, kFitThreads, kSmem, s>>>(S, floor_rel, max_sweeps, kTol, F, Gm, status, sym_from);
   return cudaGetLastError();
 }
 
@@ -676,4 +833,28 @@ cudaError_t launch_key_pca_fold(const float* A, const float* sigma, const float*
   return cudaGetLastError();
 }
 
+}  // namespace saki
+
+namespace saki {
+cudaError_t launch_sap_fold(const float* A, const float* F, const float* sigma, int Hq, int Hk, int r, int svd,
+                            float* L, float* R, cudaStream_t s) {
+  const int smem = (int)(sizeof(float) * (kD * (kD + 1) + kD * r));
+  cudaError_t e = cudaFuncSetAttribute(sap_fold_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  note_launch();
+  sap_fold_kernel<<<Hq, kD, smem, s>>>(A, F, sigma, Hq, Hk, r, svd, L, R);
+  return cudaGetLastError();
+}
+}  // namespace saki
+
+namespace saki {
+cudaError_t launch_spectrum(const float* S, int nmat, float edge, int max_sweeps, float* lam, int* spikes, int* status,
+                            cudaStream_t s) {
+  if (nmat == 0) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(spectrum_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+  if (e != cudaSuccess) return e;
+  note_launch();
+  spectrum_kernel<<<nmat, kFitThreads, kSmem, s>>>(S, edge, max_sweeps, kTol, lam, spikes, status);
+  return cudaGetLastError();
+}
 }  // namespace saki

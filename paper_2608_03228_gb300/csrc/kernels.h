@@ -98,8 +98,12 @@ cudaError_t launch_gram(const void* q_calib, const void* k_calib, int64_t n, int
 
 // factor F (F F^T = S, floor applied, row-major) and G = pseudo-inverse transpose of F
 // (stored transposed, i.e. column-major), per matrix
+// matrices m >= sym_from store the symmetric roots (eigen path) instead
 cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps,
-                          float* F, float* Gm, int* status, cudaStream_t s);
+                          float* F, float* Gm, int* status, cudaStream_t s, int sym_from = 1 << 30);
+// projector variants (SAP-svd: svd = 1, SAP-map: svd = 0) folded from a SAKI fit
+cudaError_t launch_sap_fold(const float* A, const float* F, const float* sigma, int Hq, int Hk, int r, int svd,
+                            float* L, float* R, cudaStream_t s);
 
 // per query head: C' = Fq^T A Fk, Jacobi SVD, factors L, R, sigma, loss, nu
 // Cws: scratch [Hq][d][d] (C'^T per head)
@@ -179,5 +183,19 @@ struct PartOffsets {
 // [rows][k]: the k best of the union, descending, global indices
 cudaError_t launch_merge_parts(const int32_t* idx_in, const float* score_in, const PartOffsets& po, int parts,
                                int64_t rows, int k, int32_t* idx, float* score, cudaStream_t s);
+
+// ---------------------------------------------------------------- Sec. 7 / App. C diagnostics
+// sum_t ||x_t - mu||^4 per calibration matrix (keys centered on mu when given) into acc (zeroed)
+cudaError_t launch_fourth_moment(const void* q, const void* k, int64_t n, int Hq, int Hk, const float* mu, int dtype,
+                                 double* acc, cudaStream_t s);
+// Ledoit-Wolf shrinkage of nmat moment matrices in place (rho per matrix if given)
+cudaError_t launch_shrink(float* S, const double* acc4, int64_t n, int nmat, float* rho, cudaStream_t s);
+// eigenvalues (descending) of each correlation matrix of S, and the count above edge
+cudaError_t launch_spectrum(const float* S, int nmat, float edge, int max_sweeps, float* lam, int* spikes, int* status,
+                            cudaStream_t s);
+// per head: sum s^2, sum (s - s_hat)^2, pairs over every stride-th visible key (out [Hq][3], zeroed)
+cudaError_t launch_score_mse(const void* Q, const float* A, const void* K, const float* L, const void* codes,
+                             const float* nu, const int64_t* qinfo, int64_t T, int64_t N, int Hq, int G, int r,
+                             int64_t stride, int dtype, double* out, cudaStream_t s);
 
 }  // namespace saki

@@ -19,16 +19,18 @@ if not os.path.exists(_LIB_PATH):
 _lib = ctypes.CDLL(_LIB_PATH)
 
 SAKI_F32, SAKI_BF16 = 0, 1
-SAKI_FLAG_SORTED, SAKI_FLAG_CHECK = 1, 2
-SAKI_METHOD_SAKI, SAKI_METHOD_KEY_PCA, SAKI_METHOD_WEIGHT_SVD = 0, 1, 2
-METHODS = {"saki": SAKI_METHOD_SAKI, "key_pca": SAKI_METHOD_KEY_PCA, "weight_svd": SAKI_METHOD_WEIGHT_SVD}
+SAKI_FLAG_SORTED, SAKI_FLAG_CHECK, SAKI_FLAG_SHRINK = 1, 2, 4
+SAKI_METHOD_SAKI, SAKI_METHOD_KEY_PCA, SAKI_METHOD_WEIGHT_SVD, SAKI_METHOD_SAP_SVD, SAKI_METHOD_SAP_MAP = 0, 1, 2, 3, 4
+METHODS = {"saki": SAKI_METHOD_SAKI, "key_pca": SAKI_METHOD_KEY_PCA, "weight_svd": SAKI_METHOD_WEIGHT_SVD,
+           "sap_svd": SAKI_METHOD_SAP_SVD, "sap_map": SAKI_METHOD_SAP_MAP}
 SAKI_OP_FIT, SAKI_OP_BUILD_INDEX, SAKI_OP_SCORE_TOPK, SAKI_OP_RECALL = 0, 1, 2, 3
+SAKI_OP_KEY_SPECTRUM, SAKI_OP_SCORE_MSE = 4, 5
 STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED", 3: "SAKI_ERR_CUDA",
           4: "SAKI_ERR_NUMERIC", 5: "SAKI_ERR_NOT_CONVERGED", 6: "SAKI_ERR_WORKSPACE", 7: "SAKI_ERR_TIMEOUT"}
 EXPORTS = ("saki_workspace_size", "saki_fit", "saki_build_index", "saki_score_topk", "saki_recall",
            "saki_status_string", "saki_version", "saki_score_topk_noalloc", "saki_launch_count",
            "saki_kernel_timer_start", "saki_kernel_timer_stop", "saki_workspace_status", "saki_noalloc_status",
-           "saki_debug_inject_stall", "saki_merge_topk")
+           "saki_debug_inject_stall", "saki_merge_topk", "saki_key_spectrum", "saki_score_mse")
 SAKI_KERNEL_SELECT, SAKI_KERNEL_EXACT, SAKI_KERNEL_FIT, SAKI_KERNEL_MOMENTS, SAKI_KERNEL_BUILD, SAKI_KERNEL_FACTOR = (
     1, 2, 3, 4, 5, 6)
 SAKI_NOALLOC_SCRATCH_BYTES = 16 << 20
@@ -67,6 +69,10 @@ _lib.saki_debug_inject_stall.restype = ctypes.c_int
 _lib.saki_debug_inject_stall.argtypes = [_i32]
 _lib.saki_merge_topk.restype = ctypes.c_int
 _lib.saki_merge_topk.argtypes = [ctypes.POINTER(Config), _i32, _i64, _vp, _vp, _vp, _vp, _vp, _vp]
+_lib.saki_key_spectrum.restype = ctypes.c_int
+_lib.saki_key_spectrum.argtypes = [ctypes.POINTER(Config), _i64, _vp, ctypes.c_float, _vp, _vp, _vp, _sz, _vp]
+_lib.saki_score_mse.restype = ctypes.c_int
+_lib.saki_score_mse.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout), _i64] + [_vp] * 8 + [_sz, _vp]
 _lib.saki_status_string.restype = ctypes.c_char_p
 _lib.saki_status_string.argtypes = [ctypes.c_int]
 _lib.saki_version.restype = ctypes.c_char_p
@@ -172,6 +178,26 @@ def saki_noalloc_status(stream=None) -> None:
 def saki_debug_inject_stall(kind: int) -> None:
     """Test hook: the next tensor-core launch of this kernel kind stalls its producer."""
     _check(_lib.saki_debug_inject_stall(kind), "saki_debug_inject_stall")
+
+
+def saki_key_spectrum(cfg: Config, k_calib, eig, spikes, tau_int=1.0, workspace=None, stream=None) -> None:
+    """Sec. 7: eigenvalues of each KV head's key correlation matrix (descending,
+    eig [Hk][d]) and the count above the Marchenko-Pastur edge (spikes [Hk] int32)."""
+    n = k_calib.shape[1]
+    need = saki_workspace_size(cfg, SAKI_OP_KEY_SPECTRUM)
+    ws = workspace if workspace is not None else _workspace(need, k_calib.device)
+    _check(_lib.saki_key_spectrum(ctypes.byref(cfg), n, _ptr(k_calib), float(tau_int), _ptr(eig), _ptr(spikes),
+                                  _ptr(ws), ws.numel(), _stream(stream)), "saki_key_spectrum")
+
+
+def saki_score_mse(cfg: Config, layout: HostLayout, Q, A, K, L, sketch, out, nu=None, key_stride=1, workspace=None,
+                   stream=None) -> None:
+    """App. C: per head sum s^2, sum (s - s_hat)^2, pairs (out [Hq][3] float64)."""
+    need = saki_workspace_size(cfg, SAKI_OP_SCORE_MSE, layout)
+    ws = workspace if workspace is not None else _workspace(need, Q.device)
+    _check(_lib.saki_score_mse(ctypes.byref(cfg), ctypes.byref(layout.c), int(key_stride), _ptr(Q), _ptr(A), _ptr(K),
+                               _ptr(L), _ptr(sketch), _ptr(nu), _ptr(out), _ptr(ws), ws.numel(), _stream(stream)),
+           "saki_score_mse")
 
 
 def saki_merge_topk(cfg: Config, idx_parts, score_parts, part_offsets, idx, score=None, stream=None) -> None:

@@ -81,7 +81,7 @@ def _cfg(lib, **kw):
 @pytest.mark.parametrize("kw,code", [
     (dict(num_kv_heads=3), 1), (dict(rank=0), 1), (dict(rank=129), 1), (dict(topk=0), 1), (dict(topk=129), 2),
     (dict(head_dim=64), 2), (dict(dtype=7), 1), (dict(center=2), 1), (dict(eig_floor_rel=-1.0), 1),
-    (dict(max_sweeps=-1), 1), (dict(flags=4), 1), (dict(method=3), 1), (dict(method=-1), 1),
+    (dict(max_sweeps=-1), 1), (dict(flags=64), 1), (dict(flags=8), 1), (dict(method=5), 1), (dict(method=-1), 1),
 ])
 def test_config_validation(lib, kw, code):
     cfg = _cfg(lib, **kw)

@@ -99,6 +99,31 @@ def test_fit_comparison_indexes(lib, tiny, method, center):
         np.testing.assert_allclose(g["nu"][h], ref["nu"][h], atol=1e-4 * max(1.0, np.abs(ref["nu"][h]).max()))
 
 
+@pytest.mark.parametrize("method", ["sap_svd", "sap_map"])
+@pytest.mark.parametrize("center", [0, 1])
+def test_fit_projector_variants(lib, tiny, method, center):
+    """Sec. 6's projector variants through saki_fit: M = A Q Q^T with Q the raw
+    right singular vectors of C (SAP-svd) or an orthonormal basis of the
+    optimum's key-side span (SAP-map), against the oracle's sap_*_head."""
+    w, data, _ = tiny
+    g = _gpu_fit(lib, w, data, center=center, method=method)
+    ref = O.fit(data["q_calib"], data["k_calib"], data["A"], w.rank, center=bool(center))
+    fn = O.sap_svd_head if method == "sap_svd" else O.sap_map_head
+    for h in range(w.num_q_heads):
+        gk = h // w.group
+        res = fn(ref["Sq"][h], ref["Sk"][gk], data["A"][h], w.rank)
+        if _rel_gap(ref["sigma"][h], w.rank) >= 1e-3:
+            assert map_rel_err(g["L"][h], g["R"][h], res["M"]) <= MAP_REL, (method, h)
+        R = g["R"][h].astype(np.float64)
+        np.testing.assert_allclose(R.T @ R, np.eye(w.rank), atol=1e-5)
+        np.testing.assert_allclose(g["L"][h], data["A"][h].astype(np.float64) @ R, atol=1e-5 * np.abs(g["L"][h]).max())
+        # the signs follow the oracle's rule (largest-|.| entry of each column positive)
+        top = np.argmax(np.abs(R), axis=0)
+        assert np.all(R[top, np.arange(w.rank)] > 0)
+        np.testing.assert_allclose(g["sigma"][h], ref["sigma"][h], atol=1e-4 * ref["sigma"][h][0], rtol=0)
+        np.testing.assert_allclose(g["nu"][h], ref["nu"][h], atol=1e-4 * max(1.0, np.abs(ref["nu"][h]).max()))
+
+
 def test_comparison_index_recall_end_to_end(lib, tiny):
     """fit -> index -> select -> recall with each comparison index, against the
     oracle's chain for the same index (the Tab. 1 measurement on synthetic data)."""

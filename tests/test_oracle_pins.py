@@ -530,3 +530,76 @@ def test_fit_maps_query_heads_to_their_own_kv_head():
             np.testing.assert_allclose(base["loss"], [2.1] * 4, rtol=1e-12)
         else:                        # data-blind: every head keeps two unit directions of I
             np.testing.assert_allclose(base["loss"], [d - r] * 4, rtol=1e-12)
+
+
+# ------------------------------------------------------- Sec. 7 diagnostics
+@pytest.mark.parametrize("center", [False, True])
+def test_ledoit_wolf_matches_sklearn(center):
+    cov = pytest.importorskip("sklearn.covariance")
+    rng = np.random.default_rng(21)
+    X = rng.standard_normal((60, 12)) @ rng.standard_normal((12, 12)) + (1.5 if center else 0.0)
+    S, rho, _ = O.ledoit_wolf(X, center)
+    ref, ref_rho = cov.ledoit_wolf(X, assume_centered=not center)
+    np.testing.assert_allclose(S, ref, rtol=1e-10, atol=1e-12)
+    assert abs(rho - ref_rho) <= 1e-12
+
+
+def test_ledoit_wolf_limits():
+    rng = np.random.default_rng(22)
+    # many samples of a strongly anisotropic distribution: almost no shrinkage
+    X = rng.standard_normal((20000, 8)) * np.array([10, 5, 3, 2, 1, 1, 0.5, 0.2])
+    _, rho, _ = O.ledoit_wolf(X, False)
+    assert 0 <= rho < 1e-3
+    # fewer samples than dimensions of an isotropic distribution: heavy shrinkage
+    X = rng.standard_normal((8, 64))
+    S, rho, _ = O.ledoit_wolf(X, False)
+    assert rho > 0.5
+    np.testing.assert_allclose(np.trace(S), np.trace(X.T @ X / 8), rtol=1e-12)   # the trace is kept
+
+
+def test_correlation_spectrum_and_mp_edge():
+    rng = np.random.default_rng(23)
+    d, n = 64, 4096
+    # white data: the largest sample eigenvalue sits at the MP edge, no spike
+    X = rng.standard_normal((n, d)) * rng.uniform(0.5, 3.0, d)     # scales drop out of the correlation
+    S = X.T @ X / n
+    lam = O.correlation_spectrum(S)
+    assert abs(lam.sum() - d) < 1e-9                                # unit diagonal
+    edge = O.mp_upper_edge(d, n)
+    assert edge == pytest.approx((1 + np.sqrt(d / n)) ** 2)
+    assert abs(lam[0] - edge) < 0.08 and O.mp_spike_count(S, n) == 0
+    # five planted spikes far above the edge are all counted
+    U = np.linalg.qr(rng.standard_normal((d, 5)))[0]
+    Xs = rng.standard_normal((n, d)) + (rng.standard_normal((n, 5)) * np.sqrt([40, 30, 20, 15, 10])) @ U.T
+    assert O.mp_spike_count(Xs.T @ Xs / n, n) == 5
+    # autocorrelation shrinks the effective sample: the edge moves out
+    assert O.mp_upper_edge(d, n, tau_int=3.2) > edge
+
+
+def test_score_mse_reduction_by_double_loop_and_full_rank():
+    rng = np.random.default_rng(24)
+    d, Hq, N = 6, 2, 9
+    Q = rng.standard_normal((Hq, N, d))
+    K = rng.standard_normal((1, N, d)) + 0.5
+    A = rng.standard_normal((Hq, d, d))
+    L = rng.standard_normal((Hq, d, 3))
+    codes = rng.standard_normal((Hq, N, 3))
+    nu = rng.standard_normal((Hq, d))
+    off, q_seq, q_vis = np.array([0, N]), np.zeros(N, np.int32), np.arange(1, N + 1)
+    out = O.score_mse(Q, A, K, L, codes, nu, off, q_seq, q_vis, group=2, key_stride=2)
+    for h in range(Hq):
+        ss = se = cnt = 0.0
+        for t in range(N):
+            for j in range(0, t + 1, 2):
+                s = sum(Q[h, t, a] * A[h, a, b] * K[0, j, b] for a in range(d) for b in range(d))
+                sh = sum(sum(L[h, a, c] * Q[h, t, a] for a in range(d)) * codes[h, j, c] for c in range(3))
+                sh += sum(Q[h, t, a] * nu[h, a] for a in range(d))
+                ss, se, cnt = ss + s * s, se + (s - sh) ** 2, cnt + 1
+        np.testing.assert_allclose(out[h], [ss, se, cnt], rtol=1e-12)
+    # r = d with centered codes and the mean term: the index reproduces q^T A k
+    kc = rng.standard_normal((300, d)) + 1.0
+    qc = rng.standard_normal((300, d))
+    res = O.fit(qc[None], kc[None], A[:1], d, center=True)
+    codes = O.build_index(K, res["R"], res["mu"], "f32", 1)
+    out = O.score_mse(Q[:1], A[:1], K, res["L"], codes, res["nu"], off, q_seq, q_vis, group=1)
+    assert out[0, 1] <= 1e-12 * out[0, 0]
