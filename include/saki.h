@@ -138,6 +138,8 @@ typedef struct saki_layout {
 #define SAKI_OP_RECALL 3
 #define SAKI_OP_KEY_SPECTRUM 4
 #define SAKI_OP_SCORE_MSE 5
+#define SAKI_OP_MOMENTS 6
+#define SAKI_OP_RECONSTRUCT 7   /* total_keys: the number of rows to reconstruct */
 
 /* Bytes of device workspace `op` needs.  FIT uses n_calib; BUILD_INDEX uses
  * total_keys; SCORE_TOPK and RECALL use the layout.  Returns 0 if the arguments
@@ -183,6 +185,52 @@ SAKI_API saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const voi
                      const void* k_calib, const float* A, float* L, float* R, float* mu,
                      float* nu, float* sigma, float* loss, void* workspace,
                      size_t workspace_bytes, saki_stream stream);
+
+/* saki_moments -- online tracking of the calibration moments (Sec. 2: online
+ * updates of Sq and Sk compose with the method).  Adds a batch of n_new
+ * calibration rows to running moments that so far cover n_prev rows:
+ *   q_new [Hq][n_new][d], k_new [Hk][n_new][d] (dtype)
+ *   Sq [Hq][d][d], Sk [Hk][d][d] f32, in/out; mu [Hk][d] f32 in/out (keys'
+ *   running mean, required when center = 1; zeroed when center = 0)
+ * Moments are normalised by 1/n; with center = 1 the key moments are merged by
+ * the pooled-variance identity, so after any sequence of calls they equal
+ * saki_fit's moments of all the rows at once (up to rounding).  n_prev = 0
+ * starts afresh (the inputs' previous contents are ignored).  Stream-ordered;
+ * workspace of saki_workspace_size(SAKI_OP_MOMENTS) with the error-word header
+ * (saki_workspace_status). */
+SAKI_API saki_status saki_moments(const saki_config* cfg, int64_t n_new, const void* q_new,
+                                  const void* k_new, int64_t n_prev, float* Sq, float* Sk, float* mu,
+                                  void* workspace, size_t workspace_bytes, saki_stream stream);
+
+/* saki_fit_moments -- saki_fit from given moments (Sq [Hq][d][d], Sk [Hk][d][d],
+ * mu [Hk][d] when center = 1), e.g. the running moments of saki_moments: the
+ * same factors, outputs, methods, status codes and workspace (SAKI_OP_FIT) as
+ * saki_fit.  SAKI_FLAG_SHRINK needs the calibration rows and is refused
+ * (SAKI_ERR_UNSUPPORTED). */
+SAKI_API saki_status saki_fit_moments(const saki_config* cfg, const float* Sq, const float* Sk,
+                                      const float* mu, const float* A, float* L, float* R, float* nu,
+                                      float* sigma, float* loss, void* workspace, size_t workspace_bytes,
+                                      saki_stream stream);
+
+/* saki_reconstruct_keys -- composition with RoPE (Sec. 6: reconstruct
+ * k_hat = mu + M_r (k - mu) and rotate).  For every query head h and each of
+ * the n_rows code rows rows[i] (device int64, rows of the sketch):
+ *   k_hat = nu_h + L_h c,  so that q^T k_hat is the index's score with the mean
+ *   term (in the paper's head coordinates, where A is absorbed, nu = mu and
+ *   L_h c = M_r (k - mu));
+ * then, when positions (device int64 [n_rows]) is given, rotated by rotary
+ * position embedding at positions[i], rotate-half convention: dimension
+ * j < d/2 pairs with j + d/2 and turns by positions[i] * rope_theta^(-2j/d)
+ * (rope_theta > 1; the angle is formed in fp64).
+ *   sketch [Hq][total_keys][r] dtype, L [Hq][d][r] f32, nu [Hq][d] f32 or NULL,
+ *   keys [Hq][n_rows][d] dtype (written).
+ * Workspace (only with positions): saki_workspace_size(SAKI_OP_RECONSTRUCT,
+ * total_keys = n_rows).  Stream-ordered; uploads nothing. */
+SAKI_API saki_status saki_reconstruct_keys(const saki_config* cfg, int64_t n_rows, const int64_t* rows,
+                                           int64_t total_keys, const void* sketch, const float* L,
+                                           const float* nu, const int64_t* positions, float rope_theta,
+                                           void* keys, void* workspace, size_t workspace_bytes,
+                                           saki_stream stream);
 
 /* saki_build_index -- Sec. 6 key codes c_j = R_h^T (k_j - mu_g) for every query
  * head h and every key row j (all sequences at once).

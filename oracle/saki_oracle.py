@@ -450,3 +450,51 @@ def score_mse(Q, A, K, L, codes, nu, seq_offsets, q_seq, q_visible, group: int, 
             sh = approx_scores(q, L[h], codes[h, base + keys]) + (0.0 if nu is None else q @ np.asarray(nu[h], F64))
             out[h] += (np.sum(s ** 2), np.sum((s - sh) ** 2), len(keys))
     return out
+
+
+# --------------------------------------------------------------------------
+# Online moment tracking (Sec. 2: online updates of Sq, Sk) and composition with
+# RoPE (Sec. 6: reconstruct k_hat = mu + M_r (k - mu) and rotate)
+# --------------------------------------------------------------------------
+def merge_moments(S1, mu1, n1: int, S2, mu2, n2: int, center: bool):
+    """Moments (1/n normalisation) of the union of two batches from each batch's
+    moments: S = (n1 S1 + n2 S2) / n, plus (n1 n2 / n^2) (mu1 - mu2)(mu1 - mu2)^T
+    for centered moments (the pooled-variance identity); mu = (n1 mu1 + n2 mu2) / n."""
+    n = n1 + n2
+    S1, S2 = np.asarray(S1, F64), np.asarray(S2, F64)
+    if n1 == 0:
+        return S2.copy(), np.asarray(mu2, F64).copy()
+    S = (n1 * S1 + n2 * S2) / n
+    if not center:
+        return S, np.zeros(S.shape[0])
+    m1, m2 = np.asarray(mu1, F64), np.asarray(mu2, F64)
+    dm = m1 - m2
+    return S + (n1 * n2 / n ** 2) * np.outer(dm, dm), (n1 * m1 + n2 * m2) / n
+
+
+def rope(x, pos, theta: float):
+    """Rotary position embedding, rotate-half convention: dimension i < d/2 pairs
+    with i + d/2 and turns by pos * theta^(-2i/d)."""
+    x = np.asarray(x, F64)
+    d = x.shape[-1]
+    half = d // 2
+    ang = np.asarray(pos, F64)[..., None] * theta ** (-2.0 * np.arange(half) / d)
+    c, s = np.cos(ang), np.sin(ang)
+    a, b = x[..., :half], x[..., half:]
+    return np.concatenate([a * c - b * s, b * c + a * s], axis=-1)
+
+
+def reconstruct_keys(codes, L, nu, rows, positions=None, theta: float = 10000.0):
+    """k_hat_j = nu_h + L_h c_j for the given code rows of every query head (in the
+    head coordinates of the paper, where A is absorbed, this is
+    mu + M_r (k - mu)); q^T k_hat_j is the index's score with the mean term.
+    With positions, each k_hat_j is then rotated by RoPE at positions[j].
+    codes [Hq][N][r], L [Hq][d][r], nu [Hq][d] or None; returns [Hq][len(rows)][d]."""
+    codes = np.asarray(codes, F64)
+    rows = np.asarray(rows)
+    out = np.einsum("hdr,hnr->hnd", np.asarray(L, F64), codes[:, rows])
+    if nu is not None:
+        out = out + np.asarray(nu, F64)[:, None, :]
+    if positions is not None:
+        out = rope(out, np.asarray(positions)[None, :], theta)
+    return out

@@ -546,6 +546,70 @@ saki_status finish(const saki_config* cfg, saki_status st, const void* workspace
   return read_status(workspace, s);
 }
 
+// The fit after the moments (Prop. 1 / Sec. 6 and the comparison indexes):
+// factors of the moments in the workspace's S, the SVD fit, the method's fold,
+// and the status words.  Shared by saki_fit and saki_fit_moments.
+saki_status fit_from_moments(const saki_config* cfg, const FitWs& w, char* ws, float* muw, const float* A, float* L,
+                             float* R, float* nu, float* sigma, float* loss, cudaStream_t s) {
+  saki_status st;
+  const int Hq = cfg->num_q_heads, Hk = cfg->num_kv_heads, nm = Hq + Hk;
+  float* S = reinterpret_cast<float*>(ws + w.S);
+  float* F = reinterpret_cast<float*>(ws + w.F);
+  float* Gm = reinterpret_cast<float*>(ws + w.G);
+  int* status = reinterpret_cast<int*>(ws + w.st);
+  const int sweeps = cfg->max_sweeps > 0 ? cfg->max_sweeps : 40;
+  // The comparison indexes reuse the fit with other inputs: weight SVD whitens
+  // with identity factors (C' = A); key PCA keeps the key factors and sets the
+  // query factors and the operator to the identity (C' = F_k, whose left singular
+  // vectors are Sk's eigenvectors), then folds A into L.
+  const int method = cfg->method;
+  float* Iw = reinterpret_cast<float*>(ws + w.I);
+  float* sig = (method == SAKI_METHOD_KEY_PCA || method == SAKI_METHOD_SAP_SVD) && !sigma
+                   ? reinterpret_cast<float*>(ws + w.sig) : sigma;
+  {
+    KernelTimer kt(SAKI_KERNEL_FACTOR, s);
+    if (method == SAKI_METHOD_WEIGHT_SVD) {
+      if ((st = cuda_status(launch_identity(F, nm, s))) != SAKI_OK) return st;
+      if ((st = cuda_status(launch_identity(Gm, nm, s))) != SAKI_OK) return st;
+    } else {
+      // SAP-svd needs the symmetric key roots (the right singular vectors of C itself)
+      const int sym_from = method == SAKI_METHOD_SAP_SVD ? Hq : (1 << 30);
+      if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s, sym_from))) !=
+          SAKI_OK)
+        return st;
+    }
+    if (method == SAKI_METHOD_KEY_PCA) {
+      if ((st = cuda_status(launch_identity(F, Hq, s))) != SAKI_OK) return st;
+      if ((st = cuda_status(launch_identity(Gm, Hq, s))) != SAKI_OK) return st;
+      if ((st = cuda_status(launch_identity(Iw, Hq, s))) != SAKI_OK) return st;
+    }
+  }
+  {
+    KernelTimer kt(SAKI_KERNEL_FIT, s);
+    const float* Afit = method == SAKI_METHOD_KEY_PCA ? Iw : A;
+    if ((st = cuda_status(launch_fit(Afit, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
+                                     reinterpret_cast<float*>(ws + w.C), L, R, sig, loss, nu, status, s))) !=
+        SAKI_OK)
+      return st;
+    if (method == SAKI_METHOD_KEY_PCA &&
+        (st = cuda_status(launch_key_pca_fold(A, sig, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, L, R, nu,
+                                              s))) != SAKI_OK)
+      return st;
+    if ((method == SAKI_METHOD_SAP_SVD || method == SAKI_METHOD_SAP_MAP) &&
+        (st = cuda_status(launch_sap_fold(A, F, sig, Hq, Hk, cfg->rank, method == SAKI_METHOD_SAP_SVD, L, R, s))) !=
+            SAKI_OK)
+      return st;
+  }
+  std::vector<int> hst(nm);
+  if ((st = cuda_status(staging().download_sync(hst.data(), status, nm * sizeof(int), s))) != SAKI_OK) return st;
+  int acc = 0;
+  for (int v : hst) acc |= v;
+  if (acc & kStTimeout) return SAKI_ERR_TIMEOUT;
+  if (acc & kStNonFinite) return SAKI_ERR_NUMERIC;
+  if (acc & kStNotConverged) return SAKI_ERR_NOT_CONVERGED;
+  return SAKI_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -676,6 +740,11 @@ size_t saki_workspace_size(const saki_config* cfg, int32_t op, const saki_layout
       return n_calib >= 1 ? fit_ws(cfg).bytes : 0;
     case SAKI_OP_BUILD_INDEX:
       return total_keys >= 0 ? build_ws(cfg, total_keys).bytes : 0;
+    case SAKI_OP_MOMENTS:
+      return kHeader + align_up((size_t)(cfg->num_q_heads + cfg->num_kv_heads) * kD * kD * sizeof(float)) +
+             align_up((size_t)cfg->num_kv_heads * kD * sizeof(float));
+    case SAKI_OP_RECONSTRUCT:   // total_keys: the number of rows to reconstruct
+      return total_keys >= 0 ? std::max<size_t>(kAlign, align_up((size_t)total_keys * (kD / 2) * sizeof(float2))) : 0;
     case SAKI_OP_KEY_SPECTRUM:
       return align_up((size_t)cfg->num_kv_heads * kD * kD * sizeof(float)) +
              align_up((size_t)cfg->num_kv_heads * kD * sizeof(float)) +
@@ -719,11 +788,8 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
   char* ws = static_cast<char*>(workspace);
   const int Hq = cfg->num_q_heads, Hk = cfg->num_kv_heads, nm = Hq + Hk;
   float* S = reinterpret_cast<float*>(ws + w.S);
-  float* F = reinterpret_cast<float*>(ws + w.F);
-  float* Gm = reinterpret_cast<float*>(ws + w.G);
   float* muw = mu ? mu : reinterpret_cast<float*>(ws + w.mu);
   int* status = reinterpret_cast<int*>(ws + w.st);
-  const int sweeps = cfg->max_sweeps > 0 ? cfg->max_sweeps : 40;
   if ((st = cuda_status(cudaMemsetAsync(status, 0, nm * sizeof(int), s))) != SAKI_OK) return st;
   if (!cfg->center && mu && (st = cuda_status(cudaMemsetAsync(mu, 0, (size_t)Hk * kD * sizeof(float), s))) != SAKI_OK)
     return st;
@@ -741,56 +807,85 @@ saki_status saki_fit(const saki_config* cfg, int64_t n_calib, const void* q_cali
       return st;
     if ((st = cuda_status(launch_shrink(S, acc4, n_calib, nm, nullptr, s))) != SAKI_OK) return st;
   }
-  // The comparison indexes reuse the fit with other inputs: weight SVD whitens
-  // with identity factors (C' = A); key PCA keeps the key factors and sets the
-  // query factors and the operator to the identity (C' = F_k, whose left singular
-  // vectors are Sk's eigenvectors), then folds A into L.
-  const int method = cfg->method;
-  float* Iw = reinterpret_cast<float*>(ws + w.I);
-  float* sig = (method == SAKI_METHOD_KEY_PCA || method == SAKI_METHOD_SAP_SVD) && !sigma
-                   ? reinterpret_cast<float*>(ws + w.sig) : sigma;
+  return fit_from_moments(cfg, w, ws, muw, A, L, R, nu, sigma, loss, s);
+}
+
+saki_status saki_moments(const saki_config* cfg, int64_t n_new, const void* q_new, const void* k_new, int64_t n_prev,
+                         float* Sq, float* Sk, float* mu, void* workspace, size_t workspace_bytes,
+                         saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  if (n_new < 1 || n_prev < 0 || !q_new || !k_new || !Sq || !Sk || !workspace) return SAKI_ERR_INVALID_ARGUMENT;
+  if (cfg->center && !mu) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {q_new, k_new, (const void*)Sq, (const void*)Sk, (const void*)mu, (const void*)workspace})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  const int Hq = cfg->num_q_heads, Hk = cfg->num_kv_heads;
+  const size_t off_S = kHeader, off_mu = off_S + align_up((size_t)(Hq + Hk) * kD * kD * sizeof(float));
+  if (workspace_bytes < off_mu + align_up((size_t)Hk * kD * sizeof(float))) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
+  char* ws = static_cast<char*>(workspace);
+  float* Sb = reinterpret_cast<float*>(ws + off_S);
+  float* mub = reinterpret_cast<float*>(ws + off_mu);
+  if ((st = cuda_status(cudaMemsetAsync(ws, 0, sizeof(int), s))) != SAKI_OK) return st;   // the header's error word
   {
-    KernelTimer kt(SAKI_KERNEL_FACTOR, s);
-    if (method == SAKI_METHOD_WEIGHT_SVD) {
-      if ((st = cuda_status(launch_identity(F, nm, s))) != SAKI_OK) return st;
-      if ((st = cuda_status(launch_identity(Gm, nm, s))) != SAKI_OK) return st;
-    } else {
-      // SAP-svd needs the symmetric key roots (the right singular vectors of C itself)
-      const int sym_from = method == SAKI_METHOD_SAP_SVD ? Hq : (1 << 30);
-      if ((st = cuda_status(launch_factor(S, nm, cfg->eig_floor_rel, sweeps, F, Gm, status, s, sym_from))) !=
+    KernelTimer kt(SAKI_KERNEL_MOMENTS, s);
+    if ((st = cuda_status(launch_gram(q_new, k_new, n_new, Hq, Hk, cfg->center, cfg->dtype, Sb, mub,
+                                      reinterpret_cast<int*>(ws), s))) != SAKI_OK)
+      return st;
+  }
+  return finish(cfg, cuda_status(launch_merge_moments(Sq, Sk, mu, Sb, mub, Hq, Hk, n_prev, n_new, cfg->center, s)),
+                ws, s);
+}
+
+saki_status saki_fit_moments(const saki_config* cfg, const float* Sq, const float* Sk, const float* mu,
+                             const float* A, float* L, float* R, float* nu, float* sigma, float* loss,
+                             void* workspace, size_t workspace_bytes, saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  if (cfg->flags & SAKI_FLAG_SHRINK) return SAKI_ERR_UNSUPPORTED;   // needs the calibration rows
+  if (!Sq || !Sk || !A || !L || !R || !workspace) return SAKI_ERR_INVALID_ARGUMENT;
+  if (cfg->center && !mu) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {(const void*)Sq, (const void*)Sk, (const void*)mu, (const void*)A, (const void*)L,
+                        (const void*)R, (const void*)nu, (const void*)sigma, (const void*)loss, (const void*)workspace})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  const FitWs w = fit_ws(cfg);
+  if (workspace_bytes < w.bytes) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (capturing(s)) return SAKI_ERR_UNSUPPORTED;
+  char* ws = static_cast<char*>(workspace);
+  const int Hq = cfg->num_q_heads, Hk = cfg->num_kv_heads, nm = Hq + Hk;
+  float* S = reinterpret_cast<float*>(ws + w.S);
+  float* muw = reinterpret_cast<float*>(ws + w.mu);
+  const size_t mat = (size_t)kD * kD * sizeof(float);
+  if ((st = cuda_status(cudaMemsetAsync(ws + w.st, 0, nm * sizeof(int), s))) != SAKI_OK) return st;
+  if ((st = cuda_status(cudaMemcpyAsync(S, Sq, Hq * mat, cudaMemcpyDeviceToDevice, s))) != SAKI_OK) return st;
+  if ((st = cuda_status(cudaMemcpyAsync(S + (size_t)Hq * kD * kD, Sk, Hk * mat, cudaMemcpyDeviceToDevice, s))) !=
+      SAKI_OK)
+    return st;
+  if (cfg->center &&
+      (st = cuda_status(cudaMemcpyAsync(muw, mu, (size_t)Hk * kD * sizeof(float), cudaMemcpyDeviceToDevice, s))) !=
           SAKI_OK)
-        return st;
-    }
-    if (method == SAKI_METHOD_KEY_PCA) {
-      if ((st = cuda_status(launch_identity(F, Hq, s))) != SAKI_OK) return st;
-      if ((st = cuda_status(launch_identity(Gm, Hq, s))) != SAKI_OK) return st;
-      if ((st = cuda_status(launch_identity(Iw, Hq, s))) != SAKI_OK) return st;
-    }
-  }
-  {
-    KernelTimer kt(SAKI_KERNEL_FIT, s);
-    const float* Afit = method == SAKI_METHOD_KEY_PCA ? Iw : A;
-    if ((st = cuda_status(launch_fit(Afit, F, Gm, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, sweeps,
-                                     reinterpret_cast<float*>(ws + w.C), L, R, sig, loss, nu, status, s))) !=
-        SAKI_OK)
-      return st;
-    if (method == SAKI_METHOD_KEY_PCA &&
-        (st = cuda_status(launch_key_pca_fold(A, sig, cfg->center ? muw : nullptr, Hq, Hk, cfg->rank, L, R, nu,
-                                              s))) != SAKI_OK)
-      return st;
-    if ((method == SAKI_METHOD_SAP_SVD || method == SAKI_METHOD_SAP_MAP) &&
-        (st = cuda_status(launch_sap_fold(A, F, sig, Hq, Hk, cfg->rank, method == SAKI_METHOD_SAP_SVD, L, R, s))) !=
-            SAKI_OK)
-      return st;
-  }
-  std::vector<int> hst(nm);
-  if ((st = cuda_status(staging().download_sync(hst.data(), status, nm * sizeof(int), s))) != SAKI_OK) return st;
-  int acc = 0;
-  for (int v : hst) acc |= v;
-  if (acc & kStTimeout) return SAKI_ERR_TIMEOUT;
-  if (acc & kStNonFinite) return SAKI_ERR_NUMERIC;
-  if (acc & kStNotConverged) return SAKI_ERR_NOT_CONVERGED;
-  return SAKI_OK;
+    return st;
+  return fit_from_moments(cfg, w, ws, muw, A, L, R, nu, sigma, loss, s);
+}
+
+saki_status saki_reconstruct_keys(const saki_config* cfg, int64_t n_rows, const int64_t* rows, int64_t total_keys,
+                                  const void* sketch, const float* L, const float* nu, const int64_t* positions,
+                                  float rope_theta, void* keys, void* workspace, size_t workspace_bytes,
+                                  saki_stream stream) {
+  saki_status st = check_cfg(cfg);
+  if (st != SAKI_OK) return st;
+  if (n_rows < 0 || total_keys < 0 || (n_rows > 0 && (!rows || !sketch || !L || !keys)))
+    return SAKI_ERR_INVALID_ARGUMENT;
+  if (positions && (!(rope_theta > 1.f) || !workspace)) return SAKI_ERR_INVALID_ARGUMENT;
+  for (const void* p : {(const void*)rows, sketch, (const void*)L, (const void*)nu, (const void*)positions,
+                        (const void*)keys, (const void*)workspace})
+    if (p && !al16(p)) return SAKI_ERR_INVALID_ARGUMENT;
+  if (positions && workspace_bytes < (size_t)n_rows * (kD / 2) * sizeof(float2)) return SAKI_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return cuda_status(launch_reconstruct(rows, n_rows, sketch, total_keys, L, nu, cfg->num_q_heads, cfg->rank,
+                                        positions, rope_theta, static_cast<float2*>(workspace), cfg->dtype, keys, s));
 }
 
 saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const void* K, const float* R,

@@ -170,3 +170,135 @@ cudaError_t launch_score_mse(const void* Q, const float* A, const void* K, const
 }
 
 }  // namespace saki
+
+// ---------------------------------------------------------------- online moments, RoPE composition
+namespace saki {
+namespace {
+
+// Running moments (in place, n1 rows so far) merged with a batch's moments (n2
+// rows): S = (n1 S + n2 B) / n, plus (n1 n2 / n^2) (mu1 - mu2)(mu1 - mu2)^T for
+// centered key moments, and mu = (n1 mu1 + n2 mu2) / n (the pooled-variance
+// identity).  One CTA per matrix, queries first.
+__global__ void __launch_bounds__(256) merge_moments_kernel(float* Sq, float* Sk, float* mu, const float* Sb,
+                                                            const float* mub, int Hq, int64_t n1, int64_t n2,
+                                                            int center) {
+  __shared__ float dm[kD];
+  const int m = blockIdx.x, tid = threadIdx.x;
+  const bool key = m >= Hq;
+  const int g = m - Hq;
+  float* S = key ? Sk + (int64_t)g * kD * kD : Sq + (int64_t)m * kD * kD;
+  const float* B = Sb + (int64_t)m * kD * kD;
+  const double n = (double)(n1 + n2);
+  const double w1 = (double)n1 / n, w2 = (double)n2 / n, c = (double)n1 * (double)n2 / (n * n);
+  const bool cen = key && center;
+  if (tid < kD) dm[tid] = cen && n1 > 0 ? mu[(int64_t)g * kD + tid] - mub[(int64_t)g * kD + tid] : 0.f;
+  __syncthreads();
+  for (int o = tid; o < kD * kD; o += 256) {
+    const int i = o / kD, j = o % kD;
+    const double v = w1 * (n1 > 0 ? (double)S[o] : 0.0) + w2 * B[o] + (cen ? c * (double)dm[i] * dm[j] : 0.0);
+    S[o] = (float)v;
+  }
+  if (key && tid < kD && mu) {
+    const double m1 = n1 > 0 ? (double)mu[(int64_t)g * kD + tid] : 0.0;
+    mu[(int64_t)g * kD + tid] = center ? (float)(w1 * m1 + w2 * mub[(int64_t)g * kD + tid]) : 0.f;
+  }
+}
+
+// cos and sin of pos * theta^(-2j/d) for j < d/2: the angle in fp64, reduced
+// modulo 2 pi before the fp32 evaluation (positions up to 2^31 keep ~1e-7 rad).
+__global__ void rope_table_kernel(const int64_t* positions, int64_t n_rows, float theta, float2* table) {
+  const int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (idx >= n_rows * (kD / 2)) return;
+  const int j = (int)(idx % (kD / 2));
+  const double inv = pow((double)theta, -2.0 * j / kD);
+  double ang = fmod((double)positions[idx / (kD / 2)] * inv, 6.283185307179586476925);
+  float sn, cs;
+  sincosf((float)ang, &sn, &cs);
+  table[idx] = make_float2(cs, sn);
+}
+
+// k_hat = nu_h + L_h c for the requested code rows of every query head, then
+// (with a table) the rotate-half RoPE rotation: dimension i < d/2 pairs with
+// i + d/2.  One warp per (row, head); L_h transposed in shared memory ([c][i],
+// conflict-free); lane l holds dimensions l, l+32, l+64, l+96, so both members
+// of each rotated pair sit in the same lane.
+template <typename Tout, typename Tin>
+__global__ void __launch_bounds__(256) reconstruct_kernel(const int64_t* rows, int64_t n_rows, const Tin* codes,
+                                                          int64_t N, const float* L, const float* nu, int r,
+                                                          const float2* table, Tout* out) {
+  extern __shared__ float sm[];
+  float* Lt = sm;                 // [r][d]
+  float* cs = Lt + r * kD;        // [8][r] code rows of the block's warps
+  const int h = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* Lh = L + (int64_t)h * kD * r;
+  for (int o = tid; o < kD * r; o += 256) Lt[(o % r) * kD + o / r] = Lh[o];
+  __syncthreads();
+  const int64_t row = blockIdx.x * 8ll + warp;
+  if (row >= n_rows) return;
+  const int64_t key = rows[row];
+  float* c = cs + warp * r;
+  for (int i = lane; i < r; i += 32) c[i] = Vec<Tin>::load1(codes + ((int64_t)h * N + key) * r + i);
+  __syncwarp();
+  float x[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) x[e] = nu ? nu[(int64_t)h * kD + lane + 32 * e] : 0.f;
+  for (int k = 0; k < r; ++k) {
+    const float ck = c[k];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) x[e] = fmaf(Lt[k * kD + lane + 32 * e], ck, x[e]);
+  }
+  if (table) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const float2 t = table[row * (kD / 2) + lane + 32 * e];
+      const float a = x[e], b = x[e + 2];
+      x[e] = a * t.x - b * t.y;
+      x[e + 2] = b * t.x + a * t.y;
+    }
+  }
+  Tout* o = out + ((int64_t)h * n_rows + row) * kD;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) o[lane + 32 * e] = from_float<Tout>(x[e]);
+}
+
+}  // namespace
+
+cudaError_t launch_merge_moments(float* Sq, float* Sk, float* mu, const float* Sb, const float* mub, int Hq, int Hk,
+                                 int64_t n1, int64_t n2, int center, cudaStream_t s) {
+  note_launch();
+  merge_moments_kernel<<<Hq + Hk, 256, 0, s>>>(Sq, Sk, mu, Sb, mub, Hq, n1, n2, center);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_reconstruct(const int64_t* rows, int64_t n_rows, const void* codes, int64_t N, const float* L,
+                               const float* nu, int Hq, int r, const int64_t* positions, float theta, float2* table,
+                               int dtype, void* out, cudaStream_t s) {
+  if (n_rows == 0) return cudaSuccess;
+  if (positions) {
+    const int64_t n = n_rows * (kD / 2);
+    note_launch();
+    rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(positions, n_rows, theta, table);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  const float2* tab = positions ? table : nullptr;
+  const dim3 grid((unsigned)((n_rows + 7) / 8), Hq);
+  const int smem = (int)(sizeof(float) * (r * kD + 8 * r));
+  note_launch();
+  if (dtype == SAKI_BF16) {
+    auto kern = reconstruct_kernel<__nv_bfloat16, __nv_bfloat16>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, 256, smem, s>>>(rows, n_rows, static_cast<const __nv_bfloat16*>(codes), N, L, nu, r, tab,
+                                 static_cast<__nv_bfloat16*>(out));
+  } else {
+    auto kern = reconstruct_kernel<float, float>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, 256, smem, s>>>(rows, n_rows, static_cast<const float*>(codes), N, L, nu, r, tab,
+                                 static_cast<float*>(out));
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace saki

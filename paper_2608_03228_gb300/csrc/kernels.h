@@ -198,4 +198,14 @@ cudaError_t launch_score_mse(const void* Q, const float* A, const void* K, const
                              const float* nu, const int64_t* qinfo, int64_t T, int64_t N, int Hq, int G, int r,
                              int64_t stride, int dtype, double* out, cudaStream_t s);
 
+// ---------------------------------------------------------------- online moments, RoPE composition
+// running moments (Sq [Hq], Sk [Hk], mu [Hk], n1 rows) merged in place with a batch's (Sb [(Hq+Hk)], mub, n2 rows)
+cudaError_t launch_merge_moments(float* Sq, float* Sk, float* mu, const float* Sb, const float* mub, int Hq, int Hk,
+                                 int64_t n1, int64_t n2, int center, cudaStream_t s);
+// k_hat = nu + L c of the given code rows per query head, RoPE-rotated when positions are given
+// (table: workspace of n_rows * d/2 float2)
+cudaError_t launch_reconstruct(const int64_t* rows, int64_t n_rows, const void* codes, int64_t N, const float* L,
+                               const float* nu, int Hq, int r, const int64_t* positions, float theta, float2* table,
+                               int dtype, void* out, cudaStream_t s);
+
 }  // namespace saki

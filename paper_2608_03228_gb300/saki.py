@@ -24,13 +24,14 @@ SAKI_METHOD_SAKI, SAKI_METHOD_KEY_PCA, SAKI_METHOD_WEIGHT_SVD, SAKI_METHOD_SAP_S
 METHODS = {"saki": SAKI_METHOD_SAKI, "key_pca": SAKI_METHOD_KEY_PCA, "weight_svd": SAKI_METHOD_WEIGHT_SVD,
            "sap_svd": SAKI_METHOD_SAP_SVD, "sap_map": SAKI_METHOD_SAP_MAP}
 SAKI_OP_FIT, SAKI_OP_BUILD_INDEX, SAKI_OP_SCORE_TOPK, SAKI_OP_RECALL = 0, 1, 2, 3
-SAKI_OP_KEY_SPECTRUM, SAKI_OP_SCORE_MSE = 4, 5
+SAKI_OP_KEY_SPECTRUM, SAKI_OP_SCORE_MSE, SAKI_OP_MOMENTS, SAKI_OP_RECONSTRUCT = 4, 5, 6, 7
 STATUS = {0: "SAKI_OK", 1: "SAKI_ERR_INVALID_ARGUMENT", 2: "SAKI_ERR_UNSUPPORTED", 3: "SAKI_ERR_CUDA",
           4: "SAKI_ERR_NUMERIC", 5: "SAKI_ERR_NOT_CONVERGED", 6: "SAKI_ERR_WORKSPACE", 7: "SAKI_ERR_TIMEOUT"}
 EXPORTS = ("saki_workspace_size", "saki_fit", "saki_build_index", "saki_score_topk", "saki_recall",
            "saki_status_string", "saki_version", "saki_score_topk_noalloc", "saki_launch_count",
            "saki_kernel_timer_start", "saki_kernel_timer_stop", "saki_workspace_status", "saki_noalloc_status",
-           "saki_debug_inject_stall", "saki_merge_topk", "saki_key_spectrum", "saki_score_mse")
+           "saki_debug_inject_stall", "saki_merge_topk", "saki_key_spectrum", "saki_score_mse",
+           "saki_moments", "saki_fit_moments", "saki_reconstruct_keys")
 SAKI_KERNEL_SELECT, SAKI_KERNEL_EXACT, SAKI_KERNEL_FIT, SAKI_KERNEL_MOMENTS, SAKI_KERNEL_BUILD, SAKI_KERNEL_FACTOR = (
     1, 2, 3, 4, 5, 6)
 SAKI_NOALLOC_SCRATCH_BYTES = 16 << 20
@@ -73,6 +74,13 @@ _lib.saki_key_spectrum.restype = ctypes.c_int
 _lib.saki_key_spectrum.argtypes = [ctypes.POINTER(Config), _i64, _vp, ctypes.c_float, _vp, _vp, _vp, _sz, _vp]
 _lib.saki_score_mse.restype = ctypes.c_int
 _lib.saki_score_mse.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(Layout), _i64] + [_vp] * 8 + [_sz, _vp]
+_lib.saki_moments.restype = ctypes.c_int
+_lib.saki_moments.argtypes = [ctypes.POINTER(Config), _i64, _vp, _vp, _i64, _vp, _vp, _vp, _vp, _sz, _vp]
+_lib.saki_fit_moments.restype = ctypes.c_int
+_lib.saki_fit_moments.argtypes = [ctypes.POINTER(Config)] + [_vp] * 10 + [_sz, _vp]
+_lib.saki_reconstruct_keys.restype = ctypes.c_int
+_lib.saki_reconstruct_keys.argtypes = [ctypes.POINTER(Config), _i64, _vp, _i64, _vp, _vp, _vp, _vp, ctypes.c_float,
+                                       _vp, _vp, _sz, _vp]
 _lib.saki_status_string.restype = ctypes.c_char_p
 _lib.saki_status_string.argtypes = [ctypes.c_int]
 _lib.saki_version.restype = ctypes.c_char_p
@@ -198,6 +206,33 @@ def saki_score_mse(cfg: Config, layout: HostLayout, Q, A, K, L, sketch, out, nu=
     _check(_lib.saki_score_mse(ctypes.byref(cfg), ctypes.byref(layout.c), int(key_stride), _ptr(Q), _ptr(A), _ptr(K),
                                _ptr(L), _ptr(sketch), _ptr(nu), _ptr(out), _ptr(ws), ws.numel(), _stream(stream)),
            "saki_score_mse")
+
+
+def saki_moments(cfg: Config, q_new, k_new, n_prev, Sq, Sk, mu=None, workspace=None, stream=None) -> None:
+    """Add a batch of calibration rows to running moments covering n_prev rows."""
+    need = saki_workspace_size(cfg, SAKI_OP_MOMENTS)
+    ws = workspace if workspace is not None else _workspace(need, q_new.device)
+    _check(_lib.saki_moments(ctypes.byref(cfg), q_new.shape[1], _ptr(q_new), _ptr(k_new), int(n_prev), _ptr(Sq),
+                             _ptr(Sk), _ptr(mu), _ptr(ws), ws.numel(), _stream(stream)), "saki_moments")
+
+
+def saki_fit_moments(cfg: Config, Sq, Sk, A, L, R, mu=None, nu=None, sigma=None, loss=None, workspace=None,
+                     stream=None) -> None:
+    need = saki_workspace_size(cfg, SAKI_OP_FIT, n_calib=1)
+    ws = workspace if workspace is not None else _workspace(need, Sq.device)
+    _check(_lib.saki_fit_moments(ctypes.byref(cfg), _ptr(Sq), _ptr(Sk), _ptr(mu), _ptr(A), _ptr(L), _ptr(R), _ptr(nu),
+                                 _ptr(sigma), _ptr(loss), _ptr(ws), ws.numel(), _stream(stream)), "saki_fit_moments")
+
+
+def saki_reconstruct_keys(cfg: Config, rows, sketch, L, keys, nu=None, positions=None, rope_theta=10000.0,
+                          workspace=None, stream=None) -> None:
+    """k_hat = nu + L c of the given code rows (device int64) of every head, RoPE-rotated at positions."""
+    n = rows.numel()
+    need = saki_workspace_size(cfg, SAKI_OP_RECONSTRUCT, total_keys=n)
+    ws = workspace if workspace is not None else _workspace(need, sketch.device)
+    _check(_lib.saki_reconstruct_keys(ctypes.byref(cfg), n, _ptr(rows), sketch.shape[1], _ptr(sketch), _ptr(L),
+                                      _ptr(nu), _ptr(positions), float(rope_theta), _ptr(keys), _ptr(ws), ws.numel(),
+                                      _stream(stream)), "saki_reconstruct_keys")
 
 
 def saki_merge_topk(cfg: Config, idx_parts, score_parts, part_offsets, idx, score=None, stream=None) -> None:

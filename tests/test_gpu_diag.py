@@ -23,8 +23,9 @@ def test_fit_with_ledoit_wolf_shrinkage(lib, center, dtype, n):
     cfg = lib.make_config(Hq, Hk, r, 16, dtype, center=center, flags=lib.SAKI_FLAG_SHRINK)
     L = torch.empty((Hq, D, r), device="cuda")
     R = torch.empty_like(L)
+    mu = torch.empty((Hk, D), device="cuda")
     ws = torch.empty(lib.saki_workspace_size(cfg, lib.SAKI_OP_FIT, n_calib=n), dtype=torch.uint8, device="cuda")
-    lib.saki_fit(cfg, to_dev(data["q_calib"], dtype), to_dev(data["k_calib"], dtype), f32(data["A"]), L, R,
+    lib.saki_fit(cfg, to_dev(data["q_calib"], dtype), to_dev(data["k_calib"], dtype), f32(data["A"]), L, R, mu=mu,
                  workspace=ws)
     torch.cuda.synchronize()
     nm = Hq + Hk

@@ -603,3 +603,53 @@ def test_score_mse_reduction_by_double_loop_and_full_rank():
     codes = O.build_index(K, res["R"], res["mu"], "f32", 1)
     out = O.score_mse(Q[:1], A[:1], K, res["L"], codes, res["nu"], off, q_seq, q_vis, group=1)
     assert out[0, 1] <= 1e-12 * out[0, 0]
+
+
+# ------------------------------------------- online moments, RoPE composition
+@pytest.mark.parametrize("center", [False, True])
+def test_merged_moments_equal_the_moments_of_the_union(center):
+    rng = np.random.default_rng(41)
+    X1 = rng.standard_normal((37, 10)) + 1.0
+    X2 = rng.standard_normal((91, 10)) * 2.0 - 0.5
+    S1, m1 = O.moments(X1, center)
+    S2, m2 = O.moments(X2, center)
+    S, mu = O.merge_moments(S1, m1, 37, S2, m2, 91, center)
+    Su, mu_u = O.moments(np.concatenate([X1, X2]), center)
+    np.testing.assert_allclose(S, Su, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(mu, mu_u, rtol=1e-12, atol=1e-12)
+    S0, mu0 = O.merge_moments(np.zeros((10, 10)), np.zeros(10), 0, S2, m2, 91, center)
+    np.testing.assert_allclose(S0, S2)
+
+
+def test_rope_hand_example_and_relative_positions():
+    # d = 4: pairs (0, 2) and (1, 3) turn by pos and pos / 100 (theta = 10^4)
+    x = np.array([1.0, 2.0, 3.0, 4.0])
+    got = O.rope(x, 1.0, 10000.0)
+    c0, s0, c1, s1 = np.cos(1.0), np.sin(1.0), np.cos(0.01), np.sin(0.01)
+    np.testing.assert_allclose(got, [1 * c0 - 3 * s0, 2 * c1 - 4 * s1, 3 * c0 + 1 * s0, 4 * c1 + 2 * s1], rtol=1e-15)
+    rng = np.random.default_rng(42)
+    q, k = rng.standard_normal(16), rng.standard_normal(16)
+    assert np.linalg.norm(O.rope(k, 37.0, 500.0)) == pytest.approx(np.linalg.norm(k))
+    base = O.rope(q, 3.0, 500.0) @ O.rope(k, 11.0, 500.0)
+    assert O.rope(q, 103.0, 500.0) @ O.rope(k, 111.0, 500.0) == pytest.approx(base, rel=1e-12)
+
+
+def test_reconstructed_keys_reproduce_the_index_scores_and_the_keys_at_full_rank():
+    rng = np.random.default_rng(43)
+    d = 12
+    A = rng.standard_normal((1, d, d))
+    kc = rng.standard_normal((400, d)) + 1.0
+    qc = rng.standard_normal((400, d))
+    K = rng.standard_normal((1, 20, d)) + 1.0
+    q = rng.standard_normal(d)
+    for r in (4, d):
+        res = O.fit(qc[None], kc[None], A, r, center=True)
+        codes = O.build_index(K, res["R"], res["mu"], "f32", 1)
+        rows = np.array([3, 0, 19, 7])
+        kh = O.reconstruct_keys(codes, res["L"], res["nu"], rows)
+        s_hat = O.approx_scores(q, res["L"][0], codes[0, rows]) + q @ res["nu"][0]
+        np.testing.assert_allclose(kh[0] @ q, s_hat, rtol=1e-10, atol=1e-10)
+        if r == d:   # M_d = A: the reconstruction is A k itself
+            np.testing.assert_allclose(kh[0], K[0, rows] @ A[0].T, rtol=2e-5, atol=2e-5)
+    rot = O.reconstruct_keys(codes, res["L"], res["nu"], rows, positions=[5, 6, 7, 8], theta=10000.0)
+    np.testing.assert_allclose(rot[0], O.rope(kh[0], np.array([5, 6, 7, 8]), 10000.0), rtol=1e-14)
