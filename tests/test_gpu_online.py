@@ -76,22 +76,21 @@ def test_reconstructed_keys_with_rope(lib, dtype):
             tol = (2.0 ** -8 if dtype == "bf16" else 0.0) * np.abs(ref) + 1e-5 * scale
             assert np.all(np.abs(got - ref) <= tol), (theta, p is None, np.abs(got - ref).max())
     # without rotation q^T k_hat is the index's score: the selection reports the same
+    if dtype != "f32":
+        return
     T = 3
-    Q = synth.round_to_bf16_grid(rng.standard_normal((Hq, T, D)).astype(np.float32))
+    Q = rng.standard_normal((Hq, T, D)).astype(np.float32)
     lay = lib.HostLayout(np.array([0, N]), np.zeros(T, np.int32), np.full(T, N))
     idx = torch.empty((Hq, T, k), dtype=torch.int32, device="cuda")
     sc = torch.empty((Hq, T, k), dtype=torch.float32, device="cuda")
-    cfg1 = lib.make_config(Hq, Hk, r, k, dtype, center=1)
-    lib.saki_score_topk(cfg1, lay, to_dev(Q, dtype), f32(L), skd, idx, score=sc, nu=f32(nu))
+    lib.saki_score_topk(lib.make_config(Hq, Hk, r, k, "f32", center=1), lay, to_dev(Q, "f32"), f32(L), skd, idx,
+                        score=sc, nu=f32(nu))
+    kh = torch.empty((Hq, k, D), dtype=torch.float32, device="cuda")
     for t in range(T):
         sel = idx[:, t].cpu().numpy()
         for h in range(Hq):
-            kh = torch.empty((Hq, k, D), dtype=torch.float32, device="cuda")
-            lib.saki_reconstruct_keys(lib.make_config(Hq, Hk, r, k, "f32") if dtype == "f32" else cfg,
-                                      torch.from_numpy(sel[h].astype(np.int64)).cuda(), skd, f32(L),
-                                      kh if dtype == "f32" else kh.to(torch.bfloat16), nu=f32(nu))
-            if dtype != "f32":
-                continue
+            lib.saki_reconstruct_keys(cfg, torch.from_numpy(sel[h].astype(np.int64)).cuda(), skd, f32(L), kh,
+                                      nu=f32(nu))
             s = kh[h].cpu().numpy().astype(np.float64) @ Q[h, t].astype(np.float64)
             ref = sc[h, t].cpu().numpy()
             np.testing.assert_allclose(s, ref, atol=SCORE_REL * np.abs(ref).max(), rtol=0)
