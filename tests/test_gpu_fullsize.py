@@ -192,8 +192,38 @@ def test_fullsize_exact_llama31(lib, llama):
 
 
 # ------------------------------------------------------------------ the other workloads
-@pytest.mark.parametrize("name", ["qwen25_7b_t4096_r32", "llama32_3b_t4096_r32", "decode_n1m_b1_r32",
-                                  "decode_n1m_b8_r32", "ragged64_mistral7b_r64"])
+@pytest.mark.parametrize("name", ["qwen25_7b_t4096_r32_n512", "qwen25_7b_t4096_r32_n32768"])
+def test_fullsize_fit_calibration_sweep(lib, name):
+    """saki_fit over all 784 Qwen2.5-7B-shaped heads at the ends of the
+    calibration-length sweep (512 and 32,768 tokens, Fig. 2A); M_r, sigma and
+    loss of sampled heads against the oracle."""
+    torch = _torch()
+    w = synth.WORKLOADS[name]
+    data = synth.make_torch(w, "cuda")
+    Hq, Hk, r = w.num_q_heads, w.num_kv_heads, w.rank
+    cfg = lib.make_config(Hq, Hk, r, w.topk, w.dtype)
+    L = torch.empty((Hq, D, r), device="cuda")
+    R = torch.empty((Hq, D, r), device="cuda")
+    sig = torch.empty((Hq, D), device="cuda")
+    loss = torch.empty((Hq,), device="cuda")
+    lib.saki_fit(cfg, data["q_calib"], data["k_calib"], data["A"], L, R, sigma=sig, loss=loss)
+    torch.cuda.synchronize()
+    for h in (0, 391, Hq - 1):
+        g = h // w.group
+        ref = O.fit(_host(data["q_calib"][h:h + 1]), _host(data["k_calib"][g:g + 1]),
+                    _host(data["A"][h:h + 1]), r, center=False)
+        s_ref = ref["sigma"][0]
+        if (s_ref[r - 1] - s_ref[r]) / s_ref[0] >= 1e-3:
+            assert map_rel_err(L[h].cpu().numpy(), R[h].cpu().numpy(), ref["M"][0]) <= MAP_REL, h
+        np.testing.assert_allclose(sig[h].cpu().numpy(), s_ref, atol=1e-4 * s_ref[0], rtol=0)
+        np.testing.assert_allclose(loss[h].item(), ref["loss"][0], rtol=1e-4, atol=1e-4 * np.sum(s_ref ** 2))
+    del data
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("name", ["qwen25_7b_t4096_r32", "qwen25_7b_t4096_r16", "qwen25_7b_t4096_r64",
+                                  "llama32_3b_t4096_r32", "decode_n1m_b1_r32", "decode_n1m_b8_r32",
+                                  "ragged64_mistral7b_r64"])
 def test_fullsize_select_workloads(lib, name):
     """Approximate and exact selection at each workload's full size."""
     torch = _torch()
