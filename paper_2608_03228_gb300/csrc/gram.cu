@@ -90,8 +90,14 @@ __device__ __forceinline__ void gram_load(const __nv_bfloat16* X, int64_t n, int
   }
 }
 
+// Rows [r0, r0 + nrows) of each matrix's n rows; the 1/n-scaled Gram is
+// written (add = 0) or added to S (add = 1).  The tensor core's fp32
+// accumulation is exact per product but its long sums drift (32,768 rows left
+// the moments about 2e-4 low), so the host cuts n into launches of at most
+// kGramRows rows and the partial moments are summed in S.
 __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, const __nv_bfloat16* Xk, int64_t n,
-                                                      int Hq, float* S, int* err) {
+                                                      int Hq, int64_t r0, int64_t nrows, int add, float* S,
+                                                      int* err) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* done = reinterpret_cast<uint64_t*>(smem + 2 * 16384);   // [2] MMA completion per tile
@@ -100,7 +106,8 @@ __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, c
   volatile int* abort_f = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const int tid = threadIdx.x, warp = tid >> 5;
   const int m = blockIdx.x;
-  const __nv_bfloat16* X = m < Hq ? Xq + (int64_t)m * n * kD : Xk + (int64_t)(m - Hq) * n * kD;
+  const __nv_bfloat16* X = (m < Hq ? Xq + (int64_t)m * n * kD : Xk + (int64_t)(m - Hq) * n * kD) + r0 * kD;
+  const int64_t nl = nrows;
   if (tid == 0) {
     tc::mbar_init(done, 1);
     tc::mbar_init(done + 1, 1);
@@ -117,15 +124,15 @@ __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, c
   tc::fence_after_sync();
   const uint32_t tmem = *tmem_slot;
   const int kb = tid & 7, mb = tid >> 3;   // this thread's 8 x 8 block: rows 8kb.., dimensions 8mb..
-  const int nch = (int)((n + kGramChunk - 1) / kGramChunk);
+  const int nch = (int)((nl + kGramChunk - 1) / kGramChunk);
   constexpr uint32_t idesc = tc::idesc_bf16(128, 128);
   uint4 w[8];
-  gram_load(X, n, 0, kb, mb, w);
+  gram_load(X, nl, 0, kb, mb, w);
   bool ok = true;
   for (int c = 0; c < nch; ++c) {
     const int b = c & 1;
     uint4 wn[8];
-    if (c + 1 < nch) gram_load(X, n, (int64_t)(c + 1) * kGramChunk, kb, mb, wn);
+    if (c + 1 < nch) gram_load(X, nl, (int64_t)(c + 1) * kGramChunk, kb, mb, wn);
     if (c >= 2) ok = tc::mbar_wait(done + b, ((c >> 1) & 1) ^ 1, abort_f);
     if (!__syncthreads_and(ok)) break;
     uint8_t* tile = smem + b * 16384;
@@ -174,10 +181,16 @@ __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, c
       tc::tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + c0, r);
       tc::tmem_ld_wait();
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        *reinterpret_cast<float4*>(Sm + c0 + 4 * q) =
-            make_float4(__uint_as_float(r[4 * q]) * inv, __uint_as_float(r[4 * q + 1]) * inv,
-                        __uint_as_float(r[4 * q + 2]) * inv, __uint_as_float(r[4 * q + 3]) * inv);
+      for (int q = 0; q < 8; ++q) {
+        float4 v = make_float4(__uint_as_float(r[4 * q]) * inv, __uint_as_float(r[4 * q + 1]) * inv,
+                               __uint_as_float(r[4 * q + 2]) * inv, __uint_as_float(r[4 * q + 3]) * inv);
+        float4* dst = reinterpret_cast<float4*>(Sm + c0 + 4 * q);
+        if (add) {
+          const float4 o = *dst;
+          v.x += o.x; v.y += o.y; v.z += o.z; v.w += o.w;
+        }
+        *dst = v;
+      }
     }
   } else if (tid == 0) {
     atomicOr(err, kStTimeout);
@@ -186,6 +199,8 @@ __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, c
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 128);
 }
+
+constexpr int64_t kGramRows = 4096;   // rows per tensor-core moment launch
 
 template <typename Tin>
 cudaError_t gram_t(const void* q, const void* k, int64_t n, int Hq, int Hk, int center, float* S,
@@ -202,10 +217,13 @@ cudaError_t gram_t(const void* q, const void* k, int64_t n, int Hq, int Hk, int 
     if (ntc > 0 && n > 0) {
       e = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kGramSmem);
       if (e != cudaSuccess) return e;
-      note_launch();
-      gram_tc_kernel<<<ntc, 128, kGramSmem, s>>>(static_cast<const __nv_bfloat16*>(q),
-                                                 static_cast<const __nv_bfloat16*>(k), n, Hq, S, err);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      for (int64_t r0 = 0; r0 < n; r0 += kGramRows) {
+        note_launch();
+        gram_tc_kernel<<<ntc, 128, kGramSmem, s>>>(static_cast<const __nv_bfloat16*>(q),
+                                                   static_cast<const __nv_bfloat16*>(k), n, Hq, r0,
+                                                   n - r0 < kGramRows ? n - r0 : kGramRows, r0 > 0 ? 1 : 0, S, err);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      }
     }
     first_cuda = ntc;
   }

@@ -245,22 +245,47 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
   }
 }
 
+// The merge of a row's per-split lists (each sorted, striped over a warp): the
+// block's four warps each merge every fourth split, the next split's keys
+// loaded while the current one is merged (a global load per split would
+// otherwise sit on the critical path, split after split), and warp 0 merges
+// the other three warps' lists in through shared memory.
 template <typename Tin, int KP>
 __global__ void __launch_bounds__(128) merge_kernel(const ScoreArgs a) {
   constexpr int EK = KP / 32;
-  const int lane = threadIdx.x & 31;
-  const int m = blockIdx.x * 4 + (threadIdx.x >> 5);
-  if (m >= a.n_merges) return;
+  __shared__ uint64_t part[3][KP];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int m = blockIdx.x;
   const int h = blockIdx.y;
   const MergeItem mi = a.merges[m];
   const uint64_t* c = a.cand + ((int64_t)h * a.cand_per_head + mi.cand) * KP;
-  uint64_t best[EK], other[EK];
+  uint64_t best[EK], nxt[EK], cur[EK];
+  int sp = warp;
 #pragma unroll
-  for (int e = 0; e < EK; ++e) best[e] = c[e * 32 + lane];
-  for (int s = 1; s < mi.nsplit; ++s) {
+  for (int e = 0; e < EK; ++e) best[e] = sp < mi.nsplit ? c[(int64_t)sp * KP + e * 32 + lane] : 0ull;
+  sp += 4;
 #pragma unroll
-    for (int e = 0; e < EK; ++e) other[e] = c[(int64_t)s * KP + e * 32 + lane];
-    warp_merge_top<EK>(best, other);
+  for (int e = 0; e < EK; ++e) nxt[e] = sp < mi.nsplit ? c[(int64_t)sp * KP + e * 32 + lane] : 0ull;
+  while (sp < mi.nsplit) {
+    const int sn = sp + 4;
+#pragma unroll
+    for (int e = 0; e < EK; ++e) {
+      cur[e] = nxt[e];
+      nxt[e] = sn < mi.nsplit ? c[(int64_t)sn * KP + e * 32 + lane] : 0ull;
+    }
+    warp_merge_top<EK>(best, cur);
+    sp = sn;
+  }
+  if (warp > 0) {
+#pragma unroll
+    for (int e = 0; e < EK; ++e) part[warp - 1][e * 32 + lane] = best[e];
+  }
+  __syncthreads();
+  if (warp > 0) return;
+  for (int j = 0; j < 3; ++j) {
+#pragma unroll
+    for (int e = 0; e < EK; ++e) cur[e] = part[j][e * 32 + lane];
+    warp_merge_top<EK>(best, cur);
   }
   if (a.seed_out) {
     // the row's k-th best key over the merged lists (0 while fewer than k)
@@ -730,7 +755,7 @@ cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, 
 
 cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s) {
   if (a.n_merges == 0) return cudaSuccess;
-  dim3 grid((a.n_merges + 3) / 4, a.Hq);
+  dim3 grid(a.n_merges, a.Hq);
   if (dtype == SAKI_BF16) {
     if (kp == 64) {
       note_launch();
