@@ -159,9 +159,9 @@ class GpuPath:
             ev[4].record()
 
     def recall_with(self, method):
-        """Median recall of a Tab. 1 comparison index (key PCA, weight SVD) on the
-        same data through the same calls (untimed; overwrites the step's index,
-        selections and recall)."""
+        """Median recall of a Tab. 1 comparison index (key PCA, weight SVD) or a
+        Sec. 6 projector variant (SAP-svd, SAP-map) on the same data through the
+        same calls (untimed; overwrites the step's index, selections and recall)."""
         S, d, w, torch = self.saki, self.data, self.w, self.torch
         cfg = S.make_config(w.num_q_heads, w.num_kv_heads, w.rank, w.topk, w.dtype, center=w.center, method=method)
         need = S.saki_workspace_size(cfg, S.SAKI_OP_FIT, n_calib=w.n_calib)
@@ -272,7 +272,7 @@ def run_ours(args, w):
     }
     if args.baselines:
         line["recall_median_by_index"] = {"saki": line["recall_median"],
-                                          **{m: g.recall_with(m) for m in ("key_pca", "weight_svd")}}
+                                          **{m: g.recall_with(m) for m in ("sap_map", "sap_svd", "key_pca", "weight_svd")}}
     if not args.no_extras and world == 1 and args.workload == "llama31_8b_t4096_r32" and not args.heads:
         del g
         torch.cuda.empty_cache()
@@ -598,7 +598,7 @@ def main():
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the decode, ragged and rank/calibration-sweep workloads timed after the headline step")
     ap.add_argument("--baselines", action="store_true",
-                    help="also report the median recall of the key-PCA and weight-SVD indexes (Tab. 1), untimed")
+                    help="also report the median recall of the SAP-map, SAP-svd, key-PCA and weight-SVD indexes (Sec. 6, Tab. 1), untimed")
     ap.add_argument("--heads", type=int, default=0,
                     help="query heads (KV heads follow the workload's group size): a smaller case of the same "
                          "shapes, for profiler captures")

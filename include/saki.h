@@ -101,7 +101,9 @@ typedef enum saki_dtype { SAKI_F32 = 0, SAKI_BF16 = 1 } saki_dtype;
                                     L = A_h Q, R = Q */
 #define SAKI_METHOD_SAP_MAP 4    /* Sec. 6 projector variant: M = A_h Q Q^T with Q an
                                     orthonormal basis (Gram-Schmidt, in column order) of the
-                                    optimum's key-side span, span(Sk^{+1/2} V_r);
+                                    optimum's key-side span, span((Sk^{1/2})^+ V_r),
+                                    (Sk^{1/2})^+ the pseudo-inverse of the symmetric root
+                                    under the eigenvalue floor;
                                     L = A_h Q, R = Q */
 
 typedef struct saki_config {

@@ -664,8 +664,9 @@ __global__ void __launch_bounds__(kD) key_pca_fold_kernel(const float* A, const 
 // The projector variants of Sec. 6 (SAP-svd, SAP-map) from a SAKI fit: an
 // orthonormal basis Q of an r-dimensional key subspace, the map M = A_h Q Q^T
 // folded as R = Q, L = A_h Q (nu = A_h mu is the fit's).  SAP-map takes the
-// optimum's key-side span, span(Sk^{+1/2} V_r): the columns of the fit's R
-// (Sk^{+1/2} V_r Sigma_r^{1/2} whatever factor of Sk whitened it), in order.
+// optimum's key-side span, span((Sk^{1/2})^+ V_r) with (Sk^{1/2})^+ the
+// pseudo-inverse of the root: the columns of the fit's R
+// ((Sk^{1/2})^+ V_r Sigma_r^{1/2} whatever factor of Sk whitened it), in order.
 // SAP-svd takes the raw right singular vectors V_r of C: with the symmetric key
 // root F_k = Sk^{1/2} (factor kernel, sym_from) the fit's R gives
 // V_r = F_k R Sigma_r^{-1/2}.  Either basis is orthonormalised by modified
