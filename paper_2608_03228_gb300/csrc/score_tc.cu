@@ -11,16 +11,16 @@
 //   2. main loop over 64-key tiles of the visible range: TMA brings the key
 //      rows (codes, or raw keys for the exact scores) into a ring of
 //      shared-memory stages; one thread issues tcgen05.mma (M = 128 queries,
-//      N = 64 keys, K = P, twice: u_hi and u_lo) into a ring of four TMEM
-//      accumulators;
+//      N = 64 keys, K = P, twice: u_hi and u_lo) into a ring of TMEM
+//      accumulators (eight of 64 columns, four of 128 at rank 128);
 //   3. four epilogue warps own one query row per thread (TMEM lane = row) and
 //      select in two passes over the same scores (the key tiles are multiplied
 //      twice; the tensor core has ample headroom): pass 1 folds every score
 //      into the row's 128 key-group maxima (one three-input maximum per two
-//      scores) and derives a certified lower bound tau on the row's k-th best
-//      score; pass 2 appends the visible keys scoring >= tau to the row's
-//      candidate column in shared memory.  The T x N score matrix is never
-//      stored.
+//      scores) and takes their k-th largest, a certified lower bound tau on
+//      the row's k-th best score; pass 2 appends the visible keys scoring
+//      >= tau to the row's candidate column in shared memory.  The T x N score
+//      matrix is never stored.
 //   4. exact top-k of the remaining candidates per row, written coalesced.
 // Roles: warp 0 = TMA producer, warp 1 = TMEM owner + MMA issuer, warps 2-5 =
 // epilogue.  Every mbarrier wait is bounded (tc.cuh); a timed-out CTA drains its
@@ -48,8 +48,12 @@ struct TcCfg {
   // unrolled selection loops (fewer inlined overflow-cut copies) and halve the
   // stage buffers, so that rank-128 columns get 144 slots
   static constexpr int NT = 64;
-  static constexpr int NB = 4;                                // TMEM accumulator ring (lets the warps drift)
-  static constexpr int BUFC = 128;                            // TMEM columns per ring buffer (a tile or a projection)
+  // TMEM accumulator ring: the four epilogue warps release a buffer together,
+  // so its depth is how far they may drift apart (their cut and bound phases
+  // take data-dependent time); eight 64-column buffers where a projection
+  // (P columns) fits one, four of 128 columns at rank 128
+  static constexpr int NB = P == 128 ? 4 : 8;
+  static constexpr int BUFC = P == 128 ? 128 : 64;           // TMEM columns per ring buffer (a tile or a projection)
   // ranks up to 64 store 32-bit key indices at a fixed distance from the
   // scores (one slot pointer serves both stores of an append); rank 128 needs
   // the room for its operands and keeps 16-bit indices in their own array
@@ -460,40 +464,74 @@ __device__ __forceinline__ void fold64(const uint32_t (&ra)[32], const uint32_t 
 }
 
 // The certified bound of pass 1.  The 128 group maxima are scores of distinct
-// visible keys, so any value tau with at least k of them >= tau bounds the row's
-// k-th best score from below.  32 of them, sorted, give pivots; one counting
-// pass tries the three around the expected rank of the k-th and keeps the
-// highest that qualifies (lower pivots on the rare rows where none does, -inf
-// as the last resort: every visible key is then a candidate).
-__device__ __forceinline__ float select_tau(const float (&g)[kGroups], int k) {
+// visible keys, so the k-th largest of them bounds the row's k-th best score
+// from below.  32 of them, sorted, give pivots: a counting pass tests three,
+// two samples apart, around the expected rank of the k-th and moves up or down
+// until one pivot leaves at least k maxima (lo) and a higher one fewer (hi).
+// The maxima between the two (at most 32) are gathered in the row's scratch
+// and ranked, which gives the k-th largest exactly; a wider bracket keeps lo,
+// and no qualifying pivot at all leaves -inf (every visible key is then a
+// candidate).  The maxima are first copied into the row's candidate column,
+// still empty, so that the counting and gathering loops run over shared memory
+// without unrolling: this code runs once per item and stays small.
+__device__ __forceinline__ float select_tau(const float (&g)[kGroups], int k, float* col, float* scr) {
   float s[32];
 #pragma unroll
   for (int u = 0; u < 32; ++u) s[u] = g[4 * u + 1];
   sort_desc<32>(s);
+#pragma unroll
+  for (int i = 0; i < kGroups; ++i) col[i * kLdc] = g[i];
   // sample q (0-based, descending) has about (q + 1) * 128 / 33 maxima at or above it
   int q = (33 * k + 127) / kGroups - 1;
-  q = q < 1 ? 1 : (q > 30 ? 30 : q);
-  float tau = -INFINITY;
+  q = q < 2 ? 2 : (q > 29 ? 29 : q);
+  float lo = -INFINITY, hi = INFINITY;
+  int nlo = kGroups, nhi = 0;
   bool pending = true;
   for (int attempt = 0; attempt < 4; ++attempt) {
-    const float p0 = pick<32>(s, q - 1), p1 = pick<32>(s, q), p2 = pick<32>(s, q + 1);
+    const float p0 = pick<32>(s, q - 2), p1 = pick<32>(s, q), p2 = pick<32>(s, q + 2);
     int n0 = 0, n1 = 0, n2 = 0;
-#pragma unroll
+#pragma unroll 4
     for (int i = 0; i < kGroups; ++i) {
-      n0 += g[i] >= p0 ? 1 : 0;
-      n1 += g[i] >= p1 ? 1 : 0;
-      n2 += g[i] >= p2 ? 1 : 0;
+      const float v = col[i * kLdc];
+      n0 += v >= p0 ? 1 : 0;
+      n1 += v >= p1 ? 1 : 0;
+      n2 += v >= p2 ? 1 : 0;
     }
     if (pending) {
-      if (n0 >= k) tau = p0;
-      else if (n1 >= k) tau = p1;
-      else if (n2 >= k) tau = p2;
-      pending = !(n2 >= k);
+      // descending pivots, ascending counts: the highest qualifying one and
+      // the lowest failing one narrow the bracket
+      if (n2 >= k && p2 > lo) { lo = p2; nlo = n2; }
+      if (n1 >= k && p1 > lo) { lo = p1; nlo = n1; }
+      if (n0 >= k && p0 > lo) { lo = p0; nlo = n0; }
+      if (n0 < k && p0 < hi) { hi = p0; nhi = n0; }
+      if (n1 < k && p1 < hi) { hi = p1; nhi = n1; }
+      if (n2 < k && p2 < hi) { hi = p2; nhi = n2; }
+      const bool up = hi == INFINITY && q > 2;      // every pivot qualified
+      const bool down = lo == -INFINITY && q < 29;  // none did
+      pending = up || down;
+      q = up ? (q < 8 ? 2 : q - 6) : (down ? (q > 23 ? 29 : q + 6) : q);
     }
     if (!__any_sync(0xffffffffu, pending)) break;
-    q = q + 3 > 30 ? 30 : q + 3;
   }
-  return tau;
+  // the (k - nhi)-th largest of the nlo - nhi maxima in [lo, hi)
+  const bool ex = nlo - nhi <= 32;
+  if (__any_sync(0xffffffffu, ex)) {
+    int c = 0;
+#pragma unroll 4
+    for (int i = 0; i < kGroups; ++i) {
+      const float v = col[i * kLdc];
+      const bool in = ex && v >= lo && v < hi;
+      if (in) scr[c] = v;
+      c += in ? 1 : 0;
+    }
+    float b[32];
+#pragma unroll
+    for (int u = 0; u < 32; ++u) b[u] = u < c ? scr[u] : -INFINITY;
+    sort_desc<32>(b);
+    const float t = pick<32>(b, k - nhi - 1);
+    if (ex) lo = t;
+  }
+  return lo;
 }
 
 // Rare path of pass 2: lanes whose column is within one chunk of the capacity
@@ -837,7 +875,7 @@ __global__ void __launch_bounds__(192, 1)
       }
       if (!ok) break;
       int cnt = 0;
-      float thr = below(select_tau(g, a.k));
+      float thr = below(select_tau(g, a.k, col.bs + col.row, scr));
       // pass 2: candidates scoring >= tau
       for (int i = 0; i < ntiles; ++i) {
         const uint32_t buf = ac % C::NB;
