@@ -291,6 +291,25 @@ __device__ __forceinline__ void pivot_cut(const Col& c, int& cnt, float& thr, in
   if (ok) thr = fmaxf(thr, pc);
 }
 
+// Bitonic sort of 16 (score, index) keys into descending order.
+__device__ __forceinline__ void sort16_desc(uint64_t (&key)[16]) {
+#pragma unroll
+  for (int size = 2; size <= 16; size <<= 1)
+#pragma unroll
+    for (int jj = size >> 1; jj > 0; jj >>= 1)
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int l = i ^ jj;
+        if (l > i) {
+          const uint64_t x = key[i], y = key[l];
+          const bool desc = (i & size) == 0;
+          const bool sw = desc ? (x < y) : (x > y);
+          key[i] = sw ? y : x;
+          key[l] = sw ? x : y;
+        }
+      }
+}
+
 // Exact cut of the lanes with `on` to their k best entries (slots [0, k)); thr
 // rises to a lower bound of the k-th best score (a later key, with a higher
 // index, must score above it to matter).  Quickselect by counting over a
@@ -398,21 +417,7 @@ __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int
 #pragma unroll
     for (int u = 0; u < 16; ++u)
       key[u] = (fin && u < nbd) ? make_key(scr[2 * u], (uint32_t)__float_as_int(scr[2 * u + 1])) : 0ull;
-#pragma unroll
-    for (int size = 2; size <= 16; size <<= 1)
-#pragma unroll
-      for (int jj = size >> 1; jj > 0; jj >>= 1)
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int l = i ^ jj;
-          if (l > i) {
-            const uint64_t x = key[i], y = key[l];
-            const bool desc = (i & size) == 0;
-            const bool sw = desc ? (x < y) : (x > y);
-            key[i] = sw ? y : x;
-            key[l] = sw ? x : y;
-          }
-        }
+    sort16_desc(key);
     float kth = hi;
 #pragma unroll
     for (int u = 0; u < 16; ++u) {
@@ -431,6 +436,113 @@ __device__ __forceinline__ void cut_to_k(const Col& c, int& cnt, float& thr, int
       pivot_cut(c, cnt, thr, k, k + 3, cnt - 1, pending && cnt - k > 8);
     while (__any_sync(0xffffffffu, pending && cnt > k)) remove_worst(c, cnt, warp_max(cnt), thr, pending && cnt > k);
   }
+}
+
+// Bin of score v among 64 equal bins over [lo, lo + 64 / scale]: the integer
+// nearest (v - lo) * scale, read from the bits of a float near 2^23 (one FMA;
+// bias = 2^23 - lo * scale), clamped to [0, 63].  Non-decreasing in v.
+__device__ __forceinline__ int bin64(float v, float scale, float bias) {
+  const int b = __float_as_int(fmaf(v, scale, bias)) - 0x4B000000;
+  return b < 0 ? 0 : (b > 63 ? 63 : b);
+}
+
+// Final exact cut of the lanes with `on` to their k best entries (slots
+// [0, k)), by histogram: 64 bins over the column's score range, counted with
+// shared-memory atomics into 16-bit halves of the row's scratch, locate the bin
+// holding the k-th best entry; entries in higher bins are kept, and those of
+// that bin (at most 16) are ranked as 64-bit (score, index) keys.  Lanes this
+// cannot settle (a degenerate range, or more than 16 entries in the boundary
+// bin, e.g. many equal scores) go through cut_to_k.
+template <class Col>
+__device__ __forceinline__ void cut_hist(const Col& c, int& cnt, float& thr, int k, float* scr, bool on) {
+  bool pending = on && cnt > k;
+  if (!__any_sync(0xffffffffu, pending)) return;
+  const int cmax = warp_max(cnt);
+  const float kNaN = __int_as_float(0x7fffffff);   // ignored by fminf / fmaxf
+  float lo = INFINITY, hi = -INFINITY;
+  for (int i = 0; i < cmax; i += 8) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const float v = i + u < cnt ? c.s(i + u) : kNaN;
+      lo = fminf(lo, v);
+      hi = fmaxf(hi, v);
+    }
+  }
+  const float scale = 64.f / (hi - lo);
+  const float bias = 8388608.f - lo * scale;
+  const bool ok = pending && hi > lo && scale <= 1e30f && fabsf(bias) <= 1e30f;
+  int* h = reinterpret_cast<int*>(scr);
+#pragma unroll
+  for (int w = 0; w < 32; ++w) h[w] = 0;
+  for (int i = 0; i < cmax; i += 8) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const float v = c.s(i + u);
+      const int b = bin64(v, scale, bias);
+      if (ok && i + u < cnt) atomicAdd(h + (b >> 1), 1 << ((b & 1) << 4));
+    }
+  }
+  // the boundary bin: counting down from the top bin, the first that reaches k
+  int bstar = -1, na = 0, nb = 0, acc = 0;
+#pragma unroll
+  for (int w = 31; w >= 0; --w) {
+    const int hw = h[w];
+#pragma unroll
+    for (int half = 1; half >= 0; --half) {
+      const int n = half ? (hw >> 16) : (hw & 0xffff);
+      const bool hit = bstar < 0 && acc + n >= k;
+      bstar = hit ? 2 * w + half : bstar;
+      na = hit ? acc : na;
+      nb = hit ? n : nb;
+      acc += n;
+    }
+  }
+  const bool fin = ok && bstar >= 0 && nb <= 16;
+  if (__any_sync(0xffffffffu, fin)) {
+    // entries above the boundary bin compacted in place, its entries to the scratch
+    int w = 0, nbd = 0;
+    for (int i = 0; i < cmax; i += 8) {
+      float v[8];
+      int j[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        v[u] = c.s(i + u);
+        j[u] = c.j(i + u);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int b = bin64(v[u], scale, bias);
+        const bool in = fin && i + u < cnt;
+        const bool sure = in && b > bstar;
+        const bool bnd = in && b == bstar;
+        if (sure) c.put(w, v[u], j[u]);
+        if (bnd) {
+          scr[2 * nbd] = v[u];
+          scr[2 * nbd + 1] = __int_as_float(j[u]);
+        }
+        w += sure ? 1 : 0;
+        nbd += bnd ? 1 : 0;
+      }
+    }
+    uint64_t key[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u)
+      key[u] = (fin && u < nbd) ? make_key(scr[2 * u], (uint32_t)__float_as_int(scr[2 * u + 1])) : 0ull;
+    sort16_desc(key);
+    float kth = thr;
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      const bool use = fin && w + u < k && u < nbd;
+      if (use) c.put(w + u, key_score(key[u]), key_index(key[u]));
+      if (use) kth = key_score(key[u]);
+    }
+    if (fin) {
+      cnt = k;
+      thr = fmaxf(thr, kth);
+      pending = false;
+    }
+  }
+  if (__any_sync(0xffffffffu, pending)) cut_to_k(c, cnt, thr, k, scr, pending);
 }
 
 // Three-input maximum (one instruction on sm_100 and later).
@@ -910,7 +1022,7 @@ __global__ void __launch_bounds__(192, 1)
         tc::fence_proxy_async_smem();
         tc::mbar_arrive(aready);
       }
-      cut_to_k(col, cnt, thr, a.k, scr, true);
+      cut_hist(col, cnt, thr, a.k, scr, true);
       if (!a.sorted && (a.k & 3) == 0) {
         // unsorted lists: each thread writes its own row, four entries per store
         if (m < t.nrows) {
