@@ -48,12 +48,13 @@ struct TcCfg {
   // unrolled selection loops (fewer inlined overflow-cut copies) and halve the
   // stage buffers, so that rank-128 columns get 144 slots
   static constexpr int NT = 64;
-  // TMEM accumulator ring: the four epilogue warps release a buffer together,
-  // so its depth is how far they may drift apart (their cut and bound phases
-  // take data-dependent time); eight 64-column buffers where a projection
-  // (P columns) fits one, four of 128 columns at rank 128
-  static constexpr int NB = P == 128 ? 4 : 8;
-  static constexpr int BUFC = P == 128 ? 128 : 64;           // TMEM columns per ring buffer (a tile or a projection)
+  // TMEM accumulator ring of eight 64-column buffers: the four epilogue warps
+  // release a buffer together, so its depth is how far they may drift apart
+  // (their cut and bound phases take data-dependent time).  A tile takes one
+  // buffer, a projection of P columns PB consecutive ones (two at rank 128).
+  static constexpr int NB = 8;
+  static constexpr int BUFC = 64;                             // TMEM columns per ring buffer
+  static constexpr int PB = (P + BUFC - 1) / BUFC;
   // ranks up to 64 store 32-bit key indices at a fixed distance from the
   // scores (one slot pointer serves both stores of an append); rank 128 needs
   // the room for its operands and keeps 16-bit indices in their own array
@@ -85,7 +86,8 @@ struct TcCfg {
   static_assert(STAGE_BYTES >= P * 128, "a projection chunk must fit a stage");
   static_assert(CAP % 8 == 0 && CAP >= 64 + 32, "candidate capacity: k + one chunk of appends");
   static_assert(NT == 64, "pass 1 folds a tile's two 32-key halves into one block of 32 groups");
-  static_assert(NT <= BUFC && P <= BUFC && TMEM_COLS <= 512, "a ring buffer holds a tile's or a projection's columns");
+  static_assert(NT <= BUFC && P <= PB * BUFC && P % PB == 0 && TMEM_COLS <= 512,
+                "a ring buffer holds a tile's columns, PB of them a projection's");
   static_assert(SMEM <= 232448, "shared memory budget");
   static_assert(OFF_STAGE % 1024 == 0 && STAGE_BYTES % 1024 == 0, "swizzled TMA tiles sit on 1024-byte boundaries");
   static_assert(OFF_SCR % 16 == 0 && OFF_BAR % 16 == 0, "16-byte scratch stores and 8-byte mbarriers stay aligned");
@@ -731,12 +733,12 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo_elem, float hi_elem) {
 // Epilogue: read the projection (P fp32 columns of this row), split u = hi + lo
 // into the two bf16 A-operand matrices.
 template <int P>
-__device__ __forceinline__ void convert_projection(uint32_t taddr, uint8_t* sA, int m) {
+__device__ __forceinline__ void convert_projection(const uint32_t (&taddr)[2], uint8_t* sA, int m) {
 #pragma unroll
   for (int c0 = 0; c0 < P; c0 += 16) {
     uint32_t r[16];
     __syncwarp();
-    tc::tmem_ld16(taddr + c0, r);
+    tc::tmem_ld16(c0 < 64 ? taddr[0] + c0 : taddr[1] + (c0 - 64), r);
     tc::tmem_ld_wait();
 #pragma unroll
     for (int h8 = 0; h8 < 2; ++h8) {
@@ -869,16 +871,19 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       uint32_t sc = 0, ac = 0;
       int it = 0;
-      constexpr uint32_t idP = tc::idesc_bf16(128, P);
+      constexpr uint32_t idP = tc::idesc_bf16(128, P / C::PB);
       constexpr uint32_t idN = tc::idesc_bf16(128, C::NT);
       const uint32_t aBase = tc::smem_u32(sA), sBase = tc::smem_u32(sStage);
       for (int item = blockIdx.x; item < a.n_items; item += gridDim.x, ++it) {
         const TcTile t = a.tiles[item / Hq];
         if (!tc::mbar_wait(qfull, it & 1, abort_f)) break;
-        uint32_t buf = ac % C::NB;
-        if (!tc::mbar_wait(acce + buf, ((ac / C::NB) & 1) ^ 1, abort_f)) break;
-        tc::fence_after_sync();
         bool ok = true;
+#pragma unroll
+        for (int q = 0; q < C::PB; ++q)
+          ok = ok && tc::mbar_wait(acce + (ac + q) % C::NB, (((ac + q) / C::NB) & 1) ^ 1, abort_f);
+        if (!ok) break;
+        tc::fence_after_sync();
+        uint32_t buf;
         uint32_t acc = 0;
         for (int s3 = 0; s3 < 3 && ok; ++s3)
           for (int kh = 0; kh < 2; ++kh) {
@@ -887,16 +892,21 @@ __global__ void __launch_bounds__(192, 1)
             tc::fence_after_sync();
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
-              tc::mma_bf16(tmem + buf * C::BUFC, tc::sdesc(aBase + kh * 16384 + kk * 32, 1024, 2),
-                           tc::sdesc(sBase + st * C::STAGE_BYTES + kk * 32, 1024, 2), idP, acc);
+              // the projection's columns p * P / PB .. of W in rows of the stage
+#pragma unroll
+              for (int q = 0; q < C::PB; ++q)
+                tc::mma_bf16(tmem + ((ac + q) % C::NB) * C::BUFC, tc::sdesc(aBase + kh * 16384 + kk * 32, 1024, 2),
+                             tc::sdesc(sBase + st * C::STAGE_BYTES + q * (P / C::PB) * 128 + kk * 32, 1024, 2), idP,
+                             acc);
               acc = 1;
             }
             tc::mma_commit(empty + st);
             ++sc;
           }
         if (!ok) break;
-        tc::mma_commit(accf + buf);
-        ++ac;
+#pragma unroll
+        for (int q = 0; q < C::PB; ++q) tc::mma_commit(accf + (ac + q) % C::NB);
+        ac += C::PB;
         if (!tc::mbar_wait(aready, it & 1, abort_f)) break;
         tc::fence_after_sync();
         const int ntiles = (t.vis_max + C::NT - 1) / C::NT;
@@ -945,14 +955,19 @@ __global__ void __launch_bounds__(192, 1)
       const TcTile t = a.tiles[item / Hq];
       const int h = item % Hq;
       if (it == 0) {  // this item's projection (later items convert theirs ahead of time)
-        const uint32_t buf = ac % C::NB;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
+        uint32_t pa[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) pa[q] = tl + ((ac + (q < C::PB ? q : 0)) % C::NB) * C::BUFC;
+#pragma unroll
+        for (int q = 0; q < C::PB; ++q)
+          ok = ok && __all_sync(0xffffffffu, tc::mbar_wait(accf + (ac + q) % C::NB, ((ac + q) / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
-        convert_projection<P>(tl + buf * C::BUFC, sA, m);
+        convert_projection<P>(pa, sA, m);
         tc::fence_before_sync();
-        tc::mbar_arrive(acce + buf);
-        ++ac;
+#pragma unroll
+        for (int q = 0; q < C::PB; ++q) tc::mbar_arrive(acce + (ac + q) % C::NB);
+        ac += C::PB;
         tc::fence_proxy_async_smem();
         tc::mbar_arrive(aready);
       }
@@ -1011,14 +1026,19 @@ __global__ void __launch_bounds__(192, 1)
       // convert the next item's projection now, so the tensor core can move on
       const int nxt = item + gridDim.x;
       if (nxt < a.n_items) {
-        const uint32_t buf = ac % C::NB;
-        ok = __all_sync(0xffffffffu, tc::mbar_wait(accf + buf, (ac / C::NB) & 1, abort_f));
+        uint32_t pa[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) pa[q] = tl + ((ac + (q < C::PB ? q : 0)) % C::NB) * C::BUFC;
+#pragma unroll
+        for (int q = 0; q < C::PB; ++q)
+          ok = ok && __all_sync(0xffffffffu, tc::mbar_wait(accf + (ac + q) % C::NB, ((ac + q) / C::NB) & 1, abort_f));
         if (!ok) break;
         tc::fence_after_sync();
-        convert_projection<P>(tl + buf * C::BUFC, sA, m);
+        convert_projection<P>(pa, sA, m);
         tc::fence_before_sync();
-        tc::mbar_arrive(acce + buf);
-        ++ac;
+#pragma unroll
+        for (int q = 0; q < C::PB; ++q) tc::mbar_arrive(acce + (ac + q) % C::NB);
+        ac += C::PB;
         tc::fence_proxy_async_smem();
         tc::mbar_arrive(aready);
       }
