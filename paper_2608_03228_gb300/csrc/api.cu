@@ -1007,11 +1007,13 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
   int32_t* ie = idx_exact ? idx_exact
                           : reinterpret_cast<int32_t*>(ws + base + align_up((size_t)cfg->num_q_heads * 2 *
                                                                             sizeof(unsigned long long)));
+  int64_t vmax = 0;   // the longest visible prefix: sizes the recall kernel's bitmap
+  for (int64_t t = 0; t < T; ++t) vmax = layout->q_visible[t] > vmax ? layout->q_visible[t] : vmax;
   if (tc) {
     if ((st = run_tc(cfg, layout, tp, kD, true, Q, A, K, nullptr, ie, nullptr, ws, s)) != SAKI_OK) return st;
     return finish(cfg,
                   cuda_status(launch_recall(idx_approx, ie, reinterpret_cast<const int32_t*>(ws + tp.off_vis), T,
-                                            cfg->num_q_heads, cfg->topk, min_visible, counters, recall, s)),
+                                            cfg->num_q_heads, cfg->topk, min_visible, vmax, counters, recall, s)),
                   ws, s);
   }
   if (T == 0 && (st = cuda_status(cudaMemsetAsync(ws, 0, sizeof(int), s))) != SAKI_OK) return st;
@@ -1037,8 +1039,8 @@ saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64
   }
   const int32_t* vis = reinterpret_cast<const int32_t*>(ws + p.off_vis);
   return finish(cfg,
-                cuda_status(launch_recall(idx_approx, ie, vis, T, cfg->num_q_heads, cfg->topk, min_visible, counters,
-                                          recall, s)),
+                cuda_status(launch_recall(idx_approx, ie, vis, T, cfg->num_q_heads, cfg->topk, min_visible, vmax,
+                                          counters, recall, s)),
                 ws, s);
 }
 

@@ -122,8 +122,9 @@ cudaError_t launch_build_generic(const void* K, const float* R, const float* mu,
                                  cudaStream_t s);
 
 // recall counters [Hq][2] (matches, rows) and final per-head recall
+// max_visible: the largest visible count of any query (sizes the bitmap path)
 cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int32_t* vis,
-                          int64_t T, int Hq, int k, int64_t min_visible,
+                          int64_t T, int Hq, int k, int64_t min_visible, int64_t max_visible,
                           unsigned long long* counters, float* recall, cudaStream_t s);
 
 // ---------------------------------------------------------------- tensor-core path

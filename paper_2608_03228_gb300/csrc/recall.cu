@@ -1,10 +1,13 @@
 // Recall of the Sec. 3 protocol: per (head, query) with at least min_visible
 // visible keys, |approx set & exact set| / k, averaged per head.  A warp walks a
-// contiguous range of (head, query) rows; per row it inserts the approximate
-// indices into a small open-addressing table in shared memory, probes it with
-// the exact ones and clears only the slots it used.  Integer counts per head
-// are flushed with atomics when the head changes, so the per-head value is
-// exact and order-free.
+// contiguous range of (head, query) rows, loading the next row's two index
+// lists while it matches the current one.  Where every row sees at most
+// kBitmapKeys keys, the warp marks the approximate indices in a bitmap of the
+// row's key range in shared memory (one atomic OR per index), tests the exact
+// ones against it and clears the words it set; otherwise it inserts them into
+// a small open-addressing table.  Integer counts per head are flushed with
+// atomics when the head changes, so the per-head value is exact and
+// order-free.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -12,8 +15,88 @@ namespace saki {
 namespace {
 constexpr int kSlots = 256;       // >= 2 k for k <= 128
 constexpr int kPerLane = 4;       // k <= 128 indices per list: at most 4 per lane
+constexpr int64_t kBitmapKeys = 24576;   // bitmap path: 8 warps x 3 KB of shared memory per block
 
 __device__ __forceinline__ uint32_t slot_of(int32_t v) { return ((uint32_t)v * 2654435761u) >> 24; }
+
+// Bitmap matching: words = bitmap words per warp (dynamic shared memory, 8 warps).
+__global__ void __launch_bounds__(256) recall_bitmap_kernel(const int32_t* ia, const int32_t* ie, const int32_t* vis,
+                                                            int64_t T, int Hq, int k, int64_t min_visible, int words,
+                                                            unsigned long long* counters) {
+  extern __shared__ uint32_t bm_all[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t* bm = bm_all + warp * words;
+  for (int o = lane; o < words; o += 32) bm[o] = 0u;
+  __syncwarp();
+  const int64_t total = (int64_t)Hq * T;
+  const int64_t nwarps = (int64_t)gridDim.x * 8;
+  const int64_t per = (total + nwarps - 1) / nwarps;
+  const int64_t r0 = ((int64_t)blockIdx.x * 8 + warp) * per;
+  const int64_t r1 = r0 + per < total ? r0 + per : total;
+  const int64_t nbits = (int64_t)words * 32;
+  int cur_h = -1;
+  unsigned long long matches = 0, rows = 0;
+  int32_t na[kPerLane], ne[kPerLane];
+  int64_t nt = r0 % T;
+  int nh = (int)(r0 / T);
+  int32_t nvis = r0 < r1 ? __ldg(vis + nt) : 0;
+  auto load_row = [&](int64_t r, int32_t (&va)[kPerLane], int32_t (&ve)[kPerLane]) {
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      const int i = lane + 32 * u;
+      const bool in = r < r1 && i < k;
+      va[u] = in ? __ldg(ia + r * k + i) : -1;
+      ve[u] = in ? __ldg(ie + r * k + i) : -1;
+    }
+  };
+  load_row(r0, na, ne);
+  for (int64_t r = r0; r < r1; ++r) {
+    int32_t av[kPerLane], ev[kPerLane];
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      av[u] = na[u];
+      ev[u] = ne[u];
+    }
+    const int h = nh;
+    const int32_t row_vis = nvis;
+    if (++nt == T) {
+      nt = 0;
+      ++nh;
+    }
+    nvis = r + 1 < r1 ? __ldg(vis + nt) : 0;
+    load_row(r + 1, na, ne);
+    if (h != cur_h) {
+      if (lane == 0 && rows) {
+        atomicAdd(counters + 2 * cur_h, matches);
+        atomicAdd(counters + 2 * cur_h + 1, rows);
+      }
+      cur_h = h;
+      matches = rows = 0;
+    }
+    if (row_vis < min_visible) continue;   // warp-uniform
+    // indices outside the bitmap (none from the selection calls) match nothing
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u)
+      if (av[u] >= 0 && av[u] < nbits) atomicOr(bm + (av[u] >> 5), 1u << (av[u] & 31));
+    __syncwarp();
+    int m = 0;
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u)
+      if (ev[u] >= 0 && ev[u] < nbits) m += (bm[ev[u] >> 5] >> (ev[u] & 31)) & 1u;
+    m = __reduce_add_sync(0xffffffffu, m);
+    matches += (unsigned long long)m;
+    rows += 1;
+    __syncwarp();
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u)
+      if (av[u] >= 0 && av[u] < nbits) bm[av[u] >> 5] = 0u;
+    __syncwarp();
+  }
+  if (lane == 0 && rows) {
+    atomicAdd(counters + 2 * cur_h, matches);
+    atomicAdd(counters + 2 * cur_h + 1, rows);
+  }
+}
 
 __global__ void __launch_bounds__(256) recall_kernel(const int32_t* ia, const int32_t* ie, const int32_t* vis,
                                                      int64_t T, int Hq, int k, int64_t min_visible,
@@ -120,7 +203,8 @@ __global__ void recall_finish_kernel(const unsigned long long* counters, int Hq,
 }  // namespace
 
 cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int32_t* vis, int64_t T, int Hq, int k,
-                          int64_t min_visible, unsigned long long* counters, float* recall, cudaStream_t s) {
+                          int64_t min_visible, int64_t max_visible, unsigned long long* counters, float* recall,
+                          cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(counters, 0, sizeof(unsigned long long) * 2 * Hq, s);
   if (e != cudaSuccess) return e;
   if (T > 0) {
@@ -130,7 +214,13 @@ cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int3
     const int64_t want = (rows + 7) / 8;   // at least one row per warp
     const int64_t blocks = want < (int64_t)sms * 4 ? want : (int64_t)sms * 4;
     note_launch();
-    recall_kernel<<<(unsigned)blocks, 256, 0, s>>>(idx_a, idx_e, vis, T, Hq, k, min_visible, counters);
+    if (max_visible <= kBitmapKeys) {
+      const int words = (int)((max_visible + 31) / 32) < 1 ? 1 : (int)((max_visible + 31) / 32);
+      recall_bitmap_kernel<<<(unsigned)blocks, 256, (size_t)8 * words * sizeof(uint32_t), s>>>(
+          idx_a, idx_e, vis, T, Hq, k, min_visible, words, counters);
+    } else {
+      recall_kernel<<<(unsigned)blocks, 256, 0, s>>>(idx_a, idx_e, vis, T, Hq, k, min_visible, counters);
+    }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   note_launch();

@@ -364,13 +364,15 @@ def test_score_topk_seeded_decode_ties(lib):
             np.testing.assert_array_equal(idx[h, t], ref, err_msg=f"h{h} t{t}")
 
 
-def test_recall_seeded_decode(lib):
+@pytest.mark.parametrize("n", [24000, 30000])
+def test_recall_seeded_decode(lib, n):
     """Exact top-k through saki_recall on a seeded decode layout (keys as the
-    tensor-core operand, four query heads per KV head) and the head recall."""
+    tensor-core operand, four query heads per KV head) and the head recall
+    (24,000 keys: the bitmap match; 30,000: the hash-table match)."""
     torch = _torch()
     Hq, Hk, r, k = 4, 1, 32, 64
     rng = np.random.default_rng(23)
-    off, q_seq, q_vis = _layout_arrays((24000,), ([-1, -1, 20000, 3000, 65, 64],))
+    off, q_seq, q_vis = _layout_arrays((n,), ([-1, -1, 20000, 3000, 65, 64],))
     T, N = len(q_seq), int(off[-1])
     Q = synth.round_to_bf16_grid(rng.standard_normal((Hq, T, D)).astype(np.float32))
     K = synth.round_to_bf16_grid(rng.standard_normal((Hk, N, D)).astype(np.float32))
