@@ -369,11 +369,11 @@ def run_e2e(g, args, torch):
 # the heads, as the pairs do, so bench.py scales these to the workload; a kernel
 # changed after its capture is left out (traffic null).
 TRAFFIC_BYTES_PER_PAIR = {
-    "select": (542111744 + 225285632) / 2148007936,
-    "exact": (889242624 + 236534016) / 2148007936,
-    "moments": (335588864 + 3024640) / 2148007936,
-    "build": (73442048 + 13277184) / 2148007936,
-    "fit": (58813440 + 44288) / 2148007936,
+    "select": (571738368 + 225124608) / 2148007936,
+    "exact": (976233984 + 235627008) / 2148007936,
+    "moments": (335573504 + 3031040) / 2148007936,
+    "build": (73458176 + 13318656) / 2148007936,
+    "fit": (58777344 + 43264) / 2148007936,
 }
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only
 
