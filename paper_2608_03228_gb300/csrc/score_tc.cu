@@ -108,13 +108,18 @@ struct TcCfg {
 
 // A row's candidate column: slot i holds a score (fp32) and its key index.
 // ColSplit keeps 16-bit indices in their own array (the host only sends
-// sequences of at most 65535 keys here); ColWide keeps 32-bit indices IOFF
-// words after their scores, so one slot pointer addresses both.
+// sequences of at most 65535 keys here); ColPair keeps (score, 32-bit index)
+// pairs of 8 bytes, so an append is a single 64-bit store (shared-memory store
+// instructions, predicated or not, are what the append loop is bound by: two
+// 32-bit stores per key took twice as long in a stand-alone loop).  kSStride
+// is the distance, in floats, between a row's consecutive scores.
 struct ColSplit {
   static constexpr bool kWide = false;
+  static constexpr int kSStride = kLdc;
   float* bs;
   uint16_t* bi;
   int row;
+  __device__ __forceinline__ float* sbase() const { return bs + row; }
   __device__ __forceinline__ float s(int i) const { return bs[i * kLdc + row]; }
   __device__ __forceinline__ int j(int i) const { return bi[i * kLdc + row]; }
   __device__ __forceinline__ void put(int i, float v, int k) const {
@@ -123,23 +128,22 @@ struct ColSplit {
   }
   __device__ __forceinline__ ColSplit at(int r) const { return ColSplit{bs, bi, r}; }
 };
-template <int IOFF>
-struct ColWide {
+struct ColPair {
   static constexpr bool kWide = true;
-  static constexpr int kIOff = IOFF;
-  float* bs;
+  static constexpr int kSStride = 2 * kLdc;
+  float2* b;
   int row;
-  __device__ __forceinline__ float s(int i) const { return bs[i * kLdc + row]; }
-  __device__ __forceinline__ int j(int i) const { return __float_as_int(bs[IOFF + i * kLdc + row]); }
+  __device__ __forceinline__ float* sbase() const { return reinterpret_cast<float*>(b + row); }
+  __device__ __forceinline__ float s(int i) const { return b[i * kLdc + row].x; }
+  __device__ __forceinline__ int j(int i) const { return __float_as_int(b[i * kLdc + row].y); }
   __device__ __forceinline__ void put(int i, float v, int k) const {
-    bs[i * kLdc + row] = v;
-    bs[IOFF + i * kLdc + row] = __int_as_float(k);
+    b[i * kLdc + row] = make_float2(v, __int_as_float(k));
   }
-  __device__ __forceinline__ ColWide at(int r) const { return ColWide{bs, r}; }
+  __device__ __forceinline__ ColPair at(int r) const { return ColPair{b, r}; }
 };
 template <class Col>
 __device__ __forceinline__ Col make_col(float* bs, uint16_t* bi, int row) {
-  if constexpr (Col::kWide) return Col{bs, row};
+  if constexpr (Col::kWide) return Col{reinterpret_cast<float2*>(bs), row};
   else return Col{bs, bi, row};
 }
 
@@ -588,13 +592,14 @@ __device__ __forceinline__ void fold64(const uint32_t (&ra)[32], const uint32_t 
 // candidate).  The maxima are first copied into the row's candidate column,
 // still empty, so that the counting and gathering loops run over shared memory
 // without unrolling: this code runs once per item and stays small.
+template <int S>
 __device__ __forceinline__ float select_tau(const float (&g)[kGroups], int k, float* col, float* scr) {
   float s[32];
 #pragma unroll
   for (int u = 0; u < 32; ++u) s[u] = g[4 * u + 1];
   sort_desc<32>(s);
 #pragma unroll
-  for (int i = 0; i < kGroups; ++i) col[i * kLdc] = g[i];
+  for (int i = 0; i < kGroups; ++i) col[i * S] = g[i];
   // sample q (0-based, descending) has about (q + 1) * 128 / 33 maxima at or above it
   int q = (33 * k + 127) / kGroups - 1;
   q = q < 2 ? 2 : (q > 29 ? 29 : q);
@@ -606,7 +611,7 @@ __device__ __forceinline__ float select_tau(const float (&g)[kGroups], int k, fl
     int n0 = 0, n1 = 0, n2 = 0;
 #pragma unroll 4
     for (int i = 0; i < kGroups; ++i) {
-      const float v = col[i * kLdc];
+      const float v = col[i * S];
       n0 += v >= p0 ? 1 : 0;
       n1 += v >= p1 ? 1 : 0;
       n2 += v >= p2 ? 1 : 0;
@@ -633,7 +638,7 @@ __device__ __forceinline__ float select_tau(const float (&g)[kGroups], int k, fl
     int c = 0;
 #pragma unroll 4
     for (int i = 0; i < kGroups; ++i) {
-      const float v = col[i * kLdc];
+      const float v = col[i * S];
       const bool in = ex && v >= lo && v < hi;
       if (in) scr[c] = v;
       c += in ? 1 : 0;
@@ -676,22 +681,20 @@ template <int CAP, class Col>
 __device__ __forceinline__ void append32(const uint32_t (&r)[32], int j0, float& thr, float* scr, const Col& c,
                                          int& cnt, int k) {
   if (__any_sync(0xffffffffu, cnt > CAP - 32)) make_room<CAP>(r, thr, scr, c, cnt, k);
-  float* ps = c.bs + cnt * kLdc + c.row;
   if constexpr (Col::kWide) {
-    // score and index through one slot pointer; the count is the pointer's advance
-    float* const p0 = ps;
+    // one 64-bit store per append; the count is the slot pointer's advance
+    float2* ps = c.b + cnt * kLdc + c.row;
+    float2* const p0 = ps;
 #pragma unroll
     for (int u = 0; u < 32; ++u) {
       const float v = __uint_as_float(r[u]);
       const bool t = v > thr;
-      if (t) {
-        ps[0] = v;
-        ps[Col::kIOff] = __int_as_float(j0 + u);
-      }
+      if (t) *ps = make_float2(v, __int_as_float(j0 + u));
       ps += t ? kLdc : 0;
     }
     cnt += (int)(ps - p0) / kLdc;
   } else {
+    float* ps = c.bs + cnt * kLdc + c.row;
     uint16_t* pi = c.bi + cnt * kLdc + c.row;
     int added = 0;
 #pragma unroll
@@ -945,7 +948,7 @@ __global__ void __launch_bounds__(192, 1)
     const int quarter = warp & 3;
     const int m = quarter * 32 + lane;
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
-    using Col = typename std::conditional<C::WIDE, ColWide<C::CAP * kLdc>, ColSplit>::type;
+    using Col = typename std::conditional<C::WIDE, ColPair, ColSplit>::type;
     const Col col = make_col<Col>(bs, bi, m);
     float* scr = scr_all + m * kScr;
     uint32_t ac = 0;
@@ -1002,7 +1005,7 @@ __global__ void __launch_bounds__(192, 1)
       }
       if (!ok) break;
       int cnt = 0;
-      float thr = below(select_tau(g, a.k, col.bs + col.row, scr));
+      float thr = below(select_tau<Col::kSStride>(g, a.k, col.sbase(), scr));
       // pass 2: candidates scoring >= tau
       for (int i = 0; i < ntiles; ++i) {
         const uint32_t buf = ac % C::NB;
