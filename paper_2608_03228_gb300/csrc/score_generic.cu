@@ -108,8 +108,11 @@ __global__ void __launch_bounds__(kThreads) score_generic_kernel(const ScoreArgs
   int* cnt_s = visq + kGroupQ;                                             // [warps][GQ]
   __shared__ unsigned long long cta_thr[kGroupQ];
 
-  const ScoreItem it = a.items[blockIdx.x];
-  const int h = blockIdx.y;
+  // one CTA per (item, query head), the heads of an item adjacent: the G
+  // heads of a KV group then stream the same key tiles together (the exact
+  // scores read a KV head's keys once from DRAM, the others hit L2)
+  const ScoreItem it = a.items[blockIdx.x / a.Hq];
+  const int h = (int)(blockIdx.x % a.Hq);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int P = a.P;
   const int nq = it.q_count;
@@ -407,8 +410,11 @@ __global__ void __launch_bounds__(192) score_decode_tc_kernel(const __grid_const
   uint64_t* drain = uready + 1;
   volatile int* abort_f = &abort_s;
 
-  const ScoreItem it = a.items[blockIdx.x];
-  const int h = blockIdx.y;
+  // one CTA per (item, query head), the heads of an item adjacent: the G
+  // heads of a KV group then stream the same key tiles together (the exact
+  // scores read a KV head's keys once from DRAM, the others hit L2)
+  const ScoreItem it = a.items[blockIdx.x / a.Hq];
+  const int h = (int)(blockIdx.x % a.Hq);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nq = it.q_count;
   const int nkeys = it.key_hi - it.key_lo;
@@ -694,7 +700,8 @@ cudaError_t launch_decode_tc_t(const ScoreArgs& a, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
   if (e != cudaSuccess) return e;
   note_launch();
-  kern<<<dim3(a.n_items, a.Hq), 192, sm, s>>>(mX, a);
+  if ((int64_t)a.n_items * a.Hq > 0x7fffffff) return cudaErrorInvalidConfiguration;
+  kern<<<(unsigned)(a.n_items * a.Hq), 192, sm, s>>>(mX, a);
   return cudaGetLastError();
 }
 
@@ -715,7 +722,8 @@ cudaError_t launch_score_t(const ScoreArgs& a, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
   if (e != cudaSuccess) return e;
   note_launch();
-  kern<<<dim3(a.n_items, a.Hq), kThreads, sm, s>>>(a);
+  if ((int64_t)a.n_items * a.Hq > 0x7fffffff) return cudaErrorInvalidConfiguration;
+  kern<<<(unsigned)(a.n_items * a.Hq), kThreads, sm, s>>>(a);
   return cudaGetLastError();
 }
 }  // namespace
