@@ -276,6 +276,33 @@ Plan make_plan(const saki_layout* L, int Hq, int kp, int dtype, int P, bool seed
   const int64_t target_per_head = std::max<int64_t>(1, (int64_t)8 * kNumSMs / Hq);
   int64_t chunk = std::max<int64_t>(2048, (work + target_per_head - 1) / target_per_head);
   chunk = (chunk + 255) / 256 * 256;
+  // split length between 70 % and 100 % of that (never longer: a group keeps at
+  // least the splits that make it seeded), chosen so the (item, head) CTAs
+  // fill their last wave best (CTAs resident per SM from the scoring kernel's
+  // occupancy; 1216 CTAs of three per SM left a last wave two-thirds full)
+  const int per_sm = score_ctas_per_sm(dtype, P, kp, p.nq);
+  int64_t base_items = 0;
+  for (const G& g : groups) base_items += g.vmax > 0 ? (g.vmax + chunk - 1) / chunk : 1;
+  // only where the waves are few: past four, a part-filled last wave costs
+  // little and the extra splits (more items, longer merges) cost more
+  if (per_sm > 0 && !groups.empty() && base_items * Hq <= (int64_t)4 * kNumSMs * per_sm) {
+    const int64_t slots = (int64_t)kNumSMs * per_sm;
+    double best_fill = -1.0;
+    int64_t best_c = chunk;
+    for (int i = -6; i <= 0; ++i) {
+      const int64_t c = std::min(chunk, (chunk * (20 + i) / 20 + 255) / 256 * 256);
+      if (c < 2048) continue;
+      int64_t items = 0;
+      for (const G& g : groups) items += g.vmax > 0 ? (g.vmax + c - 1) / c : 1;
+      const int64_t ctas = items * Hq;
+      const double fill = (double)ctas / (double)(((ctas + slots - 1) / slots) * slots);
+      if (fill > best_fill + 1e-9 || (fill > best_fill - 1e-9 && c > best_c)) {
+        best_fill = fill;
+        best_c = c;
+      }
+    }
+    chunk = best_c;
+  }
   // the tensor-core kernel takes groups of at least four queries
   const bool seedable = seed && decode_tc_eligible(dtype, P, p.nq);
   const int64_t samp = std::min<int64_t>(kSeedKeys, chunk / 8 / 128 * 128);

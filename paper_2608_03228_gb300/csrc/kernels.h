@@ -90,6 +90,9 @@ cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, 
 bool decode_tc_eligible(int dtype, int P, int nq);
 cudaError_t launch_merge(const ScoreArgs& a, int dtype, int kp, cudaStream_t s);
 size_t score_generic_smem(int P, int kp, int nq);
+// CTAs of the decode-shaped scoring kernel that serves (dtype, P, kp, group
+// width nq) resident per SM (0 if the query fails)
+int score_ctas_per_sm(int dtype, int P, int kp, int nq);
 
 // calibration moments: S [(Hq+Hk)][d][d] (queries first), mu [Hk][d]; err: set to 1
 // if a bounded wait of the tensor-core path gave up

@@ -12,6 +12,8 @@
 //
 // score_decode_tc_kernel runs the same work items with the scores from the
 // tensor core (bf16 keys or codes): see its comment.
+#include <atomic>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "tc.cuh"
@@ -705,6 +707,18 @@ cudaError_t launch_decode_tc_t(const ScoreArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+template <int P, int KP>
+int decode_tc_occupancy() {
+  using C = DcCfg<P>;
+  const int sm = C::smem(KP);
+  auto kern = score_decode_tc_kernel<P, KP>;
+  int n = 0;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, 192, sm) != cudaSuccess)
+    n = 0;
+  return n;
+}
+
 template <int KP>
 cudaError_t launch_decode_tc(const ScoreArgs& a, cudaStream_t s) {
   switch (a.P) {
@@ -713,6 +727,17 @@ cudaError_t launch_decode_tc(const ScoreArgs& a, cudaStream_t s) {
     case 64: return launch_decode_tc_t<64, KP>(a, s);
     default: return launch_decode_tc_t<128, KP>(a, s);
   }
+}
+
+template <typename Tin, int KP, int NQ>
+int score_occupancy(int P) {
+  const size_t sm = score_generic_smem(P, KP, NQ);
+  auto kern = score_generic_kernel<Tin, KP, NQ>;
+  int n = 0;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, kThreads, sm) != cudaSuccess)
+    n = 0;
+  return n;
 }
 
 template <typename Tin, int KP, int NQ>
@@ -750,6 +775,44 @@ cudaError_t launch_nq(const ScoreArgs& a, int nq, cudaStream_t s) {
 // kernel streams a decode step faster: 0.50 against 0.53 ms over 32 heads x 1M keys)
 bool decode_tc_eligible(int dtype, int P, int nq) {
   return dtype == SAKI_BF16 && nq >= 4 && (P == 16 || P == 32 || P == 64 || P == 128);
+}
+
+namespace {
+template <typename Tin, int KP>
+int occupancy_nq(int P, int nq) {
+  switch (nq) {
+    case 1: return score_occupancy<Tin, KP, 1>(P);
+    case 2: return score_occupancy<Tin, KP, 2>(P);
+    case 4: return score_occupancy<Tin, KP, 4>(P);
+    default: return score_occupancy<Tin, KP, 8>(P);
+  }
+}
+template <int KP>
+int occupancy_tc(int P) {
+  switch (P) {
+    case 16: return decode_tc_occupancy<16, KP>();
+    case 32: return decode_tc_occupancy<32, KP>();
+    case 64: return decode_tc_occupancy<64, KP>();
+    default: return decode_tc_occupancy<128, KP>();
+  }
+}
+}  // namespace
+
+int score_ctas_per_sm(int dtype, int P, int kp, int nq) {
+  // cached per (kernel kind, dtype, P, kp, group width): the query sets the
+  // kernel's shared-memory attribute, as its launch does
+  static std::atomic<int> cache[2][2][8][2][4];
+  const int tc = decode_tc_eligible(dtype, P, nq) ? 1 : 0;
+  const int pi = P == 16 ? 0 : P == 32 ? 1 : P == 64 ? 2 : P == 128 ? 3 : (P <= 8 ? 4 : P <= 24 ? 5 : P <= 48 ? 6 : 7);
+  const int qi = nq <= 1 ? 0 : nq <= 2 ? 1 : nq <= 4 ? 2 : 3;
+  std::atomic<int>& slot = cache[tc][dtype == SAKI_BF16 ? 1 : 0][pi][kp == 64 ? 0 : 1][qi];
+  int n = slot.load(std::memory_order_relaxed);
+  if (n > 0) return n;
+  if (tc) n = kp == 64 ? occupancy_tc<64>(P) : occupancy_tc<128>(P);
+  else if (dtype == SAKI_BF16) n = kp == 64 ? occupancy_nq<__nv_bfloat16, 64>(P, nq) : occupancy_nq<__nv_bfloat16, 128>(P, nq);
+  else n = kp == 64 ? occupancy_nq<float, 64>(P, nq) : occupancy_nq<float, 128>(P, nq);
+  if (n > 0 && (pi < 4)) slot.store(n, std::memory_order_relaxed);   // other ranks' smem varies with P: not cached
+  return n;
 }
 
 cudaError_t launch_score_generic(const ScoreArgs& a, int dtype, int kp, int nq, cudaStream_t s) {
