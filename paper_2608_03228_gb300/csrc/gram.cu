@@ -126,13 +126,18 @@ __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, c
   const int kb = tid & 7, mb = tid >> 3;   // this thread's 8 x 8 block: rows 8kb.., dimensions 8mb..
   const int nch = (int)((nl + kGramChunk - 1) / kGramChunk);
   constexpr uint32_t idesc = tc::idesc_bf16(128, 128);
-  uint4 w[8];
+  // two chunks of rows in flight per thread beyond the one being transposed
+  uint4 w[8], wn[8];
   gram_load(X, nl, 0, kb, mb, w);
+  gram_load(X, nl, kGramChunk, kb, mb, wn);   // rows past nl load as zeros
   bool ok = true;
   for (int c = 0; c < nch; ++c) {
     const int b = c & 1;
-    uint4 wn[8];
-    if (c + 1 < nch) gram_load(X, nl, (int64_t)(c + 1) * kGramChunk, kb, mb, wn);
+    uint4 wn2[8];
+    if (c + 2 < nch) gram_load(X, nl, (int64_t)(c + 2) * kGramChunk, kb, mb, wn2);
+    else
+#pragma unroll
+      for (int r = 0; r < 8; ++r) wn2[r] = make_uint4(0u, 0u, 0u, 0u);
     if (c >= 2) ok = tc::mbar_wait(done + b, ((c >> 1) & 1) ^ 1, abort_f);
     if (!__syncthreads_and(ok)) break;
     uint8_t* tile = smem + b * 16384;
@@ -162,9 +167,10 @@ __global__ void __launch_bounds__(128) gram_tc_kernel(const __nv_bfloat16* Xq, c
       }
       tc::mma_commit(done + b);
     }
-    if (c + 1 < nch) {
 #pragma unroll
-      for (int r = 0; r < 8; ++r) w[r] = wn[r];
+    for (int r = 0; r < 8; ++r) {
+      w[r] = wn[r];
+      wn[r] = wn2[r];
     }
   }
   // one more commit covers every multiplication issued (also after an early exit)
