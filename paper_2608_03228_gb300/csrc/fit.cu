@@ -475,6 +475,52 @@ __global__ void __launch_bounds__(kFitThreads, 2) factor_kernel(const float* S, 
 
 // Shared memory holds only the Jacobi matrix (68 KB), so two CTAs share an SM;
 // C'^T is kept in a global scratch slice (L2-resident) for the steps after the SVD.
+// out(i, j) = sum_p a(i, p) b(p, j) for 128 x 128 x 128 with kFitThreads
+// threads: a thread accumulates rows 4 (t % 32) .. + 3 and columns 8 (t / 32)
+// .. + 7 (three 16-byte shared loads per 32 FMAs); the K dimension goes in
+// chunks of 16, staged in stg (2 x 16 rows of 132 floats).  Each output is
+// summed over p in increasing order, one FMA at a time.
+constexpr int kStgLd = kD + 4;
+constexpr int kStgFloats = 2 * 16 * kStgLd;
+template <class LA, class LB, class ST>
+__device__ __forceinline__ void gemm128(LA la, LB lb, ST st, float* stg) {
+  float* At = stg;
+  float* Bt = stg + 16 * kStgLd;
+  const int tid = threadIdx.x;
+  const int i0 = (tid & 31) * 4, j0 = (tid >> 5) * 8;
+  float acc[4][8];
+#pragma unroll
+  for (int u = 0; u < 4; ++u)
+#pragma unroll
+    for (int v = 0; v < 8; ++v) acc[u][v] = 0.f;
+  for (int p0 = 0; p0 < kD; p0 += 16) {
+    __syncthreads();   // the previous chunk is consumed
+    for (int e = tid; e < 16 * kD; e += kFitThreads) {
+      const int kk = e & 15, i = e >> 4;
+      At[kk * kStgLd + i] = la(i, p0 + kk);
+      const int kb = e / kD, j = e % kD;
+      Bt[kb * kStgLd + j] = lb(p0 + kb, j);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      const float4 a4 = *reinterpret_cast<const float4*>(At + kk * kStgLd + i0);
+      const float4 b0 = *reinterpret_cast<const float4*>(Bt + kk * kStgLd + j0);
+      const float4 b1 = *reinterpret_cast<const float4*>(Bt + kk * kStgLd + j0 + 4);
+      const float a[4] = {a4.x, a4.y, a4.z, a4.w};
+      const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 8; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u)
+#pragma unroll
+    for (int v = 0; v < 8; ++v) st(i0 + u, j0 + v, acc[u][v]);
+}
+
 __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, const float* Fm, const float* Gm,
                                                              const float* mu, int Hq, int Hk, int r, int max_sweeps,
                                                              float tol, float* Cws, float* L, float* R, float* sigma,
@@ -496,32 +542,14 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
   float* Lh = L + (int64_t)h * kD * r;
   float* Rh = R + (int64_t)h * kD * r;
 
-  const int cc = tid % kD, r0 = (tid / kD) * 32;
-  {  // X = A Fk   (A rows broadcast from L1, Fk columns coalesced)
-    float acc[32];
-#pragma unroll
-    for (int u = 0; u < 32; ++u) acc[u] = 0.f;
-    for (int p = 0; p < kD; ++p) {
-      const float f = __ldg(Fk + p * kD + cc);
-#pragma unroll
-      for (int u = 0; u < 32; ++u) acc[u] = fmaf(__ldg(Ah + (r0 + u) * kD + p), f, acc[u]);
-    }
-#pragma unroll
-    for (int u = 0; u < 32; ++u) X[cc * kLdS + r0 + u] = acc[u];
-  }
+  float* stg = sm + kD * kLdJ;   // staging of the two products
+  // X = A Fk (column-major, ld kLdS)
+  gemm128([&](int i, int p) { return __ldg(Ah + i * kD + p); }, [&](int p, int j) { return __ldg(Fk + p * kD + j); },
+          [&](int i, int j, float v) { X[j * kLdS + i] = v; }, stg);
   __syncthreads();
-  {  // C'^T = X^T Fq, stored as C' column-major in the global scratch
-    float acc[32];
-#pragma unroll
-    for (int u = 0; u < 32; ++u) acc[u] = 0.f;
-    for (int p = 0; p < kD; ++p) {
-      const float f = __ldg(Fq + p * kD + cc);
-#pragma unroll
-      for (int u = 0; u < 32; ++u) acc[u] = fmaf(X[(r0 + u) * kLdS + p], f, acc[u]);
-    }
-#pragma unroll
-    for (int u = 0; u < 32; ++u) Ct[(r0 + u) * kD + cc] = acc[u];   // C'(cc, r0 + u)
-  }
+  // C'^T = X^T Fq, stored as C' column-major in the global scratch: C'(j, i) at [i * d + j]
+  gemm128([&](int i, int p) { return X[i * kLdS + p]; }, [&](int p, int j) { return __ldg(Fq + p * kD + j); },
+          [&](int i, int j, float v) { Ct[i * kD + j] = v; }, stg);
   __syncthreads();
   // Preconditioning: C' = Q1 R1 (Householder), then the Jacobi runs on R1^T, whose
   // left singular vectors are those of C'^T = R1^T Q1^T, i.e. the right singular
@@ -794,7 +822,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) spectrum_kernel(const float* S
 
 constexpr float kTol = 1e-6f;
 constexpr size_t kSmem = sizeof(float) * kD * kLdS;         // factor kernel: L and L^{-1} share one buffer
-constexpr size_t kFitSmem = sizeof(float) * kD * kLdJ;      // fit kernel: the Jacobi matrix
+constexpr size_t kFitSmem = sizeof(float) * (kD * kLdJ + kStgFloats);   // fit kernel: the Jacobi matrix, staging
 }  // namespace
 
 cudaError_t launch_factor(const float* S, int nmat, float floor_rel, int max_sweeps, float* F, float* Gm,
