@@ -369,11 +369,11 @@ def run_e2e(g, args, torch):
 # the heads, as the pairs do, so bench.py scales these to the workload; a kernel
 # changed after its capture is left out (traffic null).
 TRAFFIC_BYTES_PER_PAIR = {
-    "select": (571738368 + 225124608) / 2148007936,
-    "exact": (976233984 + 235627008) / 2148007936,
-    "moments": (335573504 + 3031040) / 2148007936,
-    "build": (73458176 + 13318656) / 2148007936,
-    "fit": (58777344 + 43264) / 2148007936,
+    "select": (566644480 + 224940800) / 2148007936,
+    "exact": (970252544 + 235156992) / 2148007936,
+    "moments": (335581184 + 3064064) / 2148007936,
+    "build": (73480704 + 13542656) / 2148007936,
+    "fit": (58788352 + 102144) / 2148007936,
 }
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only
 
