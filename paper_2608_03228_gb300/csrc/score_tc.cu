@@ -55,9 +55,9 @@ struct TcCfg {
   static constexpr int NB = 8;
   static constexpr int BUFC = 64;                             // TMEM columns per ring buffer
   static constexpr int PB = (P + BUFC - 1) / BUFC;
-  // ranks up to 64 store 32-bit key indices at a fixed distance from the
-  // scores (one slot pointer serves both stores of an append); rank 128 needs
-  // the room for its operands and keeps 16-bit indices in their own array
+  // ranks up to 64 store (score, 32-bit key index) pairs of 8 bytes (one
+  // 64-bit store per append); rank 128 needs the room for its operands and
+  // keeps 16-bit indices in their own array
   static constexpr bool WIDE = P <= 64;
   static constexpr int STAGES = P == 128 ? 2 : 4;
   // candidate slots per row: as many as the shared-memory budget leaves (a
@@ -95,12 +95,11 @@ struct TcCfg {
 
 // ---------------------------------------------------------------- selection
 // Selection of a row's top k runs in two passes over the same tensor-core scores.
-//   Pass 1 keeps, per row, the two highest scores of each of 64 key groups (key
-//   offset mod 64).  These 128 values are scores of distinct keys, so any value
-//   tau with at least k of them >= tau is a certified lower bound on the row's
-//   k-th best score: no key of the top k scores below tau.
+//   Pass 1 keeps, per row, the maximum of each of 128 key groups.  These are
+//   scores of distinct keys, so their k-th largest, tau, is a certified lower
+//   bound on the row's k-th best score: no key of the top k scores below tau.
 //   Pass 2 appends only the keys scoring >= tau to the row's candidate column
-//   (about 75 per row for independent scores with k = 64, against ~5 k ln(n/k)
+//   (about 87 per row for independent scores with k = 64, against ~5 k ln(n/k)
 //   for a streaming threshold), and a final exact cut leaves the top k.
 // Every helper runs with the warp converged: loops over candidate slots run to
 // the warp's largest count with per-lane predicates, so the 32 rows of a warp
