@@ -158,6 +158,38 @@ class GpuPath:
         if ev[4] is not None:
             ev[4].record()
 
+    def diagnostics(self, key_stride=64):
+        """Sec. 7 and App. C as reported statistics (untimed, after the step):
+        per head, the score-MSE reduction the fit predicts (1 - loss / sum of
+        sigma^2) against the one measured through the index on every
+        key_stride-th visible pair of the evaluation data (saki_score_mse); per
+        KV head, the key-correlation eigenvalues above the Marchenko-Pastur edge
+        (saki_key_spectrum) against the spikes the generator planted."""
+        S, d, w, torch = self.saki, self.data, self.w, self.torch
+        sig = self.sigma.double()
+        pred = (1.0 - self.loss.double() / (sig * sig).sum(1)).cpu().numpy()
+        out = torch.empty((w.num_q_heads, 3), dtype=torch.float64, device=self.dev)
+        S.saki_score_mse(self.cfg, self.lay, d["Q"], d["A"], d["K"], self.L, self.sketch, out,
+                         nu=self.nu if w.center else None, key_stride=key_stride)
+        o = out.cpu().numpy()
+        meas = 1.0 - o[:, 1] / o[:, 0]
+        eig = torch.empty((w.num_kv_heads, D), dtype=torch.float32, device=self.dev)
+        spikes = torch.empty((w.num_kv_heads,), dtype=torch.int32, device=self.dev)
+        S.saki_key_spectrum(self.cfg, d["k_calib"], eig, spikes)
+        found = spikes.cpu().numpy().astype(np.int64)
+        planted = synth.head_factors(w).spikes_k
+        return {
+            "score_mse_reduction": {"predicted_median": float(np.median(pred)), "measured_median": float(np.median(meas)),
+                                    "median_abs_diff": float(np.median(np.abs(meas - pred))),
+                                    "pairs": int(o[:, 2].sum()), "key_stride": key_stride},
+            # the stand-in population bulk is itself a Marchenko-Pastur spectrum (not
+            # white), so the count above the white-noise edge also takes in bulk
+            # eigenvalues: reported as the paper reports it, beside the planted count
+            "mp_spikes": {"above_edge_median": float(np.median(found)), "above_edge_min": int(found.min()),
+                          "above_edge_max": int(found.max()), "planted_median": float(np.median(planted)),
+                          "kv_heads": int(len(found))},
+        }
+
     def recall_with(self, method):
         """Median recall of a Tab. 1 comparison index (key PCA, weight SVD) or a
         Sec. 6 projector variant (SAP-svd, SAP-map) on the same data through the
@@ -274,6 +306,7 @@ def run_ours(args, w):
         line["recall_median_by_index"] = {"saki": line["recall_median"],
                                           **{m: g.recall_with(m) for m in ("sap_map", "sap_svd", "key_pca", "weight_svd")}}
     if not args.no_extras and world == 1 and args.workload == "llama31_8b_t4096_r32" and not args.heads:
+        line["diagnostics"] = g.diagnostics()
         del g
         torch.cuda.empty_cache()
         line["workloads"] = {name: measure_extra(name, what, args, pk, dev) for name, what in EXTRAS}
