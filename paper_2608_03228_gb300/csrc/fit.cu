@@ -317,7 +317,10 @@ __device__ void column_norms(const float* X, float* out, int ld = kLdS) {
 // the symmetric roots F = S^{1/2} = V Lambda^{1/2} V^T and G = S^{+1/2} (the
 // projector variant SAP-svd needs the right singular vectors of the
 // symmetric-root C itself).
-__global__ void __launch_bounds__(kFitThreads, 2) factor_kernel(const float* S, float floor_rel, int max_sweeps,
+// Three CTAs per SM (the Cholesky and inverse are bound by the latency of their
+// per-column barriers, so more resident matrices hide it: 1280 matrices in 3
+// waves instead of 5; the register cap spills a few words in the eigen fallback).
+__global__ void __launch_bounds__(kFitThreads, 3) factor_kernel(const float* S, float floor_rel, int max_sweeps,
                                                                 float tol, float* Fout, float* Gout, int* status,
                                                                 int sym_from) {
   extern __shared__ __align__(16) float sm[];
