@@ -20,9 +20,14 @@ constexpr int64_t kBitmapKeys = 24576;   // bitmap path: 8 warps x 3 KB of share
 __device__ __forceinline__ uint32_t slot_of(int32_t v) { return ((uint32_t)v * 2654435761u) >> 24; }
 
 // Bitmap matching: words = bitmap words per warp (dynamic shared memory, 8 warps).
+// A warp's rows go in groups of four, two groups in registers: the index lists
+// of the next group load while the current group is matched (a row alone left
+// too few bytes in flight).  KPL = index slots per lane (k <= 32 KPL).
+template <int KPL>
 __global__ void __launch_bounds__(256) recall_bitmap_kernel(const int32_t* ia, const int32_t* ie, const int32_t* vis,
                                                             int64_t T, int Hq, int k, int64_t min_visible, int words,
                                                             unsigned long long* counters) {
+  constexpr int R = 4;
   extern __shared__ uint32_t bm_all[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t* bm = bm_all + warp * words;
@@ -36,61 +41,71 @@ __global__ void __launch_bounds__(256) recall_bitmap_kernel(const int32_t* ia, c
   const int64_t nbits = (int64_t)words * 32;
   int cur_h = -1;
   unsigned long long matches = 0, rows = 0;
-  int32_t na[kPerLane], ne[kPerLane];
-  int64_t nt = r0 % T;
-  int nh = (int)(r0 / T);
-  int32_t nvis = r0 < r1 ? __ldg(vis + nt) : 0;
-  auto load_row = [&](int64_t r, int32_t (&va)[kPerLane], int32_t (&ve)[kPerLane]) {
+  int64_t lt = r0 % T;            // query of the next row to load
+  int64_t pt = r0 % T;            // query and head of the next row to match
+  int ph = (int)(r0 / T);
+  auto load_group = [&](int64_t rg, int32_t (&va)[R][KPL], int32_t (&ve)[R][KPL], int32_t (&vv)[R]) {
 #pragma unroll
-    for (int u = 0; u < kPerLane; ++u) {
-      const int i = lane + 32 * u;
-      const bool in = r < r1 && i < k;
-      va[u] = in ? __ldg(ia + r * k + i) : -1;
-      ve[u] = in ? __ldg(ie + r * k + i) : -1;
+    for (int j = 0; j < R; ++j) {
+      const int64_t r = rg + j;
+      const bool row_in = r < r1;
+#pragma unroll
+      for (int u = 0; u < KPL; ++u) {
+        const int i = lane + 32 * u;
+        const bool in = row_in && i < k;
+        va[j][u] = in ? __ldg(ia + r * k + i) : -1;
+        ve[j][u] = in ? __ldg(ie + r * k + i) : -1;
+      }
+      vv[j] = row_in ? __ldg(vis + lt) : 0;
+      if (row_in && ++lt == T) lt = 0;
     }
   };
-  load_row(r0, na, ne);
-  for (int64_t r = r0; r < r1; ++r) {
-    int32_t av[kPerLane], ev[kPerLane];
+  auto match_group = [&](int64_t rg, const int32_t (&va)[R][KPL], const int32_t (&ve)[R][KPL],
+                         const int32_t (&vv)[R]) {
 #pragma unroll
-    for (int u = 0; u < kPerLane; ++u) {
-      av[u] = na[u];
-      ev[u] = ne[u];
-    }
-    const int h = nh;
-    const int32_t row_vis = nvis;
-    if (++nt == T) {
-      nt = 0;
-      ++nh;
-    }
-    nvis = r + 1 < r1 ? __ldg(vis + nt) : 0;
-    load_row(r + 1, na, ne);
-    if (h != cur_h) {
-      if (lane == 0 && rows) {
-        atomicAdd(counters + 2 * cur_h, matches);
-        atomicAdd(counters + 2 * cur_h + 1, rows);
+    for (int j = 0; j < R; ++j) {
+      if (rg + j >= r1) break;   // warp-uniform
+      const int h = ph;
+      if (++pt == T) {
+        pt = 0;
+        ++ph;
       }
-      cur_h = h;
-      matches = rows = 0;
+      if (h != cur_h) {
+        if (lane == 0 && rows) {
+          atomicAdd(counters + 2 * cur_h, matches);
+          atomicAdd(counters + 2 * cur_h + 1, rows);
+        }
+        cur_h = h;
+        matches = rows = 0;
+      }
+      if (vv[j] < min_visible) continue;   // warp-uniform
+      // indices outside the bitmap (none from the selection calls) match nothing
+#pragma unroll
+      for (int u = 0; u < KPL; ++u)
+        if (va[j][u] >= 0 && va[j][u] < nbits) atomicOr(bm + (va[j][u] >> 5), 1u << (va[j][u] & 31));
+      __syncwarp();
+      int m = 0;
+#pragma unroll
+      for (int u = 0; u < KPL; ++u)
+        if (ve[j][u] >= 0 && ve[j][u] < nbits) m += (bm[ve[j][u] >> 5] >> (ve[j][u] & 31)) & 1u;
+      m = __reduce_add_sync(0xffffffffu, m);
+      matches += (unsigned long long)m;
+      rows += 1;
+      __syncwarp();
+#pragma unroll
+      for (int u = 0; u < KPL; ++u)
+        if (va[j][u] >= 0 && va[j][u] < nbits) bm[va[j][u] >> 5] = 0u;
+      __syncwarp();
     }
-    if (row_vis < min_visible) continue;   // warp-uniform
-    // indices outside the bitmap (none from the selection calls) match nothing
-#pragma unroll
-    for (int u = 0; u < kPerLane; ++u)
-      if (av[u] >= 0 && av[u] < nbits) atomicOr(bm + (av[u] >> 5), 1u << (av[u] & 31));
-    __syncwarp();
-    int m = 0;
-#pragma unroll
-    for (int u = 0; u < kPerLane; ++u)
-      if (ev[u] >= 0 && ev[u] < nbits) m += (bm[ev[u] >> 5] >> (ev[u] & 31)) & 1u;
-    m = __reduce_add_sync(0xffffffffu, m);
-    matches += (unsigned long long)m;
-    rows += 1;
-    __syncwarp();
-#pragma unroll
-    for (int u = 0; u < kPerLane; ++u)
-      if (av[u] >= 0 && av[u] < nbits) bm[av[u] >> 5] = 0u;
-    __syncwarp();
+  };
+  int32_t aA[R][KPL], eA[R][KPL], vA[R], aB[R][KPL], eB[R][KPL], vB[R];
+  load_group(r0, aA, eA, vA);
+  load_group(r0 + R, aB, eB, vB);
+  for (int64_t rg = r0; rg < r1; rg += 2 * R) {
+    match_group(rg, aA, eA, vA);
+    load_group(rg + 2 * R, aA, eA, vA);
+    match_group(rg + R, aB, eB, vB);
+    load_group(rg + 3 * R, aB, eB, vB);
   }
   if (lane == 0 && rows) {
     atomicAdd(counters + 2 * cur_h, matches);
@@ -216,8 +231,15 @@ cudaError_t launch_recall(const int32_t* idx_a, const int32_t* idx_e, const int3
     note_launch();
     if (max_visible <= kBitmapKeys) {
       const int words = (int)((max_visible + 31) / 32) < 1 ? 1 : (int)((max_visible + 31) / 32);
-      recall_bitmap_kernel<<<(unsigned)blocks, 256, (size_t)8 * words * sizeof(uint32_t), s>>>(
-          idx_a, idx_e, vis, T, Hq, k, min_visible, words, counters);
+      const size_t sm = (size_t)8 * words * sizeof(uint32_t);
+      // one wave: as many CTAs as are resident (the two row groups in registers
+      // leave room for fewer CTAs per SM than the table version)
+      auto kern = k <= 64 ? recall_bitmap_kernel<2> : recall_bitmap_kernel<4>;
+      int per_sm = 0;
+      if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, sm) != cudaSuccess || per_sm < 1)
+        per_sm = 1;
+      const int64_t bb = want < (int64_t)sms * per_sm ? want : (int64_t)sms * per_sm;
+      kern<<<(unsigned)bb, 256, sm, s>>>(idx_a, idx_e, vis, T, Hq, k, min_visible, words, counters);
     } else {
       recall_kernel<<<(unsigned)blocks, 256, 0, s>>>(idx_a, idx_e, vis, T, Hq, k, min_visible, counters);
     }
