@@ -121,14 +121,19 @@ __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_count
 constexpr int kLdJ = kD + 4;
 
 // jacobi_columns for a matrix with leading dimension kLdJ, with 16-byte shared
-// accesses and packed fp32 pairs (same rotations; it also stops after a sweep
-// whose rotations were all within sqrt(tol) of orthogonal, see below): lane
-// group q = lane / 8 of a warp holds rows 32 w + 4 sub + j (w, j < 4, sub =
-// lane % 8) of its pair's two columns, so a column moves in four 16-byte
+// accesses, packed fp32 pairs and a pair order that keeps one column of every
+// pair in registers (the same rotation rule and threshold; it also stops after
+// a sweep whose rotations were all within sqrt(tol) of orthogonal, see below):
+// lane group q = lane / 8 of a warp holds rows 32 w + 4 sub + j (w, j < 4,
+// sub = lane % 8) of its pair's two columns, so a column moves in four 16-byte
 // accesses per lane and the group's eight lanes cover all 32 banks; the dot
 // products and the rotation run on float2 pairs (two fp32 FMAs per instruction,
-// each rounded as the scalar one).
-__device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol, int* s_counter) {
+// each rounded as the scalar one).  With both columns of every pair loaded and
+// stored each round, the sweeps were bound by shared-memory bandwidth (128 KB
+// per round); the nested order halves that, with as many sweeps (fp32 emulation
+// on the bench's operators: 7 or 8 either way, the same singular values and
+// rank-r maps).
+__device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol) {
   __shared__ float s_red[kFitThreads / 32];
   __shared__ unsigned int s_off;   // bits of the sweep's largest rotated off-diagonality (>= 0)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -146,81 +151,90 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol, int* s_co
   const int q = lane >> 3, sub = lane & 7;
   const float stop_off = sqrtf(tol);
   for (int sweep = 0; sweep < max_sweeps; ++sweep) {
-    if (tid == 0) {
-      *s_counter = 0;
-      s_off = 0u;
-    }
+    if (tid == 0) s_off = 0u;
     __syncthreads();
-    int rot = 0;
-    float mo = 0.f;
-    // round-robin (circle) schedule: the players at the pair's two positions in
-    // round 0, then every player but 0 moves on by one (mod kD - 1) per round
-    int pa, pb;
-    rr_pair(0, (warp & 7) + 8 * q + 32 * (warp >> 3), pa, pb);
-    for (int round = 0; round < kD - 1; ++round, pa = pa == 0 ? 0 : (pa == kD - 1 ? 1 : pa + 1),
-             pb = pb == kD - 1 ? 1 : pb + 1) {
-      float4* xa = reinterpret_cast<float4*>(X + pa * kLdJ) + sub;
-      float4* xb = reinterpret_cast<float4*>(X + pb * kLdJ) + sub;
-      float2 a[8], b[8];
+    float mo = 0.f;   // the largest off-diagonality this thread's pairs rotated
+    // nested halving order: at level l the columns form 2^l blocks of 2h
+    // (h = 64 >> l); pair group g holds column i = g mod h of its block's top
+    // half in registers for the level's h rounds and meets the bottom half's
+    // column (i + s) mod h in round s.  Each unordered pair meets once per sweep
+    // (at the level that separates it), and a round moves one column per pair
+    // through shared memory instead of two.
+    const int g = (warp & 7) + 8 * q + 32 * (warp >> 3);
+#pragma unroll 1
+    for (int h = 64; h > 0; h >>= 1) {
+      const int i = g & (h - 1);
+      float* const top = X + 2 * (g - i) * kLdJ + 4 * sub;   // the block's first column
+      float2 a[8];
 #pragma unroll
       for (int w = 0; w < 4; ++w) {
-        const float4 va = xa[8 * w], vb = xb[8 * w];
+        const float4 va = *reinterpret_cast<const float4*>(top + i * kLdJ + 32 * w);
         a[2 * w] = make_float2(va.x, va.y);
         a[2 * w + 1] = make_float2(va.z, va.w);
-        b[2 * w] = make_float2(vb.x, vb.y);
-        b[2 * w + 1] = make_float2(vb.z, vb.w);
       }
-      float2 al2 = make_float2(0.f, 0.f), be2 = al2, ga2 = al2;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        al2 = __ffma2_rn(a[e], a[e], al2);
-        be2 = __ffma2_rn(b[e], b[e], be2);
-        ga2 = __ffma2_rn(a[e], b[e], ga2);
-      }
-      float al = al2.x + al2.y, be = be2.x + be2.y, ga = ga2.x + ga2.y;
-#pragma unroll
-      for (int m = 4; m > 0; m >>= 1) {  // butterflies leave the group's sums in all eight lanes
-        al += __shfl_xor_sync(0xffffffffu, al, m);
-        be += __shfl_xor_sync(0xffffffffu, be, m);
-        ga += __shfl_xor_sync(0xffffffffu, ga, m);
-      }
-      const float off = fabsf(ga) * rsqrtf(al) * rsqrtf(be);
-      if (ga != 0.f && al > tiny && be > tiny && off > tol) {
-        mo = fmaxf(mo, off);
-        // the angle only needs to be close (fast divisions); c = 1 / sqrt(1 + t^2)
-        // is rounded correctly, so that the rotation stays orthogonal
-        const float zeta = __fdividef(be - al, 2.f * ga);
-        const float t = fabsf(zeta) > 1e18f ? __fdividef(0.5f, zeta)
-                                            : __fdividef(copysignf(1.f, zeta), fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
-        const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
-        const float sn = c * t;
-        const float2 c2 = make_float2(c, c), s2 = make_float2(sn, sn), ms2 = make_float2(-sn, -sn);
+#pragma unroll 1
+      for (int s = 0; s < h; ++s) {
+        float4* xb = reinterpret_cast<float4*>(top + (h + ((i + s) & (h - 1))) * kLdJ);
+        float2 b[8];
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
-          const float2 na0 = __ffma2_rn(ms2, b[2 * w], __fmul2_rn(c2, a[2 * w]));
-          const float2 na1 = __ffma2_rn(ms2, b[2 * w + 1], __fmul2_rn(c2, a[2 * w + 1]));
-          const float2 nb0 = __ffma2_rn(s2, a[2 * w], __fmul2_rn(c2, b[2 * w]));
-          const float2 nb1 = __ffma2_rn(s2, a[2 * w + 1], __fmul2_rn(c2, b[2 * w + 1]));
-          xa[8 * w] = make_float4(na0.x, na0.y, na1.x, na1.y);
-          xb[8 * w] = make_float4(nb0.x, nb0.y, nb1.x, nb1.y);
+          const float4 vb = xb[8 * w];
+          b[2 * w] = make_float2(vb.x, vb.y);
+          b[2 * w + 1] = make_float2(vb.z, vb.w);
         }
-        if (sub == 0) ++rot;
+        float2 al2 = make_float2(0.f, 0.f), be2 = al2, ga2 = al2;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          al2 = __ffma2_rn(a[e], a[e], al2);
+          be2 = __ffma2_rn(b[e], b[e], be2);
+          ga2 = __ffma2_rn(a[e], b[e], ga2);
+        }
+        float al = al2.x + al2.y, be = be2.x + be2.y, ga = ga2.x + ga2.y;
+#pragma unroll
+        for (int m = 4; m > 0; m >>= 1) {  // butterflies leave the group's sums in all eight lanes
+          al += __shfl_xor_sync(0xffffffffu, al, m);
+          be += __shfl_xor_sync(0xffffffffu, be, m);
+          ga += __shfl_xor_sync(0xffffffffu, ga, m);
+        }
+        const float off = fabsf(ga) * rsqrtf(al) * rsqrtf(be);
+        if (ga != 0.f && al > tiny && be > tiny && off > tol) {
+          mo = fmaxf(mo, off);
+          // the angle only needs to be close (fast divisions); c = 1 / sqrt(1 + t^2)
+          // is rounded correctly, so that the rotation stays orthogonal
+          const float zeta = __fdividef(be - al, 2.f * ga);
+          const float t = fabsf(zeta) > 1e18f ? __fdividef(0.5f, zeta)
+                                              : __fdividef(copysignf(1.f, zeta), fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
+          const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
+          const float sn = c * t;
+          const float2 c2 = make_float2(c, c), s2 = make_float2(sn, sn), ms2 = make_float2(-sn, -sn);
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            const float2 nb0 = __ffma2_rn(s2, a[2 * w], __fmul2_rn(c2, b[2 * w]));
+            const float2 nb1 = __ffma2_rn(s2, a[2 * w + 1], __fmul2_rn(c2, b[2 * w + 1]));
+            a[2 * w] = __ffma2_rn(ms2, b[2 * w], __fmul2_rn(c2, a[2 * w]));
+            a[2 * w + 1] = __ffma2_rn(ms2, b[2 * w + 1], __fmul2_rn(c2, a[2 * w + 1]));
+            xb[8 * w] = make_float4(nb0.x, nb0.y, nb1.x, nb1.y);
+          }
+        }
+        if (s == h - 1) {   // the level's last round: the top-half column goes home
+#pragma unroll
+          for (int w = 0; w < 4; ++w)
+            *reinterpret_cast<float4*>(top + i * kLdJ + 32 * w) =
+                make_float4(a[2 * w].x, a[2 * w].y, a[2 * w + 1].x, a[2 * w + 1].y);
+        }
+        __syncthreads();
       }
-      __syncthreads();
     }
-    if (sub == 0 && rot) {   // one counter per pair group
-      atomicAdd(s_counter, rot);
-      atomicMax(&s_off, __float_as_uint(mo));
-    }
+    if (sub == 0 && mo > 0.f) atomicMax(&s_off, __float_as_uint(mo));   // one update per pair group
     __syncthreads();
-    const int total = *s_counter;
     const float max_off = __uint_as_float(s_off);
     __syncthreads();
-    // done when nothing rotated, or when every rotated pair was within sqrt(tol)
-    // of orthogonal: cyclic Jacobi converges quadratically there, so the next
-    // sweep would find the pairs near tol (float32 emulation on the bench's
-    // operators: the same singular values and rank-r maps, one or two sweeps fewer)
-    if (total == 0 || max_off <= stop_off) return true;
+    // done when every rotated pair was within sqrt(tol) of orthogonal (max_off
+    // stays 0 when nothing rotated): cyclic Jacobi converges quadratically
+    // there, so the next sweep would find the pairs near tol (float32 emulation
+    // on the bench's operators: the same singular values and rank-r maps, one
+    // or two sweeps fewer)
+    if (max_off <= stop_off) return true;
   }
   return false;
 }
@@ -533,7 +547,6 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
   __shared__ float sig[kD];
   __shared__ float sgn[kD];
   __shared__ int perm[kD];
-  __shared__ int counter;
   const int h = blockIdx.x, g = h / (Hq / Hk);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const float* Ah = A + (int64_t)h * kD * kD;
@@ -576,7 +589,7 @@ __global__ void __launch_bounds__(kFitThreads, 2) fit_kernel(const float* A, con
   }
   __syncthreads();
 
-  const bool conv = jacobi_columns_v4(X, max_sweeps, tol, &counter);
+  const bool conv = jacobi_columns_v4(X, max_sweeps, tol);
   if (!conv && tid == 0) status[h] |= kStNotConverged;
   column_norms(X, sig, kLdJ);
   __syncthreads();
