@@ -242,10 +242,12 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol) {
 // Householder QR of the matrix in X (column-major, leading dimension kLdS), in
 // place: on return R occupies the upper triangle (diagonal included); below it,
 // the reflector vectors are left behind.  Needs kFitThreads threads.  One
-// barrier per column: warp 0 updates column j + 1 first and then derives the
-// next reflector from it while the other warps finish step j (parameters
-// double-buffered by step parity); the new diagonal is written without a
-// barrier, as the trailing update never reads it.
+// barrier per column: warp 0, whose first trailing column is j + 1, derives the
+// next reflector from it once its columns are done (parameters double-buffered
+// by step parity); the new diagonal is written without a barrier, as the
+// trailing update never reads it.  Lane l holds rows l + 32 u of every column
+// it touches, and a warp reduces four columns' dot products together (the
+// step's cost is the latency of those butterflies, not their arithmetic).
 
 // Reflector parameters of column x below row j - 1 (warp-wide; lane 0 writes):
 // alpha (the new diagonal), v_j, and 2 / |v|^2 (0 when there is nothing to reflect).
@@ -268,44 +270,58 @@ __device__ __forceinline__ void householder_par(const float* x, int j, float* pa
 __device__ void householder_r(float* X) {
   __shared__ float s_par[2][3];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int kWarps = kFitThreads / 32;
   if (warp == 0) householder_par(X, 0, s_par[0], lane);
   __syncthreads();
   for (int j = 0; j < kD - 1; ++j) {
     const float* par = s_par[j & 1];
     float* nxt = s_par[(j + 1) & 1];
     const float v0 = par[1], inv = par[2];
-    float* xj = X + j * kLdS;
+    const float* xj = X + j * kLdS;
     if (inv > 0.f) {
-      // trailing columns: c -= (2 v.c / |v|^2) v, two columns per warp at a time
-      for (int c = j + 1 + warp; c < kD; c += 2 * (kFitThreads / 32)) {
-        const int c2 = c + kFitThreads / 32;
-        float* xc = X + c * kLdS;
-        float* xd = X + (c2 < kD ? c2 : c) * kLdS;
-        float d1 = lane == 0 ? v0 * xc[j] : 0.f, d2 = lane == 0 ? v0 * xd[j] : 0.f;
-        for (int i = j + 1 + lane; i < kD; i += 32) {
-          d1 = fmaf(xj[i], xc[i], d1);
-          d2 = fmaf(xj[i], xd[i], d2);
+      // the reflector v in the lane's rows lane + 32 u: v_j = v0, v_i = x_j(i) below
+      float v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = lane + 32 * u;
+        v[u] = i > j ? xj[i] : (i == j ? v0 : 0.f);
+      }
+      // trailing columns c = j + 1 + warp + 16 t, four per warp at a time: their
+      // dot products with v reduce together, so the butterflies overlap
+#pragma unroll 1
+      for (int c0 = j + 1 + warp; c0 < kD; c0 += 4 * kWarps) {
+        float x[4][4], dt[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int c = c0 + t * kWarps;
+          dt[t] = 0.f;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            x[t][u] = c < kD ? X[c * kLdS + lane + 32 * u] : 0.f;
+            dt[t] = fmaf(v[u], x[t][u], dt[t]);
+          }
         }
 #pragma unroll
-        for (int m = 16; m > 0; m >>= 1) {
-          d1 += __shfl_xor_sync(0xffffffffu, d1, m);
-          d2 += __shfl_xor_sync(0xffffffffu, d2, m);
-        }
-        const float f1 = d1 * inv, f2 = d2 * inv;
-        if (lane == 0) {
-          xc[j] = fmaf(-f1, v0, xc[j]);
-          if (c2 < kD) xd[j] = fmaf(-f2, v0, xd[j]);
-        }
-        for (int i = j + 1 + lane; i < kD; i += 32) {
-          xc[i] = fmaf(-f1, xj[i], xc[i]);
-          if (c2 < kD) xd[i] = fmaf(-f2, xj[i], xd[i]);
-        }
-        if (c == j + 1) {   // warp 0: column j + 1 is final for step j + 1
-          __syncwarp();
-          householder_par(xc, j + 1, nxt, lane);
+        for (int m = 16; m > 0; m >>= 1)
+#pragma unroll
+          for (int t = 0; t < 4; ++t) dt[t] += __shfl_xor_sync(0xffffffffu, dt[t], m);
+        // c -= (2 v.c / |v|^2) v on rows j and below
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int c = c0 + t * kWarps;
+          const float f = dt[t] * inv;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int i = lane + 32 * u;
+            if (c < kD && i >= j) X[c * kLdS + i] = fmaf(-f, v[u], x[t][u]);
+          }
         }
       }
-      if (tid == 0) xj[j] = par[0];
+      if (warp == 0) {   // warp 0 updated column j + 1 (c0 = j + 1): the next reflector
+        __syncwarp();
+        householder_par(X + (j + 1) * kLdS, j + 1, nxt, lane);
+      }
+      if (tid == 0) X[j * kLdS + j] = par[0];
     } else if (warp == 0) {
       householder_par(X + (j + 1) * kLdS, j + 1, nxt, lane);   // nothing to reflect: column j + 1 unchanged
     }
