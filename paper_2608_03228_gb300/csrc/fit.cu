@@ -384,16 +384,16 @@ __global__ void __launch_bounds__(kFitThreads, 3) factor_kernel(const float* S, 
   }
   const float trace = red[0];
 
-  const bool sym = m >= sym_from;
-  if (sym && tid == 0) flag = 3;   // skip the Cholesky path
-  __syncthreads();
-  // Cholesky, right-looking, in place
-  for (int j = 0; j < kD && !sym; ++j) {
+  const bool sym = m >= sym_from;   // symmetric roots: skip the Cholesky path
+  // Cholesky, right-looking, in place; every thread reads the same pivot (the
+  // last barrier of step j - 1 made it final), so all leave together
+  bool chol_ok = !sym;
+  for (int j = 0; j < kD && chol_ok; ++j) {
     const float piv = Sb[j * kLdS + j];
-    const bool ok = piv > 0.f && isfinite(piv);
-    if (!ok) { if (tid == 0) flag = 1; }
-    __syncthreads();
-    if (flag) break;
+    if (!(piv > 0.f && isfinite(piv))) {
+      chol_ok = false;
+      break;
+    }
     const float ljj = sqrtf(piv);
     for (int i = j + 1 + tid; i < kD; i += kFitThreads) Sb[i * kLdS + j] /= ljj;
     __syncthreads();
@@ -406,7 +406,6 @@ __global__ void __launch_bounds__(kFitThreads, 3) factor_kernel(const float* S, 
     __syncthreads();
   }
 
-  bool chol_ok = (flag == 0) && !sym;
   if (chol_ok) {
     // Linv = F^{-1} by right-looking substitution on the identity: row i is
     // divided by F_ii, then subtracted (times F_ri) from every row below it.
@@ -459,7 +458,9 @@ __global__ void __launch_bounds__(kFitThreads, 3) factor_kernel(const float* S, 
     return;
   }
 
-  // exact floor: eigenpairs from one-sided Jacobi on S itself
+  // exact floor: eigenpairs from one-sided Jacobi on S itself (the barrier: a
+  // failed pivot leaves the Cholesky loop without one, and Xb overwrites Sb)
+  __syncthreads();
   for (int o = tid; o < kD * kD; o += kFitThreads) Xb[(o % kD) * kLdS + (o / kD)] = Sm[o];
   __syncthreads();
   const bool conv = jacobi_columns(Xb, max_sweeps, tol, &counter);
