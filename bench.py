@@ -397,16 +397,18 @@ def run_e2e(g, args, torch):
 
 
 # DRAM bytes (read + write) per visible pair, from one ncu capture of each kernel
-# as it stands (profiles/score_tc_llama31_h32.md: the Llama-3.1-8B shapes at 256
-# query heads, inputs larger than L2).  At fixed T and N the traffic grows with
-# the heads, as the pairs do, so bench.py scales these to the workload; a kernel
-# changed after its capture is left out (traffic null).
+# as it stands (profiles/score_tc_llama31_h32.md and profiles/fit_gram_llama31_h32.md:
+# the Llama-3.1-8B shapes at 256 query heads, inputs larger than L2).  At fixed T
+# and N the traffic grows with the heads, as the pairs do, so bench.py scales
+# these to the workload; a kernel changed after its capture is left out (traffic
+# null).
 TRAFFIC_BYTES_PER_PAIR = {
     "select": (566644480 + 224940800) / 2148007936,
     "exact": (970252544 + 235156992) / 2148007936,
     "moments": (335581184 + 3064064) / 2148007936,
     "build": (73480704 + 13542656) / 2148007936,
-    "fit": (58788352 + 102144) / 2148007936,
+    "fit": (58884096 + 257536) / 2148007936,
+    "factor": (21018368 + 12544) / 2148007936,
 }
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only
 
