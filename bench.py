@@ -407,7 +407,6 @@ TRAFFIC_BYTES_PER_PAIR = {
     "exact": (970252544 + 235156992) / 2148007936,
     "moments": (335581184 + 3064064) / 2148007936,
     "build": (73480704 + 13542656) / 2148007936,
-    "fit": (58884096 + 257536) / 2148007936,
     "factor": (21018368 + 12544) / 2148007936,
 }
 TRAFFIC_WORKLOAD = "llama31_8b_t4096_r32"   # the figures hold for these shapes only

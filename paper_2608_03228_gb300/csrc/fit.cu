@@ -116,6 +116,18 @@ __device__ bool jacobi_columns(float* X, int max_sweeps, float tol, int* s_count
   return false;
 }
 
+// x . y over the 128 rows that a lane group of eight holds (16 per lane as
+// float2 pairs), in all eight lanes.
+__device__ __forceinline__ float group_dot(const float2 (&x)[8], const float2 (&y)[8]) {
+  float2 p = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int e = 0; e < 8; ++e) p = __ffma2_rn(x[e], y[e], p);
+  float v = p.x + p.y;
+#pragma unroll
+  for (int m = 4; m > 0; m >>= 1) v += __shfl_xor_sync(0xffffffffu, v, m);
+  return v;
+}
+
 // Leading dimension of the fit kernel's Jacobi matrix: 16-byte aligned columns
 // whose starts step through the banks by four.
 constexpr int kLdJ = kD + 4;
@@ -136,6 +148,7 @@ constexpr int kLdJ = kD + 4;
 __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol) {
   __shared__ float s_red[kFitThreads / 32];
   __shared__ unsigned int s_off;   // bits of the sweep's largest rotated off-diagonality (>= 0)
+  __shared__ float s_nrm[kD];      // squared norms of the rotating columns, carried through a level
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float fro = 0.f;
   for (int o = tid; o < kD * kD; o += kFitThreads) {
@@ -172,9 +185,14 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol) {
         a[2 * w] = make_float2(va.x, va.y);
         a[2 * w + 1] = make_float2(va.z, va.w);
       }
+      // squared norms: exact at the level's start (the top-half column here, each
+      // bottom-half column in round 0, where exactly one group meets it), then
+      // carried through the rotations, |a'|^2 = |a|^2 - t g and |b'|^2 = |b|^2 + t g
+      float al = group_dot(a, a);
 #pragma unroll 1
       for (int s = 0; s < h; ++s) {
-        float4* xb = reinterpret_cast<float4*>(top + (h + ((i + s) & (h - 1))) * kLdJ);
+        const int cb = 2 * (g - i) + h + ((i + s) & (h - 1));
+        float4* xb = reinterpret_cast<float4*>(top + (cb - 2 * (g - i)) * kLdJ);
         float2 b[8];
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
@@ -182,20 +200,8 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol) {
           b[2 * w] = make_float2(vb.x, vb.y);
           b[2 * w + 1] = make_float2(vb.z, vb.w);
         }
-        float2 al2 = make_float2(0.f, 0.f), be2 = al2, ga2 = al2;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          al2 = __ffma2_rn(a[e], a[e], al2);
-          be2 = __ffma2_rn(b[e], b[e], be2);
-          ga2 = __ffma2_rn(a[e], b[e], ga2);
-        }
-        float al = al2.x + al2.y, be = be2.x + be2.y, ga = ga2.x + ga2.y;
-#pragma unroll
-        for (int m = 4; m > 0; m >>= 1) {  // butterflies leave the group's sums in all eight lanes
-          al += __shfl_xor_sync(0xffffffffu, al, m);
-          be += __shfl_xor_sync(0xffffffffu, be, m);
-          ga += __shfl_xor_sync(0xffffffffu, ga, m);
-        }
+        const float ga = group_dot(a, b);
+        float be = s == 0 ? group_dot(b, b) : s_nrm[cb];
         const float off = fabsf(ga) * rsqrtf(al) * rsqrtf(be);
         if (ga != 0.f && al > tiny && be > tiny && off > tol) {
           mo = fmaxf(mo, off);
@@ -206,6 +212,8 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol) {
                                               : __fdividef(copysignf(1.f, zeta), fabsf(zeta) + sqrtf(fmaf(zeta, zeta, 1.f)));
           const float c = 1.f / sqrtf(fmaf(t, t, 1.f));
           const float sn = c * t;
+          al = fmaxf(fmaf(-t, ga, al), 0.f);
+          be = fmaxf(fmaf(t, ga, be), 0.f);
           const float2 c2 = make_float2(c, c), s2 = make_float2(sn, sn), ms2 = make_float2(-sn, -sn);
 #pragma unroll
           for (int w = 0; w < 4; ++w) {
@@ -216,6 +224,7 @@ __device__ bool jacobi_columns_v4(float* X, int max_sweeps, float tol) {
             xb[8 * w] = make_float4(nb0.x, nb0.y, nb1.x, nb1.y);
           }
         }
+        if (sub == 0) s_nrm[cb] = be;
         if (s == h - 1) {   // the level's last round: the top-half column goes home
 #pragma unroll
           for (int w = 0; w < 4; ++w)
