@@ -218,6 +218,87 @@ def test_bf16_rounding_matches_torch_on_fp32_values():
     np.testing.assert_array_equal(O.round_bf16(x.astype(np.float64)), ref)
 
 
+def test_round_to_float32_is_round_to_nearest_even():
+    """Hand cases of IEEE binary32 rounding (24-bit significand): halfway
+    values go to the even neighbour, anything above halfway rounds up."""
+    u = 2.0 ** -23   # float32 spacing at 1
+    cases = [(1 + u / 2, 1.0),                    # halfway, 1 is even
+             (1 + 3 * u / 2, 1 + 2 * u),          # halfway, 1 + 2u is even
+             (1 + u / 2 + 2.0 ** -40, 1 + u),     # just above halfway
+             (-(1 + u / 2), -1.0),
+             (3.0, 3.0)]
+    for x, want in cases:
+        assert float(O.round_to("f32", np.array([x]))[0]) == want, x
+    x = np.random.default_rng(9).standard_normal(64)
+    np.testing.assert_array_equal(O.round_to("bf16", x), O.round_bf16(x))
+    with pytest.raises(ValueError):
+        O.round_to("f16", x)
+
+
+# ------------------------------------------------------------ oracle helpers
+def test_psd_roots_match_scipy_sqrtm_on_a_definite_matrix():
+    scipy_linalg = pytest.importorskip("scipy.linalg")
+    rng = np.random.default_rng(10)
+    B = rng.standard_normal((12, 12))
+    S = B @ B.T + 0.5 * np.eye(12)
+    root, iroot = O.psd_roots(S)
+    ref = np.real(scipy_linalg.sqrtm(S))
+    np.testing.assert_allclose(root, ref, atol=1e-10)
+    np.testing.assert_allclose(iroot, np.linalg.inv(ref), atol=1e-10)
+
+
+def test_psd_roots_drop_eigenvalues_below_the_floor():
+    """App. A: eigenvalues below floor * lambda_max count as zero in both roots.
+    Built from a seeded orthogonal basis with eigenvalues 40 x (1, 0.5, 2e-6,
+    5e-7, 0): at the 1e-6 relative floor the third is kept and the last two are
+    dropped (an absolute floor of 1e-6 would keep the fourth, 2e-5)."""
+    U, _ = np.linalg.qr(np.random.default_rng(11).standard_normal((5, 5)))
+    lam = 40.0 * np.array([1.0, 0.5, 2e-6, 5e-7, 0.0])
+    S = (U * lam) @ U.T
+    root, iroot = O.psd_roots(S, floor_rel=1e-6)
+    kept = U[:, :3]
+    P = kept @ kept.T
+    np.testing.assert_allclose(root @ root, S - lam[3] * np.outer(U[:, 3], U[:, 3]), atol=1e-11)
+    np.testing.assert_allclose(iroot @ root, P, atol=1e-8)
+    np.testing.assert_allclose(root @ iroot, P, atol=1e-8)
+    np.testing.assert_allclose(iroot @ S @ iroot, P, atol=1e-8)
+    np.testing.assert_allclose(iroot @ U[:, 3], 0.0, atol=1e-8)   # dropped directions vanish
+    np.testing.assert_allclose(root, root.T, atol=1e-14)
+    np.testing.assert_allclose(iroot, iroot.T, atol=1e-8)
+
+
+def test_canonical_signs_hand_example_and_ties():
+    """Each column pair is flipped so that R's largest-magnitude entry is
+    positive (ties: the first such row); L R^T is unchanged."""
+    L = np.array([[1.0, 2.0, 5.0], [3.0, 4.0, 6.0]])
+    R = np.array([[1.0, -3.0, -2.0], [2.0, 1.0, 2.0]])
+    L2, R2 = O.canonical_signs(L, R)
+    np.testing.assert_array_equal(R2, [[1.0, 3.0, 2.0], [2.0, -1.0, -2.0]])
+    np.testing.assert_array_equal(L2, [[1.0, -2.0, -5.0], [3.0, -4.0, -6.0]])
+    np.testing.assert_array_equal(L2 @ R2.T, L @ R.T)
+    np.testing.assert_array_equal(R, [[1.0, -3.0, -2.0], [2.0, 1.0, 2.0]])   # inputs untouched
+
+
+def test_orthonormal_basis_spans_the_columns_and_matches_householder_qr():
+    X = np.random.default_rng(12).standard_normal((16, 5))
+    Q = O._orth(X)
+    np.testing.assert_allclose(Q.T @ Q, np.eye(5), atol=1e-12)
+    np.testing.assert_allclose(Q @ Q.T, X @ np.linalg.solve(X.T @ X, X.T), atol=1e-12)
+    Qh, Rh = np.linalg.qr(X)   # Householder; Gram-Schmidt gives R a positive diagonal
+    np.testing.assert_allclose(Q, Qh * np.sign(np.diag(Rh)), atol=1e-12)
+
+
+def test_projector_map_factors():
+    rng = np.random.default_rng(13)
+    Q = O._orth(rng.standard_normal((8, 3)))
+    A = rng.standard_normal((8, 8))
+    out = O._projector_head(Q, A)
+    np.testing.assert_allclose(out["M"], A @ Q @ Q.T, atol=1e-12)
+    np.testing.assert_allclose(out["R"].T @ out["R"], np.eye(3), atol=1e-12)
+    np.testing.assert_allclose(np.abs(out["R"]), np.abs(Q), atol=0)
+    np.testing.assert_allclose(out["L"], A @ out["R"], atol=1e-12)
+
+
 # ------------------------------------------------------------ selection, recall
 def test_topk_against_brute_force_with_ties():
     rng = np.random.default_rng(5)
