@@ -324,6 +324,31 @@ def test_recall_golden_example():
     assert O.median_over_heads([0.2, 0.9, 0.5, 0.7]) == 0.6
 
 
+def test_recall_boundary_divisor_and_head_mean():
+    """Sec. 3 protocol: a row with exactly min_visible visible keys counts; the
+    divisor is k even when fewer than k keys are visible (a row of 3 visible
+    keys with min_visible 3 and k 4 scores 3/4 with every key found); a head's
+    recall is the mean of its rows (1, 1 and 1/4: 0.75, where the median is 1)."""
+    k = 4
+    ia = np.array([[0, 1, 2, 3], [0, 1, 2, -1], [9, 8, 7, 3]])
+    ie = np.array([[3, 2, 1, 0], [2, 1, 0, -1], [0, 1, 2, 3]])
+    rows = O.recall_rows(ia, ie, np.array([10, 3, 10]), 3, k)
+    np.testing.assert_array_equal(rows, [1.0, 0.75, 0.25])
+    rows = O.recall_rows(ia, ie, np.array([10, 3, 10]), 4, k)
+    assert np.isnan(rows[1]) and rows[0] == 1.0
+    ia2 = np.array([[[0, 1, 2, 3], [4, 5, 6, 7], [9, 8, 7, 3]]])
+    ie2 = np.array([[[0, 1, 2, 3], [7, 6, 5, 4], [0, 1, 2, 3]]])
+    assert O.head_recall(ia2, ie2, np.array([10, 10, 10]), 5, k)[0] == 0.75
+
+
+def test_bf16_rounding_matches_torch_in_the_subnormal_range():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(14)
+    x = (rng.uniform(-1, 1, 20000) * 2.0 ** rng.integers(-149, -120, 20000)).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.round_bf16(x.astype(np.float64)), ref)
+
+
 def test_margin_condition_guarantees_exact_top_k():
     """Prop. 2: |s - s_hat| <= eps for all j and 2 eps < gamma_k => same top-k set;
     at 2 eps > gamma_k a perturbation exists that swaps the boundary pair."""
@@ -358,6 +383,29 @@ def test_full_rank_index_reproduces_exact_scores_with_centering():
     codes = O.build_index(K, res["R"], res["mu"], "f32", 1)
     s_hat = O.approx_scores(q, res["L"][0], codes[0]) + q @ res["nu"][0]
     np.testing.assert_allclose(s_hat, O.exact_scores(q, A, K[0]), rtol=2e-5, atol=2e-5)
+    # the selection's returned scores carry the same q^T nu term
+    Q = q[None, None, :]
+    off, seq, vis = np.array([0]), np.array([0]), np.array([40])
+    _, S_hat = O.score_topk(Q, res["L"], codes, off, seq, vis, 8, nu=res["nu"])
+    _, S = O.exact_topk(Q, A[None], K, off, seq, vis, 8, 1)
+    np.testing.assert_allclose(S_hat[0, 0], S[0, 0], rtol=2e-5, atol=2e-5)
+
+
+def test_build_index_maps_query_heads_to_their_kv_head():
+    """GQA (Sec. 6): with 2 KV heads and groups of 2, query head h codes the
+    keys of KV head h // 2.  KV head g holds keys (g + 1) e_0 with mean
+    (g + 1) / 2 e_0 (head 0) or e_0 (head 1); R_h has (h + 1) at (0, 0), so code
+    entry 0 is (g + 1 - mu_g) (h + 1): 0.5, 1, 3, 4 for h = 0..3."""
+    d, N, r = 4, 3, 2
+    K = np.zeros((2, N, d))
+    K[0, :, 0], K[1, :, 0] = 1.0, 2.0
+    R = np.zeros((4, d, r))
+    for h in range(4):
+        R[h, 0, 0] = h + 1
+    mu = np.array([[0.5, 0, 0, 0], [1.0, 0, 0, 0]])
+    codes = O.build_index(K, R, mu, "f32", group=2)
+    np.testing.assert_array_equal(codes[:, :, 0], np.array([[0.5] * N, [1.0] * N, [3.0] * N, [4.0] * N]))
+    np.testing.assert_array_equal(codes[:, :, 1], 0.0)
 
 
 def test_exact_scores_by_double_loop():
@@ -636,6 +684,22 @@ def test_ledoit_wolf_limits():
     S, rho, _ = O.ledoit_wolf(X, False)
     assert rho > 0.5
     np.testing.assert_allclose(np.trace(S), np.trace(X.T @ X / 8), rtol=1e-12)   # the trace is kept
+
+
+def test_ledoit_wolf_clips_the_intensity_at_one():
+    """rho = min(b2, d2) / d2: four draws in six dimensions (seed 0) give an
+    estimated error b2 above the dispersion d2, so S* is the scaled identity."""
+    X = np.random.default_rng(0).standard_normal((4, 6))
+    S, _ = O.moments(X, False)
+    m = np.trace(S) / 6
+    d2 = np.sum((S - m * np.eye(6)) ** 2)
+    b2 = sum(np.sum((np.outer(x, x) - S) ** 2) for x in X) / 16
+    assert b2 > d2
+    S_star, rho, _ = O.ledoit_wolf(X, False)
+    assert rho == 1.0
+    np.testing.assert_allclose(S_star, m * np.eye(6), atol=1e-14)
+    sk = pytest.importorskip("sklearn.covariance")
+    np.testing.assert_allclose(sk.ledoit_wolf(X, assume_centered=True)[1], 1.0)
 
 
 def test_correlation_spectrum_and_mp_edge():
