@@ -11,8 +11,8 @@
 //   2. main loop over 64-key tiles of the visible range: TMA brings the key
 //      rows (codes, or raw keys for the exact scores) into a ring of
 //      shared-memory stages; one thread issues tcgen05.mma (M = 128 queries,
-//      N = 64 keys, K = P, twice: u_hi and u_lo) into a ring of TMEM
-//      accumulators (eight of 64 columns, four of 128 at rank 128);
+//      N = 64 keys, K = P, twice: u_hi and u_lo) into a ring of eight TMEM
+//      accumulators of 64 columns (a rank-128 projection spans two);
 //   3. four epilogue warps own one query row per thread (TMEM lane = row) and
 //      select in two passes over the same scores (the key tiles are multiplied
 //      twice; the tensor core has ample headroom): pass 1 folds every score
