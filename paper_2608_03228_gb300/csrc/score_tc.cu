@@ -183,23 +183,6 @@ __device__ __forceinline__ float pick(const float (&s)[N], int q) {
   return p;
 }
 
-// Entries scoring >= p among the lane's first cnt (slots read up to the warp's cmax).
-template <class Col>
-__device__ __forceinline__ int count_ge(const Col& c, int cnt, int cmax, float p) {
-  int n0 = 0, n1 = 0;
-  for (int i = 0; i < cmax; i += 8) {
-    float v[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) v[u] = c.s(i + u);
-#pragma unroll
-    for (int u = 0; u < 8; u += 2) {
-      n0 += (i + u < cnt && v[u] >= p) ? 1 : 0;
-      n1 += (i + u + 1 < cnt && v[u + 1] >= p) ? 1 : 0;
-    }
-  }
-  return n0 + n1;
-}
-
 // Lanes with `on` keep their entries scoring >= p (in place, order preserved).
 template <class Col>
 __device__ __forceinline__ int compact_ge(const Col& c, int cnt, int cmax, float p, bool on) {
