@@ -216,7 +216,8 @@ SAKI_API saki_status saki_fit_moments(const saki_config* cfg, const float* Sq, c
 
 /* saki_reconstruct_keys -- composition with RoPE (Sec. 6: reconstruct
  * k_hat = mu + M_r (k - mu) and rotate).  For every query head h and each of
- * the n_rows code rows rows[i] (device int64, rows of the sketch):
+ * the n_rows code rows rows[i] (device int64, rows of the sketch; a row
+ * outside [0, total_keys) reads nothing and its key comes out NaN):
  *   k_hat = nu_h + L_h c,  so that q^T k_hat is the index's score with the mean
  *   term (in the paper's head coordinates, where A is absorbed, nu = mu and
  *   L_h c = M_r (k - mu));
@@ -227,7 +228,10 @@ SAKI_API saki_status saki_fit_moments(const saki_config* cfg, const float* Sq, c
  *   sketch [Hq][total_keys][r] dtype, L [Hq][d][r] f32, nu [Hq][d] f32 or NULL,
  *   keys [Hq][n_rows][d] dtype (written).
  * Workspace (only with positions): saki_workspace_size(SAKI_OP_RECONSTRUCT,
- * total_keys = n_rows).  Stream-ordered; uploads nothing. */
+ * total_keys = n_rows).  SAKI_ERR_INVALID_ARGUMENT for negative counts, NULL
+ * tensors when n_rows > 0, positions without a workspace or with rope_theta
+ * <= 1, or a misaligned pointer; SAKI_ERR_WORKSPACE if the workspace is too
+ * small.  Stream-ordered; uploads nothing (so it may be captured). */
 SAKI_API saki_status saki_reconstruct_keys(const saki_config* cfg, int64_t n_rows, const int64_t* rows,
                                            int64_t total_keys, const void* sketch, const float* L,
                                            const float* nu, const int64_t* positions, float rope_theta,
@@ -239,7 +243,14 @@ SAKI_API saki_status saki_reconstruct_keys(const saki_config* cfg, int64_t n_row
  *   K      [Hk][total_keys][d] dtype
  *   R      [Hq][d][r] f32
  *   mu     [Hk][d] f32, read only when center = 1 (then required)
- *   sketch [Hq][total_keys][r] dtype, written; rounded to nearest-even. */
+ *   sketch [Hq][total_keys][r] dtype, written; rounded to nearest-even.
+ * Workspace: saki_workspace_size(SAKI_OP_BUILD_INDEX) bytes, required for bf16
+ * uncentered keys (the tensor-core path, which reports a device timeout through
+ * the header's error word); other builds take none (NULL allowed; a workspace
+ * passed along gets its error word cleared).  SAKI_ERR_INVALID_ARGUMENT for
+ * NULL tensors when total_keys > 0, a missing mu when center = 1, a missing
+ * workspace on the tensor-core path or a misaligned pointer; SAKI_ERR_WORKSPACE
+ * if the workspace is too small.  Stream-ordered. */
 SAKI_API saki_status saki_build_index(const saki_config* cfg, int64_t total_keys, const void* K,
                              const float* R, const float* mu, void* sketch, void* workspace,
                              size_t workspace_bytes, saki_stream stream);
@@ -259,7 +270,16 @@ SAKI_API saki_status saki_build_index(const saki_config* cfg, int64_t total_keys
  * Decode-shaped groups (at least four bf16 queries of one sequence whose keys
  * are cut into eight or more splits) first run a sample pass over the head of
  * every split, whose per-query bound starts each split's selection; the result
- * is the same as without it. */
+ * is the same as without it.
+ * Workspace: saki_workspace_size(SAKI_OP_SCORE_TOPK) bytes, required when T > 0
+ * (T = 0 returns SAKI_OK and launches nothing).  SAKI_ERR_INVALID_ARGUMENT for
+ * a malformed layout (seq_offsets[0] != 0, a decreasing offset, q_seq out of
+ * range, q_visible beyond its sequence) or NULL / misaligned tensors;
+ * SAKI_ERR_UNSUPPORTED for d != 128, k > 128, more than 65535 query heads,
+ * more than 2^31 - 1 queries or a sequence of more than 2^31 - 2 keys;
+ * SAKI_ERR_WORKSPACE if the
+ * workspace holds neither plan.  Stream-ordered; a device timeout is read by
+ * saki_workspace_status. */
 SAKI_API saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, const void* Q,
                             const float* L, const void* sketch, const float* nu, int32_t* idx,
                             float* score, void* workspace, size_t workspace_bytes,
@@ -272,7 +292,11 @@ SAKI_API saki_status saki_score_topk(const saki_config* cfg, const saki_layout* 
  *   idx_approx [Hq][T][k] int32   e.g. the output of saki_score_topk
  *   idx_exact  [Hq][T][k] int32 or NULL (then kept in the workspace)
  *   recall     [Hq] f32, NaN for a head with no qualifying query
- * Medians across heads (Tab. 1) are left to the caller. */
+ * Medians across heads (Tab. 1) are left to the caller.
+ * Workspace: saki_workspace_size(SAKI_OP_RECALL) bytes, always required (it
+ * holds the per-head counts, and the exact lists when idx_exact is NULL).
+ * Errors as saki_score_topk (recall and workspace must not be NULL).
+ * Stream-ordered; a device timeout is read by saki_workspace_status. */
 SAKI_API saki_status saki_recall(const saki_config* cfg, const saki_layout* layout, int64_t min_visible,
                         const void* Q, const float* A, const void* K, const int32_t* idx_approx,
                         int32_t* idx_exact, float* recall, void* workspace,
@@ -301,7 +325,10 @@ SAKI_API saki_status saki_key_spectrum(const saki_config* cfg, int64_t n_calib, 
  * 1 - sum_{i>r} sigma_i^2 / sum_i sigma_i^2 of saki_fit.
  *   Q [Hq][T][d], K [Hk][total_keys][d], sketch [Hq][total_keys][r] (dtype),
  *   A [Hq][d][d], L [Hq][d][r], nu [Hq][d] f32 or NULL, out [Hq][3] double.
- * Stream-ordered (workspace header as the selection calls). */
+ * Workspace: saki_workspace_size(SAKI_OP_SCORE_MSE) bytes, with the error-word
+ * header of the selection calls.  SAKI_ERR_INVALID_ARGUMENT for key_stride < 1,
+ * NULL out or workspace, NULL inputs when T > 0, a malformed layout or a
+ * misaligned pointer; SAKI_ERR_WORKSPACE if too small.  Stream-ordered. */
 SAKI_API saki_status saki_score_mse(const saki_config* cfg, const saki_layout* layout, int64_t key_stride,
                                     const void* Q, const float* A, const void* K, const float* L,
                                     const void* sketch, const float* nu, double* out, void* workspace,
@@ -369,7 +396,6 @@ SAKI_API saki_status saki_score_topk_noalloc(const saki_config* cfg, const saki_
  * no counterpart in the paper. */
 SAKI_API saki_status saki_noalloc_status(saki_stream stream);
 
-/* Static description of a status code. */
 /* ---------------------------------------------------------------- profiling aids
  * Not part of the method (the paper has no counterpart): a launch count and
  * per-kernel device timing, for benchmarks that report kernel-level rooflines.
@@ -405,6 +431,8 @@ SAKI_API saki_status saki_debug_inject_stall(int32_t kind);
 SAKI_API saki_status saki_kernel_timer_start(int32_t kind);
 SAKI_API saki_status saki_kernel_timer_stop(int32_t kind, double* total_ms, int64_t* launches);
 
+/* Static description of a status code (never NULL; "unknown status" for
+ * values outside saki_status). */
 SAKI_API const char* saki_status_string(saki_status status);
 
 /* Library version as "major.minor.patch". */

@@ -236,8 +236,10 @@ __global__ void __launch_bounds__(256) reconstruct_kernel(const int64_t* rows, i
   const int64_t row = blockIdx.x * 8ll + warp;
   if (row >= n_rows) return;
   const int64_t key = rows[row];
+  const bool valid = key >= 0 && key < N;   // a row outside the sketch reads nothing and comes out NaN
   float* c = cs + warp * r;
-  for (int i = lane; i < r; i += 32) c[i] = Vec<Tin>::load1(codes + ((int64_t)h * N + key) * r + i);
+  for (int i = lane; i < r; i += 32)
+    c[i] = valid ? Vec<Tin>::load1(codes + ((int64_t)h * N + key) * r + i) : __int_as_float(0x7fc00000);
   __syncwarp();
   float x[4];
 #pragma unroll
