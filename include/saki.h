@@ -277,9 +277,8 @@ SAKI_API saki_status saki_build_index(const saki_config* cfg, int64_t total_keys
  * range, q_visible beyond its sequence) or NULL / misaligned tensors;
  * SAKI_ERR_UNSUPPORTED for d != 128, k > 128, more than 65535 query heads,
  * more than 2^31 - 1 queries or a sequence of more than 2^31 - 2 keys;
- * SAKI_ERR_WORKSPACE if the
- * workspace holds neither plan.  Stream-ordered; a device timeout is read by
- * saki_workspace_status. */
+ * SAKI_ERR_WORKSPACE if the workspace holds neither plan.  Stream-ordered; a
+ * device timeout is read by saki_workspace_status. */
 SAKI_API saki_status saki_score_topk(const saki_config* cfg, const saki_layout* layout, const void* Q,
                             const float* L, const void* sketch, const float* nu, int32_t* idx,
                             float* score, void* workspace, size_t workspace_bytes,
