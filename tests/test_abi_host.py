@@ -166,3 +166,68 @@ def test_seeded_decode_reserves_the_sample_pass(lib):
     one = _layout(lib, [1 << 20], [0], [1 << 20])
     assert lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8), lib.SAKI_OP_SCORE_TOPK, one) == \
         lib.saki_workspace_size(_cfg(lib, num_q_heads=32, num_kv_heads=8, dtype="f32"), lib.SAKI_OP_SCORE_TOPK, one)
+
+
+def test_build_index_argument_checks(lib):
+    cfg = _cfg(lib)   # bf16, uncentered, r = 32, groups of 4: the tensor-core build
+    call = lambda n, mu, sk, ws, nb: lib._lib.saki_build_index(ctypes.byref(cfg), n, FAKE, FAKE, mu, sk, ws, nb, None)
+    need = lib.saki_workspace_size(cfg, lib.SAKI_OP_BUILD_INDEX, total_keys=100)
+    assert need > 256
+    assert call(100, None, None, FAKE, need) == 1        # no sketch
+    assert call(-1, None, FAKE, FAKE, need) == 1         # negative key count
+    assert call(100, None, FAKE, None, 0) == 1           # the tensor-core path needs its workspace
+    assert call(100, None, FAKE, FAKE, need - 1) == 6
+    cfg.center = 1
+    assert call(100, None, FAKE, FAKE, need) == 1        # centered keys need mu
+
+
+def test_selection_layout_and_size_limits(lib):
+    cfg = _cfg(lib)
+    call = lambda lay, ws=FAKE: lib._lib.saki_score_topk(ctypes.byref(cfg), ctypes.byref(lay.c), FAKE, FAKE, FAKE,
+                                                         None, FAKE, None, ws, 1 << 40, None)
+    bad_start = lib.HostLayout(np.array([5, 100], np.int64), [0], [3])
+    decreasing = lib.HostLayout(np.array([0, 100, 50], np.int64), [0], [3])
+    for lay in (bad_start, decreasing):
+        assert call(lay) == 1
+    huge = lib.HostLayout(np.array([0, 1 << 31], np.int64), np.zeros(0, np.int32), np.zeros(0, np.int64))
+    assert call(huge) == 2                               # a sequence beyond 2^31 - 2 keys
+    empty = _layout(lib, [100], np.zeros(0, np.int32), np.zeros(0, np.int64))
+    assert call(empty, ws=None) == 0                     # no queries: nothing to do, nothing launched
+    assert call(_layout(lib, [100], [0], [5]), ws=None) == 1   # queries need a workspace
+    assert lib._lib.saki_recall(ctypes.byref(cfg), ctypes.byref(empty.c), 65, FAKE, FAKE, FAKE, FAKE, None, FAKE,
+                                None, 1 << 40, None) == 1   # recall always needs its workspace
+    big = _cfg(lib, num_q_heads=65536 * 2, num_kv_heads=2)
+    assert lib._lib.saki_score_topk(ctypes.byref(big), ctypes.byref(empty.c), FAKE, FAKE, FAKE, None, FAKE, None,
+                                    FAKE, 1 << 40, None) == 2
+
+
+def test_score_mse_and_reconstruct_argument_checks(lib):
+    cfg = _cfg(lib)
+    lay = _layout(lib, [100], [0, 0], [10, 20])
+    mse = lambda stride, out, ws, nb: lib._lib.saki_score_mse(ctypes.byref(cfg), ctypes.byref(lay.c), stride, FAKE,
+                                                              FAKE, FAKE, FAKE, FAKE, None, out, ws, nb, None)
+    need = lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_MSE, lay)
+    assert need >= 256 + 2 * 16
+    assert mse(0, FAKE, FAKE, need) == 1
+    assert mse(1, None, FAKE, need) == 1
+    assert mse(1, FAKE, None, need) == 1
+    assert mse(1, FAKE, FAKE, need - 1) == 6
+    rec = lambda n, pos, theta, ws, nb: lib._lib.saki_reconstruct_keys(ctypes.byref(cfg), n, FAKE, 100, FAKE, FAKE,
+                                                                        None, pos, theta, FAKE, ws, nb, None)
+    assert rec(-1, None, 10000.0, None, 0) == 1
+    assert rec(4, FAKE, 1.0, FAKE, 1 << 20) == 1         # rope_theta must exceed 1
+    assert rec(4, FAKE, 10000.0, None, 0) == 1           # rotation needs its workspace
+    need = lib.saki_workspace_size(cfg, lib.SAKI_OP_RECONSTRUCT, total_keys=4)
+    assert need >= 4 * 64 * 8
+    assert rec(4, FAKE, 10000.0, FAKE, 4 * 64 * 8 - 1) == 6
+
+
+def test_merge_argument_checks(lib):
+    cfg = _cfg(lib)
+    offs = (ctypes.c_int64 * 65)(*range(0, 65 * 100, 100))
+    call = lambda parts, o: lib._lib.saki_merge_topk(ctypes.byref(cfg), parts, 4, FAKE, FAKE, o, FAKE, None, None)
+    assert call(0, offs) == 1
+    assert call(65, offs) == 2                           # at most 64 parts
+    neg = (ctypes.c_int64 * 2)(0, -5)
+    assert call(2, neg) == 1
+    assert lib.saki_status_string(99) == "unknown status"
