@@ -66,3 +66,35 @@ def test_cuda_core_peak_from_unit_counts():
     assert pk["alu_tops"] == pytest.approx(152 * 128 * pk["sm_max_mhz"] * 1e6 / 1e12)
     assert pk["fp32_tflops"] == pytest.approx(2 * pk["alu_tops"])
     assert pk["source"] in ("measured", "fallback")
+
+
+def test_clock_sampler_parses_the_query_lines(monkeypatch):
+    """The sampler reads nvidia-smi's CSV lines (fields: SM clock, max SM clock,
+    power, active reasons mask, then the four reason flags); a stand-in process
+    prints canned lines, one of them malformed."""
+    import subprocess
+    import time
+    lines = ["2070, 2070, 900.5, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+             "2055, 2070, 1350.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active",
+             "[N/A], 2070, 1000.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+             "2070, 2070, 1000.0, 0x0, Not Active, Not Active, Not Active, Not Active"]
+    script = "import time\nfor l in %r: print(l, flush=True)\ntime.sleep(60)" % (lines,)
+    real = subprocess.Popen
+    monkeypatch.setattr(bench.subprocess, "Popen", lambda cmd, **kw: real([sys.executable, "-c", script], **kw))
+    c = bench.ClockSampler(0)
+    c.start()
+    for _ in range(100):
+        if len(c.lines) >= 4:
+            break
+        time.sleep(0.05)
+    out = c.stop()
+    assert out == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+
+
+def test_clock_sampler_without_nvidia_smi(monkeypatch):
+    def missing(*a, **kw):
+        raise OSError("no nvidia-smi")
+    monkeypatch.setattr(bench.subprocess, "Popen", missing)
+    c = bench.ClockSampler(0)
+    c.start()
+    assert c.stop() == {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
