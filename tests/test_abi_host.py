@@ -231,3 +231,43 @@ def test_merge_argument_checks(lib):
     neg = (ctypes.c_int64 * 2)(0, -5)
     assert call(2, neg) == 1
     assert lib.saki_status_string(99) == "unknown status"
+
+
+def test_plain_c_program_links_and_calls_the_abi(lib, tmp_path):
+    """The boundary is usable from C without Python: a C program includes
+    saki.h, links libsaki.so, sizes workspaces and receives argument errors
+    (every call here returns before any device work)."""
+    src = tmp_path / "use.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include <stdint.h>
+#include "saki.h"
+int main(void) {
+  saki_config c = {0};
+  c.num_q_heads = 8; c.num_kv_heads = 2; c.head_dim = 128; c.rank = 32; c.topk = 64;
+  c.dtype = SAKI_BF16; c.eig_floor_rel = 1e-6f;
+  int64_t off[2] = {0, 4096};
+  int32_t qs[1] = {0};
+  int64_t qv[1] = {4096};
+  saki_layout L = {1, off, 1, qs, qv};
+  size_t fit = saki_workspace_size(&c, SAKI_OP_FIT, NULL, 16, 0);
+  size_t sel = saki_workspace_size(&c, SAKI_OP_SCORE_TOPK, &L, 0, 0);
+  c.rank = 0;
+  size_t bad = saki_workspace_size(&c, SAKI_OP_FIT, NULL, 16, 0);
+  saki_status st = saki_fit(&c, 16, NULL, NULL, NULL, NULL, NULL, NULL, NULL, NULL, NULL, NULL, 0, NULL);
+  printf("%zu %zu %zu %d %s\n", fit, sel, bad, (int)st, saki_version());
+  puts(saki_status_string(st));
+  return 0;
+}''')
+    exe = tmp_path / "use"
+    libdir = os.path.dirname(lib.library_path())
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"), str(src), "-L", libdir,
+                    "-lsaki", "-Wl,-rpath," + libdir, "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.splitlines()
+    fit, sel, bad, st, ver = out[0].split()
+    cfg = _cfg(lib)
+    assert int(fit) == lib.saki_workspace_size(cfg, lib.SAKI_OP_FIT, n_calib=16) > 0
+    lay = _layout(lib, [4096], [0], [4096])
+    assert int(sel) == lib.saki_workspace_size(cfg, lib.SAKI_OP_SCORE_TOPK, lay) > 0
+    assert int(bad) == 0 and int(st) == 1 and ver == lib.saki_version()
+    assert out[1] == "invalid argument"
